@@ -1,0 +1,164 @@
+/*
+ * dla.h -- C ABI of the GB300 (sm_103a) Dynamic Linear Attention forward path
+ * (DLA, arXiv 2606.10650).
+ *
+ * The library computes, per (batch b, head h) stream, the multi-state linear
+ * attention of the paper:
+ *   - Information-Aware Dynamic State Merging (Sec. 3.1, Algorithm 1): each
+ *     token state s_t = v_t k_t^T is scored against the most recent state S,
+ *     I_t = ||N(s_t) - N(S)||_F / (||N(S)||_F + eps) with N the whole-matrix
+ *     RMSNorm (gain 1); b_t = 1[I_t >= tau] opens a new state, otherwise the
+ *     token is added to the open state (Sec. 3.1 update rule);
+ *   - Capacity-Bounded Memory Modeling (Sec. 3.2, Algorithm 2): a
+ *     chronologically ordered cache of at most C states; before appending to a
+ *     full cache the adjacent pair i* = argmin (Ibar_i + Ibar_{i+1}) /
+ *     (n_i + n_{i+1}) is merged (S, n and Ibar summed, the rest shifted);
+ *   - the read-out (Eq. capacity_bounded_output):
+ *     o_t = sum_{i < m_t} lambda_{t,i} S_i q_t over the cache after token t.
+ *
+ * Conventions
+ *   - Every pointer argument is DEVICE memory owned by the caller, except the
+ *     dla_params / dla_cache structs themselves, which are read on the host.
+ *     The library never allocates device memory and frees nothing.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All device
+ *     work is enqueued asynchronously on it; argument errors are returned
+ *     synchronously before anything is enqueued.  A launch failure returns
+ *     DLA_ERR_CUDA.  No C++ exception crosses this interface.
+ *   - Layouts are row-major and contiguous:
+ *       q, k, v   [B, T, H, d]   (bf16 or fp32, see dla_dtype)
+ *       lambda    [B, T, H, C]   fp32, logical cache slot i = 0 is the oldest
+ *                                state; entries i >= m_t are ignored;
+ *                                NULL means every lambda is 1 (Algorithm 2's
+ *                                un-weighted sum)
+ *       o         [B, T, H, d]   fp32 or bf16 (dla_params.out_dtype)
+ *       boundary  [B, H, T]      uint8, b_t (the first token of an empty
+ *                                cache is reported as 1)
+ *       merge_log [B, H, T]      int32, i* of the merge at token t, else -1
+ *   - States are d_v x d_k matrices S = sum_s v_s k_s^T (the recurrent form of
+ *     Sec. 2), stored row-major [d_v][d_k].
+ *   - Supported: d_k = d_v = d in {64, 128}; 2 <= C <= 64; T >= 1.  Anything
+ *     else returns DLA_ERR_UNSUPPORTED (shape outside the built kernels) or
+ *     DLA_ERR_INVALID_ARG (meaningless value).
+ */
+#ifndef DLA_H
+#define DLA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DLA_VERSION 1
+
+typedef enum {
+  DLA_OK = 0,
+  DLA_ERR_INVALID_ARG = 1,  /* NULL where a pointer is required, bad value   */
+  DLA_ERR_UNSUPPORTED = 2,  /* shape/dtype outside the built kernels         */
+  DLA_ERR_WORKSPACE = 3,    /* workspace NULL or smaller than required       */
+  DLA_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed          */
+  DLA_ERR_TIMEOUT = 5,      /* a bounded device wait gave up                 */
+  DLA_ERR_DEVICE_CHECK = 6  /* a device-side consistency check failed        */
+} dla_status;
+
+typedef enum { DLA_BF16 = 0, DLA_F32 = 1 } dla_dtype;
+
+/* Method parameters (Sec. 3.1 / 3.2).  Defaults (dla_default_params): tau 0.6
+ * and capacity 30 are the paper's defaults (Sec. 4 ablation / Sec. 4.1);
+ * eps = rms_eps = 1e-6.
+ *   score_mode 0: Algorithm 1's score, token state s_t against the last state.
+ *   score_mode 1: Eq. (importance_score) read literally: N(S + s_t) against N(S).
+ *   from_cache  0: dla_forward starts from an empty cache (prefill);
+ *               1: it continues from the contents of `cache` (chunked prefill). */
+typedef struct {
+  double tau;
+  double eps;
+  double rms_eps;
+  int capacity;
+  int score_mode;
+  dla_dtype out_dtype;
+  int from_cache;
+} dla_params;
+
+/* The state cache M of Algorithm 2 for B x H streams (device memory, caller
+ * owned).  Physical slots hold the states; `slot` maps logical order (0 =
+ * oldest) to physical slots so that merges move no state data.
+ *   states [B][H][C][d_v][d_k] fp32   physical slots
+ *   slot   [B][H][C] int32           logical -> physical (a permutation of
+ *                                    0..m-1 on the first m entries)
+ *   n      [B][H][C] int32           tokens per state, logical order
+ *   ibar   [B][H][C] double          summed token scores, logical order
+ *   m      [B][H]    int32           live states (including the open one) */
+typedef struct {
+  float* states;
+  int32_t* slot;
+  int32_t* n;
+  double* ibar;
+  int32_t* m;
+  int B, H, C, dk, dv;
+} dla_cache;
+
+/* Fills *p with the defaults listed above. */
+void dla_default_params(dla_params* p);
+
+/* Bytes of one contiguous device block that dla_cache_carve can split into a
+ * cache for B x H streams (256-byte aligned sub-arrays). */
+size_t dla_cache_bytes(int B, int H, int C, int dk, int dv);
+
+/* Points the members of *out into `base` (device memory of at least
+ * dla_cache_bytes(...) bytes, 256-byte aligned).  Enqueues nothing. */
+dla_status dla_cache_carve(void* base, size_t bytes, int B, int H, int C, int dk, int dv,
+                           dla_cache* out);
+
+/* Empties every stream's cache: m = 0, slot = identity, n = 0, ibar = 0
+ * (Algorithm 2, "M <- [ ]").  State data is not cleared: slots >= m are never
+ * read. */
+dla_status dla_init_cache(const dla_cache* cache, void* stream);
+
+/* Workspace bytes dla_forward needs for these sizes.  with_output = 0 sizes it
+ * for a call with o == NULL (no read-out staging).  dla_forward accepts any
+ * workspace at least dla_forward_min_workspace(...) large and splits the
+ * sequence into more passes when it is smaller than this preferred size. */
+size_t dla_forward_workspace(const dla_params* p, int B, int T, int H, int dk, int dv,
+                             dla_dtype in_dtype, int with_output);
+size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int dk, int dv,
+                                 dla_dtype in_dtype, int with_output);
+
+/* Prefill / training-shaped forward over T tokens of B x H streams
+ * (Algorithm 1 + Algorithm 2 + Eq. capacity_bounded_output).
+ *   q, k, v, lam, o, boundary, merge_log: layouts above; o, lam, boundary and
+ *   merge_log may be NULL (lam NULL = all ones; o NULL skips the read-out).
+ *   cache: optional.  If given (dims B, H, C = p->capacity, d), it receives
+ *   the final cache; with p->from_cache = 1 it is also the starting cache.
+ *   With cache == NULL the cache lives in the workspace and from_cache must
+ *   be 0.
+ *   workspace: device memory of ws_bytes >= dla_forward_min_workspace(...). */
+dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
+                       int dv, const void* q, const void* k, const void* v, const float* lam,
+                       void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
+                       void* workspace, size_t ws_bytes, void* stream);
+
+/* One recurrent step (Sec. 3.1 inference rule + Algorithm 2 + read-out) for
+ * every stream: token (q, k, v) [B, H, d] against the persistent cache, which
+ * is updated in place.  lam [B, H, C] fp32 or NULL; o [B, H, d] (out_dtype);
+ * boundary [B, H] uint8 or NULL; merge_idx [B, H] int32 (i* or -1) or NULL.
+ * p->capacity must equal cache->C. */
+dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtype in_dtype,
+                           const void* q, const void* k, const void* v, const float* lam,
+                           void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
+
+/* Message of the last error returned on this host thread ("" if none). */
+const char* dla_last_error(void);
+
+/* Short name of a status code. */
+const char* dla_status_string(dla_status s);
+
+/* DLA_VERSION of the built library. */
+int dla_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DLA_H */

@@ -1,0 +1,327 @@
+// dla_api.cu -- extern "C" entry points of libdla.so (see include/dla.h).
+//
+// Host logic only: argument checks, workspace layout, the round schedule of
+// the forward pass and the kernel launches.  Every compute step runs in the
+// kernels of dla_scan.cu / dla_readout_*.cu / dla_decode.cu.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "dla.h"
+#include "dla_kernels.h"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+dla_status fail(dla_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+dla_status ok() {
+  g_err[0] = '\0';
+  return DLA_OK;
+}
+
+inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+struct CacheLayout {
+  size_t states, slot, n, ibar, m, total;
+};
+
+CacheLayout cache_layout(int B, int H, int C, int dk, int dv) {
+  CacheLayout L;
+  const size_t BH = (size_t)B * H;
+  size_t off = 0;
+  L.states = off; off = align256(off + BH * C * (size_t)dk * dv * sizeof(float));
+  L.slot = off;   off = align256(off + BH * C * sizeof(int32_t));
+  L.n = off;      off = align256(off + BH * C * sizeof(int32_t));
+  L.ibar = off;   off = align256(off + BH * C * sizeof(double));
+  L.m = off;      off = align256(off + BH * sizeof(int32_t));
+  L.total = off;
+  return L;
+}
+
+// Read-out interval (tokens per K2 CTA / per snapshot) of a configuration.
+int readout_interval(dla_dtype /*in_dtype*/) { return dla::kReadoutSimtInterval; }
+
+struct FwdPlan {
+  int interval;      // tokens per snapshot interval
+  int nsnap_total;   // intervals over the whole sequence
+  int R;             // intervals per round
+  int pool_cap;      // pool entries per stream per round
+  size_t off_status, off_bnd, off_mlog, off_cache, off_m0, off_ids, off_pool, total;
+};
+
+size_t pool_elt(dla_dtype in_dtype) { return in_dtype == DLA_BF16 ? 2 : 4; }
+
+FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
+                 bool with_output, bool need_trace, bool need_cache) {
+  FwdPlan P;
+  const size_t BH = (size_t)B * H;
+  const int C = p->capacity;
+  P.interval = readout_interval(in_dtype);
+  P.nsnap_total = (T + P.interval - 1) / P.interval;
+  P.R = R;
+  const int per_snap = C < P.interval + 1 ? C : P.interval + 1;
+  P.pool_cap = with_output ? C + (R - 1) * per_snap : 0;
+  size_t off = 0;
+  P.off_status = off; off = align256(off + 256);
+  P.off_bnd = off;    if (need_trace) off = align256(off + BH * T);
+  P.off_mlog = off;   if (need_trace) off = align256(off + BH * T * sizeof(int32_t));
+  P.off_cache = off;  if (need_cache) off = align256(off + cache_layout(B, H, C, d, d).total);
+  P.off_m0 = off;     if (with_output) off = align256(off + BH * R * sizeof(int32_t));
+  P.off_ids = off;    if (with_output) off = align256(off + BH * R * C * sizeof(int32_t));
+  P.off_pool = off;   if (with_output) off = align256(off + BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype));
+  P.total = off;
+  return P;
+}
+
+constexpr size_t kPreferredWorkspace = (size_t)8 << 30;  // 8 GiB of read-out staging
+
+dla_status check_params(const dla_params* p) {
+  if (!p) return fail(DLA_ERR_INVALID_ARG, "params is NULL");
+  if (!isfinite(p->tau)) return fail(DLA_ERR_INVALID_ARG, "tau must be finite");
+  if (!(p->eps >= 0.0) || !(p->rms_eps >= 0.0)) return fail(DLA_ERR_INVALID_ARG, "eps and rms_eps must be >= 0");
+  if (p->capacity < 2) return fail(DLA_ERR_INVALID_ARG, "capacity must be >= 2 (Algorithm 2 merges a pair)");
+  if (p->capacity > dla::kMaxC) return fail(DLA_ERR_UNSUPPORTED, "capacity %d > %d", p->capacity, dla::kMaxC);
+  if (p->score_mode != 0 && p->score_mode != 1) return fail(DLA_ERR_INVALID_ARG, "score_mode must be 0 or 1");
+  if (p->out_dtype != DLA_BF16 && p->out_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad out_dtype");
+  if (p->from_cache != 0 && p->from_cache != 1) return fail(DLA_ERR_INVALID_ARG, "from_cache must be 0 or 1");
+  return DLA_OK;
+}
+
+dla_status check_shape(int dk, int dv) {
+  if (dk != dv) return fail(DLA_ERR_UNSUPPORTED, "d_k (%d) != d_v (%d) is not built", dk, dv);
+  if (dk != 64 && dk != 128) return fail(DLA_ERR_UNSUPPORTED, "d = %d not built (64 or 128)", dk);
+  return DLA_OK;
+}
+
+dla_status check_cache(const dla_cache* c, int B, int H, int C, int d) {
+  if (!c->states || !c->slot || !c->n || !c->ibar || !c->m) return fail(DLA_ERR_INVALID_ARG, "cache has a NULL member");
+  if (c->B != B || c->H != H || c->C != C || c->dk != d || c->dv != d)
+    return fail(DLA_ERR_INVALID_ARG, "cache dims (B=%d H=%d C=%d dk=%d dv=%d) do not match the call (B=%d H=%d C=%d d=%d)",
+                c->B, c->H, c->C, c->dk, c->dv, B, H, C, d);
+  if (!aligned(c->states, 16) || !aligned(c->ibar, 8) || !aligned(c->slot, 4) || !aligned(c->n, 4) || !aligned(c->m, 4))
+    return fail(DLA_ERR_INVALID_ARG, "cache arrays are misaligned (states need 16 bytes)");
+  return DLA_OK;
+}
+
+dla_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(DLA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+}  // namespace
+
+extern "C" {
+
+void dla_default_params(dla_params* p) {
+  if (!p) return;
+  p->tau = 0.6;
+  p->eps = 1e-6;
+  p->rms_eps = 1e-6;
+  p->capacity = 30;
+  p->score_mode = 0;
+  p->out_dtype = DLA_F32;
+  p->from_cache = 0;
+}
+
+int dla_version(void) { return DLA_VERSION; }
+
+const char* dla_last_error(void) { return g_err; }
+
+const char* dla_status_string(dla_status s) {
+  switch (s) {
+    case DLA_OK: return "DLA_OK";
+    case DLA_ERR_INVALID_ARG: return "DLA_ERR_INVALID_ARG";
+    case DLA_ERR_UNSUPPORTED: return "DLA_ERR_UNSUPPORTED";
+    case DLA_ERR_WORKSPACE: return "DLA_ERR_WORKSPACE";
+    case DLA_ERR_CUDA: return "DLA_ERR_CUDA";
+    case DLA_ERR_TIMEOUT: return "DLA_ERR_TIMEOUT";
+    case DLA_ERR_DEVICE_CHECK: return "DLA_ERR_DEVICE_CHECK";
+  }
+  return "DLA_ERR_UNKNOWN";
+}
+
+size_t dla_cache_bytes(int B, int H, int C, int dk, int dv) {
+  if (B < 1 || H < 1 || C < 1 || dk < 1 || dv < 1) return 0;
+  return cache_layout(B, H, C, dk, dv).total;
+}
+
+dla_status dla_cache_carve(void* base, size_t bytes, int B, int H, int C, int dk, int dv, dla_cache* out) {
+  if (!base || !out) return fail(DLA_ERR_INVALID_ARG, "base and out must be non-NULL");
+  if (B < 1 || H < 1 || C < 2 || dk < 1 || dv < 1) return fail(DLA_ERR_INVALID_ARG, "bad cache dims");
+  if (!aligned(base, 256)) return fail(DLA_ERR_INVALID_ARG, "cache base must be 256-byte aligned");
+  CacheLayout L = cache_layout(B, H, C, dk, dv);
+  if (bytes < L.total) return fail(DLA_ERR_WORKSPACE, "cache block has %zu bytes, needs %zu", bytes, L.total);
+  char* c = (char*)base;
+  out->states = (float*)(c + L.states);
+  out->slot = (int32_t*)(c + L.slot);
+  out->n = (int32_t*)(c + L.n);
+  out->ibar = (double*)(c + L.ibar);
+  out->m = (int32_t*)(c + L.m);
+  out->B = B; out->H = H; out->C = C; out->dk = dk; out->dv = dv;
+  return ok();
+}
+
+dla_status dla_init_cache(const dla_cache* cache, void* stream) {
+  if (!cache) return fail(DLA_ERR_INVALID_ARG, "cache is NULL");
+  if (cache->B < 1 || cache->H < 1 || cache->C < 2) return fail(DLA_ERR_INVALID_ARG, "bad cache dims");
+  if (!cache->slot || !cache->n || !cache->ibar || !cache->m) return fail(DLA_ERR_INVALID_ARG, "cache has a NULL member");
+  cudaError_t e = dla::launch_init_cache(cache->slot, cache->n, cache->ibar, cache->m, cache->B * cache->H, cache->C,
+                                         (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
+  return ok();
+}
+
+static FwdPlan choose_plan(const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype, bool with_output,
+                           bool need_trace, bool need_cache, size_t budget) {
+  const int nsnap = (T + readout_interval(in_dtype) - 1) / readout_interval(in_dtype);
+  if (!with_output) return plan_for(1, p, B, T, H, d, in_dtype, false, need_trace, need_cache);
+  int lo = 1, hi = nsnap;
+  FwdPlan best = plan_for(1, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
+  if (best.total > budget) return best;
+  while (lo < hi) {  // largest R whose workspace fits the budget
+    int mid = lo + (hi - lo + 1) / 2;
+    if (plan_for(mid, p, B, T, H, d, in_dtype, true, need_trace, need_cache).total <= budget) lo = mid;
+    else hi = mid - 1;
+  }
+  return plan_for(lo, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
+}
+
+size_t dla_forward_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype,
+                             int with_output) {
+  if (!p || B < 1 || T < 1 || H < 1 || dk < 1 || dv < 1) return 0;
+  // sized for the worst case of the call: trace and cache held in the workspace
+  return choose_plan(p, B, T, H, dk, in_dtype, with_output != 0, true, true, kPreferredWorkspace).total;
+}
+
+size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype,
+                                 int with_output) {
+  if (!p || B < 1 || T < 1 || H < 1 || dk < 1 || dv < 1) return 0;
+  return plan_for(1, p, B, T, H, dk, in_dtype, with_output != 0, true, true).total;
+}
+
+dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv, const void* q,
+                       const void* k, const void* v, const float* lam, void* o, const dla_cache* cache,
+                       uint8_t* boundary, int32_t* merge_log, void* workspace, size_t ws_bytes, void* stream) {
+  dla_status s = check_params(p);
+  if (s != DLA_OK) return s;
+  if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
+  if (B < 1 || T < 1 || H < 1) return fail(DLA_ERR_INVALID_ARG, "B, T, H must be >= 1");
+  if ((s = check_shape(dk, dv)) != DLA_OK) return s;
+  const int d = dk, C = p->capacity;
+  if ((long long)B * T * H * d >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
+  if (!k || !v) return fail(DLA_ERR_INVALID_ARG, "k and v must be non-NULL");
+  const bool with_output = (o != nullptr);
+  if (with_output && !q) return fail(DLA_ERR_INVALID_ARG, "q must be non-NULL when o is requested");
+  const size_t vec = 16;
+  if (!aligned(k, vec) || !aligned(v, vec) || (q && !aligned(q, vec)) || (o && !aligned(o, vec)))
+    return fail(DLA_ERR_INVALID_ARG, "q, k, v, o must be 16-byte aligned");
+  if (lam && !aligned(lam, 4)) return fail(DLA_ERR_INVALID_ARG, "lambda must be 4-byte aligned");
+  if (cache) {
+    if ((s = check_cache(cache, B, H, C, d)) != DLA_OK) return s;
+  } else if (p->from_cache) {
+    return fail(DLA_ERR_INVALID_ARG, "from_cache = 1 needs a cache");
+  }
+  if (!workspace) return fail(DLA_ERR_WORKSPACE, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(DLA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const bool need_trace = (boundary == nullptr) || (merge_log == nullptr);
+  const bool need_cache = (cache == nullptr);
+  FwdPlan P = choose_plan(p, B, T, H, d, in_dtype, with_output, need_trace, need_cache, ws_bytes);
+  if (P.total > ws_bytes)
+    return fail(DLA_ERR_WORKSPACE, "workspace has %zu bytes, needs at least %zu", ws_bytes, P.total);
+
+  cudaStream_t st = (cudaStream_t)stream;
+  char* ws = (char*)workspace;
+  int32_t* status = (int32_t*)(ws + P.off_status);
+  uint8_t* bnd = boundary ? boundary : (uint8_t*)(ws + P.off_bnd);
+  int32_t* mlog = merge_log ? merge_log : (int32_t*)(ws + P.off_mlog);
+  dla_cache live;
+  if (cache) {
+    live = *cache;
+  } else {
+    dla_cache_carve(ws + P.off_cache, cache_layout(B, H, C, d, d).total, B, H, C, d, d, &live);
+  }
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);
+  if (e != cudaSuccess) return cuda_fail(e, "status reset");
+  if (!p->from_cache) {
+    e = dla::launch_init_cache(live.slot, live.n, live.ibar, live.m, B * H, C, st);
+    if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
+  }
+
+  dla::ScanArgs sa;
+  memset(&sa, 0, sizeof(sa));
+  sa.k = k; sa.v = v;
+  sa.B = B; sa.T = T; sa.H = H;
+  sa.sp.tau = p->tau; sa.sp.eps = p->eps; sa.sp.rms_eps = p->rms_eps; sa.sp.score_mode = p->score_mode;
+  sa.C = C;
+  sa.states = live.states; sa.slot = live.slot; sa.n = live.n; sa.ibar = live.ibar; sa.m = live.m;
+  sa.boundary = bnd; sa.merge_log = mlog;
+  sa.status = status;
+  const bool in_bf16 = (in_dtype == DLA_BF16);
+  const bool pool_bf16 = in_bf16;
+  if (!with_output) {
+    sa.t_begin = 0; sa.t_end = T;
+    sa.pool = nullptr; sa.pool_cap = 0; sa.nsnap = 1; sa.snap_chunks = 1;
+    e = dla::launch_scan(sa, d, in_bf16, pool_bf16, st);
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    return ok();
+  }
+  dla::ReadoutArgs ra;
+  memset(&ra, 0, sizeof(ra));
+  ra.q = q; ra.k = k; ra.v = v; ra.lam = lam; ra.o = o;
+  ra.out_bf16 = (p->out_dtype == DLA_BF16);
+  ra.B = B; ra.T = T; ra.H = H; ra.C = C;
+  ra.boundary = bnd; ra.merge_log = mlog;
+  ra.interval = P.interval;
+  sa.pool = ws + P.off_pool; sa.pool_cap = P.pool_cap;
+  sa.snap_m0 = (int32_t*)(ws + P.off_m0); sa.snap_ids = (int32_t*)(ws + P.off_ids);
+  sa.snap_chunks = P.interval / dla::kScanL;
+  ra.pool = sa.pool; ra.pool_cap = sa.pool_cap; ra.snap_m0 = sa.snap_m0; ra.snap_ids = sa.snap_ids;
+  const int round_tokens = P.R * P.interval;
+  for (int t0 = 0; t0 < T; t0 += round_tokens) {
+    const int t1 = (T - t0 < round_tokens) ? T : t0 + round_tokens;
+    sa.t_begin = t0; sa.t_end = t1;
+    sa.nsnap = (t1 - t0 + P.interval - 1) / P.interval;
+    e = dla::launch_scan(sa, d, in_bf16, pool_bf16, st);
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
+    e = dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st);
+    if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+  }
+  return ok();
+}
+
+dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtype in_dtype, const void* q,
+                           const void* k, const void* v, const float* lam, void* o, uint8_t* boundary,
+                           int32_t* merge_idx, void* stream) {
+  dla_status s = check_params(p);
+  if (s != DLA_OK) return s;
+  if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
+  if (!cache) return fail(DLA_ERR_INVALID_ARG, "cache is NULL");
+  if ((s = check_shape(cache->dk, cache->dv)) != DLA_OK) return s;
+  if ((s = check_cache(cache, cache->B, cache->H, p->capacity, cache->dk)) != DLA_OK) return s;
+  if (!q || !k || !v || !o) return fail(DLA_ERR_INVALID_ARG, "q, k, v and o must be non-NULL");
+  if (lam && !aligned(lam, 4)) return fail(DLA_ERR_INVALID_ARG, "lambda must be 4-byte aligned");
+  dla::DecodeArgs da;
+  memset(&da, 0, sizeof(da));
+  da.q = q; da.k = k; da.v = v; da.lam = lam; da.o = o;
+  da.out_bf16 = (p->out_dtype == DLA_BF16);
+  da.B = cache->B; da.H = cache->H; da.C = cache->C;
+  da.sp.tau = p->tau; da.sp.eps = p->eps; da.sp.rms_eps = p->rms_eps; da.sp.score_mode = p->score_mode;
+  da.states = cache->states; da.slot = cache->slot; da.n = cache->n; da.ibar = cache->ibar; da.m = cache->m;
+  da.boundary = boundary; da.merge_idx = merge_idx;
+  cudaError_t e = dla::launch_decode(da, cache->dk, in_dtype == DLA_BF16, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,118 @@
+// dla_common.cuh -- shared device helpers of the DLA sm_103a kernels.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dla_kernels.h"
+
+namespace dla {
+
+// State Information Score from three scalars of the token state s = v k^T
+// and the open state S (Sec. 3.1 / Algorithm 1 with the whole-matrix RMSNorm
+// N(X) = X / sqrt(||X||^2 / D + rms_eps)):
+//   a = ||s||^2 = ||k||^2 ||v||^2,  beta = <s, S> = v^T S k,  gam = ||S||^2.
+// Mode 0 compares N(s) with N(S) (Algorithm 1); mode 1 compares N(S + s)
+// with N(S) (Eq. importance_score read literally).  Since
+// ||N(A) - N(B)||^2 = |A|^2/ra^2 + |B|^2/rb^2 - 2<A,B>/(ra rb), the score
+// needs no d x d work once a, beta, gam are known.
+__device__ __forceinline__ double info_score(double a, double beta, double gam, double D,
+                                             const ScoreParams& p) {
+  double AA, BB, AB;
+  if (p.score_mode == 1) {
+    AA = gam + 2.0 * beta + a;
+    BB = gam;
+    AB = gam + beta;
+  } else {
+    AA = a;
+    BB = gam;
+    AB = beta;
+  }
+  AA = fmax(AA, 0.0);
+  BB = fmax(BB, 0.0);
+  double ra = sqrt(AA / D + p.rms_eps);
+  double rb = sqrt(BB / D + p.rms_eps);
+  double num2 = AA / (ra * ra) + BB / (rb * rb) - 2.0 * AB / (ra * rb);
+  double num = sqrt(fmax(num2, 0.0));
+  double den = sqrt(BB) / rb + p.eps;
+  return num / den;
+}
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T x);
+template <>
+__device__ __forceinline__ float to_f32<float>(float x) { return x; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float x);
+template <>
+__device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
+
+// Loads 4 consecutive elements (16-byte aligned for fp32, 8-byte for bf16) as floats.
+__device__ __forceinline__ float4 load4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 load4(const __nv_bfloat16* p) {
+  uint2 u = *reinterpret_cast<const uint2*>(p);
+  __nv_bfloat162 a = *reinterpret_cast<__nv_bfloat162*>(&u.x);
+  __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162*>(&u.y);
+  float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+  return make_float4(fa.x, fa.y, fb.x, fb.y);
+}
+
+__device__ __forceinline__ void store4(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+__device__ __forceinline__ void store4(__nv_bfloat16* p, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y);
+  __nv_bfloat162 b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Warp argmin over (value, index) pairs; lowest index wins exact ties.
+__device__ __forceinline__ void warp_argmin(double& v, int& i) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    double ov = __shfl_xor_sync(0xffffffffu, v, o);
+    int oi = __shfl_xor_sync(0xffffffffu, i, o);
+    if (ov < v || (ov == v && oi < i)) {
+      v = ov;
+      i = oi;
+    }
+  }
+}
+
+// Adjacent-pair argmin of Algorithm 2 over logical entries 0..m-1 (m >= 2):
+// i* = argmin_i (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}), lowest i on ties.
+// Called by one full warp; every lane returns i*.
+__device__ __forceinline__ int pair_argmin_warp(const int* n, const double* ibar, int m) {
+  const int lane = threadIdx.x & 31;
+  double best = 1.0 / 0.0;
+  int bi = 0x7fffffff;
+  for (int i = lane; i + 1 < m; i += 32) {
+    double dens = (ibar[i] + ibar[i + 1]) / (double)(n[i] + n[i + 1]);
+    if (dens < best) {
+      best = dens;
+      bi = i;
+    }
+  }
+  warp_argmin(best, bi);
+  return bi;
+}
+
+}  // namespace dla

@@ -1,0 +1,94 @@
+// dla_kernels.h -- internal launch interface between the C ABI (dla_api.cu)
+// and the kernels.  Not part of the public header.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace dla {
+
+constexpr int kMaxC = 64;   // largest supported capacity C
+constexpr int kScanL = 64;  // tokens per scan chunk (K1)
+
+// Method parameters of the score / boundary test (Sec. 3.1).
+struct ScoreParams {
+  double tau, eps, rms_eps;
+  int score_mode;
+};
+
+// K1: sequential scan of one round [t_begin, t_end) of every stream.
+struct ScanArgs {
+  const void* k;
+  const void* v;
+  int B, T, H;
+  int t_begin, t_end;
+  ScoreParams sp;
+  int C;
+  // live cache (fp32 states in physical slots, logical metadata)
+  float* states;
+  int32_t* slot;
+  int32_t* n;
+  double* ibar;
+  int32_t* m;
+  // per-token trace [B, H, T]
+  uint8_t* boundary;
+  int32_t* merge_log;
+  // read-out snapshots (pool == nullptr: no read-out in this call)
+  void* pool;
+  int pool_cap;          // entries per stream
+  int32_t* snap_m0;      // [B*H][nsnap]
+  int32_t* snap_ids;     // [B*H][nsnap][C]
+  int nsnap;             // snapshot intervals in this round
+  int snap_chunks;       // scan chunks per snapshot interval
+  int32_t* status;       // device status word (0 = ok)
+};
+
+// K2: read-out of one round, one CTA per (snapshot interval, stream).
+struct ReadoutArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const float* lam;      // [B, T, H, C] or nullptr
+  void* o;               // [B, T, H, d]
+  int out_bf16;
+  int B, T, H, C;
+  int t_begin, t_end;
+  const uint8_t* boundary;
+  const int32_t* merge_log;
+  const void* pool;
+  int pool_cap;
+  const int32_t* snap_m0;
+  const int32_t* snap_ids;
+  int nsnap;
+  int interval;          // tokens per snapshot interval
+};
+
+// K3: one decode step of every stream.
+struct DecodeArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const float* lam;      // [B, H, C] or nullptr
+  void* o;               // [B, H, d]
+  int out_bf16;
+  int B, H, C;
+  ScoreParams sp;
+  float* states;
+  int32_t* slot;
+  int32_t* n;
+  double* ibar;
+  int32_t* m;
+  uint8_t* boundary;     // [B, H] or nullptr
+  int32_t* merge_idx;    // [B, H] or nullptr
+};
+
+cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
+size_t scan_smem_bytes(int d);
+cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
+constexpr int kReadoutSimtInterval = 64;
+cudaError_t launch_decode(const DecodeArgs& a, int d, bool in_bf16, cudaStream_t s);
+cudaError_t launch_init_cache(int32_t* slot, int32_t* n, double* ibar, int32_t* m, int BH, int C,
+                              cudaStream_t s);
+
+}  // namespace dla

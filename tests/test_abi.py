@@ -1,0 +1,80 @@
+"""Host-side checks of the C ABI: the library builds, loads and exports every
+entry point include/dla.h declares, and argument errors come back as status
+codes before anything touches a GPU (no compute calls here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import __graft_entry__
+from paper_2606_10650_gb300 import dla
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    __graft_entry__.build()
+    return dla.lib()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "dla.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dla_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ["dla_forward", "dla_decode_step", "dla_init_cache", "dla_forward_workspace", "dla_cache_bytes"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for n in _declared():
+        assert hasattr(L, n), n
+    assert set(_declared()) == set(dla.EXPORTED)
+    assert L.dla_version() == 1
+
+
+def _fake(addr=1 << 20):
+    return ctypes.c_void_p(addr)
+
+
+def _fwd(L, p, dt=dla.DLA_BF16, B=1, T=64, H=2, d=128, k=True, ws_bytes=1 << 40, ws=True, o=True):
+    return L.dla_forward(ctypes.byref(p), dt, B, T, H, d, d, _fake(), _fake() if k else None, _fake(), None,
+                         _fake() if o else None, None, None, None, _fake(1 << 24) if ws else None, ws_bytes, None)
+
+
+def test_argument_errors_return_status_codes(L):
+    p = dla.make_params(0.6, 8)
+    assert _fwd(L, dla.make_params(0.6, 1)) == 1          # C < 2: Algorithm 2 needs a pair
+    assert _fwd(L, dla.make_params(0.6, 65)) == 2         # beyond the built capacity
+    assert _fwd(L, dla.make_params(float("nan"), 8)) == 1
+    assert _fwd(L, dla.make_params(0.6, 8, score_mode=3)) == 1
+    assert _fwd(L, p, d=96) == 2
+    assert _fwd(L, p, k=False) == 1
+    assert _fwd(L, p, B=0) == 1
+    assert _fwd(L, p, ws=False) == 3
+    assert _fwd(L, p, ws_bytes=1024) == 3
+    assert b"workspace" in L.dla_last_error()
+    assert L.dla_status_string(3) == b"DLA_ERR_WORKSPACE"
+
+
+def test_workspace_sizes_are_monotone(L):
+    p = dla.make_params(0.6, 32)
+    full = L.dla_forward_workspace(ctypes.byref(p), 2, 16384, 16, 128, 128, 0, 1)
+    mini = L.dla_forward_min_workspace(ctypes.byref(p), 2, 16384, 16, 128, 128, 0, 1)
+    none = L.dla_forward_workspace(ctypes.byref(p), 2, 16384, 16, 128, 128, 0, 0)
+    assert 0 < none < mini <= full
+
+
+def test_cache_carve_layout(L):
+    nb = L.dla_cache_bytes(2, 3, 4, 64, 64)
+    assert nb >= 2 * 3 * 4 * 64 * 64 * 4
+    c = dla.dla_cache()
+    assert L.dla_cache_carve(_fake(1 << 30), nb, 2, 3, 4, 64, 64, ctypes.byref(c)) == 0
+    assert c.states == 1 << 30 and c.C == 4
+    assert all(getattr(c, f) % 256 == 0 for f in ("states", "slot", "n", "ibar", "m"))
+    assert L.dla_cache_carve(_fake(1 << 30), nb - 1, 2, 3, 4, 64, 64, ctypes.byref(c)) == 3

@@ -1,0 +1,169 @@
+"""GPU parity of the CUDA path (through the C ABI) against the fp64 oracle on
+decision-safe seeded inputs, at sizes where the oracle checks every stream,
+token and state.  Sizes span several scan chunks / read-out intervals and a
+ragged tail."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_10650_gb300 import dla
+from paper_2606_10650_gb300 import workloads as W
+from parity_util import TOL, compare, run_gpu, run_oracle, structural_checks, upload
+from safe_inputs import safe_batch, safe_stream
+
+pytestmark = pytest.mark.gpu
+
+
+def _safe(w, T=None, seed=None, score_mode=0):
+    T = w.total_tokens if T is None else T
+    q, k, v, lam = W.host_batch(w, seed=seed, T=T)
+    for b in range(w.B):
+        for h in range(w.H):
+            r = safe_stream(w, b, h, T=T, seed=seed, score_mode=score_mode)
+            q[b, :, h], k[b, :, h], v[b, :, h], lam[b, :, h] = r["q"], r["k"], r["v"], r["lam"]
+    return q, k, v, lam
+
+
+CASES = {
+    # name: (workload, overrides)
+    "tiny_fp32": ("tiny", dict()),
+    "standard_bf16": ("standard", dict(B=1, H=3, T=1000)),
+    "regime_bf16": ("regime", dict(B=1, H=2, T=2500)),
+    "long_churn_bf16": ("long", dict(B=1, H=2, T=1500, block=256)),
+    "d64_bf16": ("standard", dict(B=2, H=2, T=700, d=64, C=8, tau=1.4215)),
+    "d128_fp32": ("tiny", dict(B=1, H=2, T=300, d=128, C=6, tau=1.4142)),
+}
+
+
+@pytest.mark.parametrize("case", list(CASES))
+def test_forward_parity(case):
+    name, ov = CASES[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    r = run_oracle(w, q, k, v, lam)
+    rep = {}
+    compare(w, g, r, report=rep)
+    structural_checks(w, g, w.T)
+    assert g["boundary"].sum() > 2
+    print(case, rep)
+
+
+def test_merges_are_exercised():
+    """The small cases above do merge (the fixtures are not vacuous)."""
+    w = W.get("long", B=1, H=1, T=1200, block=256)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    assert (g["merge_log"] >= 0).sum() > 100
+
+
+def test_lambda_null_is_causal_linear_attention():
+    """lambda = NULL (all ones): merges only regroup sums, so o must be causal
+    linear attention (Eq. linear_attn_parallel), whatever the decisions."""
+    w = W.get("standard", B=1, H=2, T=777)
+    q, k, v, _ = W.host_batch(w, T=w.T)
+    g = run_gpu(w, q, k, v, None)
+    for h in range(w.H):
+        Q, K, V = q[0, :, h], k[0, :, h], v[0, :, h]
+        O = np.tril(Q @ K.T) @ V
+        assert np.abs(g["o"][0, :, h] - O).max() <= TOL["bf16"]
+
+
+def test_score_mode_literal_equation():
+    """score_mode 1 (Eq. importance_score with S_t = S_{t-1} + s_t)."""
+    w0 = W.get("tiny", T=400)
+    q, k, v, lam = W.host_batch(w0, T=w0.T)
+    st = oracle.Stream(w0.C, w0.d, w0.d, 1e300, score_mode=1)
+    _, _, _, it = st.run(q[0, :, 0], k[0, :, 0], v[0, :, 0])
+    w = dataclasses.replace(w0, tau=float(np.quantile(it[1:], 0.8)))
+    q, k, v, lam = _safe(w, score_mode=1)
+    g = run_gpu(w, q, k, v, lam, score_mode=1)
+    r = run_oracle(w, q, k, v, lam, score_mode=1)
+    compare(w, g, r)
+    assert g["boundary"].sum() > 10
+
+
+def test_bf16_output_dtype():
+    w = W.get("standard", B=1, H=2, T=300)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam, out_dtype=torch.bfloat16)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r, tol=TOL["bf16"] + 2.0 ** -8 * np.abs(r["o"]).max())
+
+
+@pytest.mark.parametrize("T", [1, 2, 63, 64, 65, 129])
+def test_edge_lengths(T):
+    w = W.get("tiny", T=T, C=3)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+    assert g["boundary"][0, 0, 0] == 1
+
+
+def test_many_rounds_small_workspace():
+    """The smallest workspace forces one read-out interval per round; the
+    result must not change."""
+    w = W.get("regime", B=1, H=2, T=1100)
+    q, k, v, lam = _safe(w)
+    p = dla.make_params(w.tau, w.C)
+    nb = dla.dla_forward_min_workspace(p, w.B, w.T, w.H, w.d, w.d, dla.DLA_BF16, True)
+    g = run_gpu(w, q, k, v, lam, ws_bytes=nb)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+
+
+def test_prefill_continuation_from_cache():
+    """forward(T0) then forward(T - T0) from the cache equals forward(T)."""
+    w = W.get("regime", B=1, H=2, T=1300)
+    q, k, v, lam = _safe(w)
+    T0 = 517
+    r = run_oracle(w, q, k, v, lam)
+    wa = dataclasses.replace(w, T=T0)
+    ga = run_gpu(wa, q[:, :T0], k[:, :T0], v[:, :T0], lam[:, :T0])
+    wb = dataclasses.replace(w, T=w.T - T0)
+    gb = run_gpu(wb, q[:, T0:], k[:, T0:], v[:, T0:], lam[:, T0:], cache=ga["cache"], from_cache=True)
+    bnd = np.concatenate([ga["boundary"], gb["boundary"]], axis=2)
+    ml = np.concatenate([ga["merge_log"], gb["merge_log"]], axis=2)
+    o = np.concatenate([ga["o"], gb["o"]], axis=1)
+    g = dict(boundary=bnd, merge_log=ml, o=o, cache=gb["cache"])
+    compare(w, g, r)
+
+
+def test_decode_steps_match_prefill():
+    """dla_forward over T0 tokens, then one dla_decode_step per token, equals
+    the oracle over all T tokens (Sec. 3.1 inference rule is the same
+    recurrence)."""
+    w = W.get("decode", B=3, H=2, T=300, decode_steps=90, C=16)
+    Ttot = w.total_tokens
+    q, k, v, lam = _safe(w, T=Ttot)
+    r = run_oracle(w, q, k, v, lam)
+    wp = dataclasses.replace(w, decode_steps=0)
+    gp = run_gpu(wp, q[:, :w.T], k[:, :w.T], v[:, :w.T], lam[:, :w.T], want_o=False)
+    cache = gp["cache"]
+    dev = torch.device("cuda:0")
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    o_all = np.zeros((w.B, w.decode_steps, w.H, w.d))
+    b_all = np.zeros((w.B, w.H, w.decode_steps), np.uint8)
+    m_all = np.zeros((w.B, w.H, w.decode_steps), np.int32)
+    for s in range(w.decode_steps):
+        t = w.T + s
+        qt, kt, vt, lt = upload(w, q[:, t], k[:, t], v[:, t], lam[:, t])
+        o = torch.empty((w.B, w.H, w.d), dtype=torch.float32, device=dev)
+        bb = torch.empty((w.B, w.H), dtype=torch.uint8, device=dev)
+        mi = torch.empty((w.B, w.H), dtype=torch.int32, device=dev)
+        dla.dla_decode_step(p, cache, qt.contiguous(), kt.contiguous(), vt.contiguous(), lt.contiguous(), o, bb, mi)
+        o_all[:, s] = o.double().cpu().numpy()
+        b_all[:, :, s] = bb.cpu().numpy()
+        m_all[:, :, s] = mi.cpu().numpy()
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(gp["boundary"], r["boundary"][:, :, :w.T])
+    np.testing.assert_array_equal(b_all, r["boundary"][:, :, w.T:])
+    np.testing.assert_array_equal(m_all, r["merge_log"][:, :, w.T:])
+    assert np.abs(o_all - r["o"][:, w.T:]).max() <= TOL["bf16"]
+    g = dict(boundary=r["boundary"], merge_log=r["merge_log"], o=None, cache=cache)
+    compare(w, g, r)
+    assert b_all.sum() > 0 and (m_all >= 0).sum() > 0
