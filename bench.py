@@ -1,0 +1,479 @@
+#!/usr/bin/env python3
+"""Throughput of the GB300 DLA forward path (one JSON line on stdout).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dla|reference]
+
+Headline: prefill tokens/s of the regime-shift workload (B=2, H=16, T=16384,
+d=128, C=32, bf16 inputs, fp32 states) -- one step is one dla_forward call
+over the whole batch (scan, snapshots, read-out), inputs resident in HBM.
+The same line carries the decode workload (256 sequences x 32 heads, d=128,
+C=64, fp32 cache pre-filled by an 8K-token prefill; one step is one
+dla_decode_step for every stream), the roofline of the dominant kernel of
+each (CUDA events on the library's stream), the end-to-end figure through the
+public API with host buffers, and the fp64 oracle timed on the host cores
+(cpu_baseline).  The path shards by independent (batch, head) streams, so
+N > 1 runs N independent replicas (weak scaling, no collective on the data
+path).  ``--impl reference`` times the oracle instead (the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+PREFILL_METRIC = "DLA tokens/sec (prefill, T=16K, C=32)"
+DECODE_METRIC = "DLA decode tokens/sec"
+FP32_LANES_PER_SM = 128  # FFMA lanes per SM (Blackwell)
+
+
+# ---------------------------------------------------------------- helpers
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sustained=float(p["bf16_tflops_sustained"]), sm_max_mhz=float(p.get("sm_max_mhz", 2070.0)),
+                    source="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, sm_max_mhz=2070.0, source="fallback")
+
+
+class Dist:
+    def __init__(self):
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch
+            import torch.distributed as dist
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def reduce(self, x, op):
+        if not self.pg:
+            return x
+        import torch
+        dev = torch.device("cuda", self.local) if torch.cuda.is_available() else torch.device("cpu")
+        t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX if op == "max" else self.pg.ReduceOp.SUM)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+class Clocks:
+    """nvidia-smi sampling (200 ms) around a timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="dla_clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 10:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return float("nan")
+
+        loaded = [r for r in rows if num(r[4]) > 0] or rows
+        sm = [num(r[1]) for r in loaded]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in loaded for i in range(4) if r[6 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(num(r[2]) for r in rows),
+                "power_w_max": max(num(r[3]) for r in rows), "samples": len(rows), "samples_under_load": len(loaded),
+                "reasons": reasons}
+
+
+def kernel_table(timing, steps):
+    total = sum(ms for _, ms in timing.values()) or 1.0
+    return {k: {"launches": n, "ms_total": round(ms, 4), "ms_per_launch": round(ms / n, 5) if n else None,
+                "share": round(ms / total, 4)} for k, (n, ms) in timing.items() if n}
+
+
+# ---------------------------------------------------------------- prefill
+
+def bench_prefill(args, dist, pk):
+    import numpy as np
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+    from paper_2606_10650_gb300 import workloads as W
+
+    dev = torch.device("cuda", dist.local)
+    torch.cuda.set_device(dev)
+    w = W.get(args.workload)
+    if args.T:
+        w = W.get(args.workload, T=args.T)
+    q, k, v, lam = W.host_batch(w, T=w.T)
+    qt, kt, vt = (W.to_device(x, w.dtype, dev) for x in (q, k, v))
+    lt = torch.from_numpy(lam.astype(np.float32)).to(dev)
+    B, T, H, d = kt.shape
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    in_code = dla.DLA_BF16 if w.dtype == "bf16" else dla.DLA_F32
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    o = torch.empty((B, T, H, d), dtype=torch.float32, device=dev)
+    bnd = torch.empty((B, H, T), dtype=torch.uint8, device=dev)
+    ml = torch.empty((B, H, T), dtype=torch.int32, device=dev)
+    nb = dla.dla_forward_workspace(p, B, T, H, d, d, in_code, True)
+    buf = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    ws = (buf, (buf.data_ptr() + 255) // 256 * 256, nb)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        dla.dla_forward(p, qt, kt, vt, lt, o, cache, bnd, ml, workspace=ws, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    dla.dla_timing_read(reset=True)
+    clocks = Clocks(dist.local)
+    clocks.start()
+    dist.barrier()
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(False)
+    dist.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    timing = dla.dla_timing_read(reset=True)
+    ms_max = dist.reduce(ms, "max")
+    tokens = B * T
+    # algorithmic work from the decision trace: m_t = live states after token t
+    m_t = torch.cumsum(bnd.to(torch.int64), 2) - torch.cumsum((ml >= 0).to(torch.int64), 2)
+    sum_m = int(m_t.sum().item())
+    BH = B * H
+    flops_readout = 2.0 * d * d * sum_m
+    flops_total = 2.0 * d * d * (sum_m + 2 * T * BH)
+    kt_tab = kernel_table(timing, args.steps)
+    ro_n, ro_ms = timing["readout"]
+    fp32_peak = pk_fp32(pk)
+    # flops_readout is per step; the launches of a step share it
+    achieved = flops_readout * args.steps / (ro_ms * 1e-3) / 1e12 if ro_n else None
+    roof = {"kernel": "readout", "bound": "alu", "achieved": round(achieved, 3) if achieved else None,
+            "peak": round(fp32_peak, 2), "unit": "TFLOP/s",
+            "frac": round(achieved / fp32_peak, 4) if achieved else None, "traffic": None,
+            "peak_note": "fp32 FFMA peak: 152 SMs x 128 lanes x 2 flop x sm_max_mhz of MEASURED_PEAKS.json",
+            "work_per_launch": f"2*d^2*sum_t m_t / launches per step = "
+                               f"{flops_readout * args.steps / max(1, ro_n):.4g} flop"}
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        qh, kh, vh = (x.cpu().pin_memory() for x in (qt, kt, vt))
+        lh = lt.cpu().pin_memory()
+        oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+        n_e2e = max(2, min(args.steps, 10))
+
+        def e2e_step():
+            qt.copy_(qh, non_blocking=True)
+            kt.copy_(kh, non_blocking=True)
+            vt.copy_(vh, non_blocking=True)
+            lt.copy_(lh, non_blocking=True)
+            step()
+            oh.copy_(o, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        dist.barrier()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = dist.reduce(a0.elapsed_time(a1) / n_e2e, "max")
+        hb = sum(x.numel() * x.element_size() for x in (qh, kh, vh, lh))
+        e2e = {"value": round(dist.world * tokens / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
+               "h2d_bytes_per_step": hb, "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e}
+    res = {"value": dist.world * tokens / (ms_max * 1e-3), "ms_per_step": ms_max, "tokens_per_step": tokens,
+           "roofline": roof, "kernels": kt_tab, "clocks": clk, "e2e": e2e,
+           "gpu_launches": sum(n for n, _ in timing.values()),
+           "algorithmic_tflops": flops_total / (ms_max * 1e-3) / 1e12, "sum_m": sum_m,
+           "boundaries": int(bnd.sum().item()), "merges": int((ml >= 0).sum().item())}
+    del qt, kt, vt, lt, o, buf, cache
+    torch.cuda.empty_cache()
+    return res
+
+
+def pk_fp32(pk):
+    return 152 * FP32_LANES_PER_SM * 2 * pk["sm_max_mhz"] * 1e6 / 1e12
+
+
+# ---------------------------------------------------------------- decode
+
+def bench_decode(args, dist, pk):
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+    from paper_2606_10650_gb300 import workloads as W
+
+    dev = torch.device("cuda", dist.local)
+    w = W.get("decode")
+    B, H, d, C, Tp = w.B, w.H, w.d, w.C, w.T
+    if args.decode_batch:
+        B = args.decode_batch
+    p = dla.make_params(w.tau, C, w.eps, w.rms_eps)
+    cache = dla.Cache(B, H, C, d, device=dev)
+    gb = 32 if B % 32 == 0 else B
+    nb = dla.dla_forward_workspace(p, gb, Tp, H, d, d, dla.DLA_BF16, False)
+    buf = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    ws = (buf, (buf.data_ptr() + 255) // 256 * 256, nb)
+    t0 = time.time()
+    for g in range(B // gb):  # seeded 8K-token prefill, 32 sequences at a time, scan only (o = NULL)
+        _, kk, vv, _ = W.device_iid_batch(w, gb, Tp, seed=w.seed * 1000 + g, device=dev, with_lam=False)
+        dla.dla_forward(p, None, kk, vv, None, None, cache.sub(g * gb, gb), None, None, workspace=ws)
+        del kk, vv
+    torch.cuda.synchronize()
+    prefill_s = time.time() - t0
+    del buf
+    nsteps = args.warmup + args.steps
+    wd = W.get("decode", B=B)
+    qs, ks, vs, ls = W.device_decode_steps(wd, nsteps, seed=w.seed * 1000 + 999, device=dev)
+    o = torch.empty((B, H, d), dtype=torch.float32, device=dev)
+    bflag = torch.empty((B, H), dtype=torch.uint8, device=dev)
+    midx = torch.empty((B, H), dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        dla.dla_decode_step(p, cache, qs[i], ks[i], vs[i], ls[i], o, bflag, midx, stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    m_before = cache.view("m").to(torch.int64)
+    bytes_per_step = float(((m_before + 1) * d * d * 4).sum().item())
+    dla.dla_timing_read(reset=True)
+    dist.barrier()
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    nb_fire = 0
+    for i in range(args.warmup, nsteps):
+        step(i)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(False)
+    dist.barrier()
+    ms = dist.reduce(e0.elapsed_time(e1) / args.steps, "max")
+    timing = dla.dla_timing_read(reset=True)
+    dn, dms = timing["decode"]
+    achieved = bytes_per_step / (dms / dn * 1e-3) / 1e9
+    roof = {"kernel": "decode", "bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
+            "frac": round(achieved / pk["hbm"], 4), "traffic": None,
+            "work_per_launch": f"sum over streams (m+1)*d^2*4 = {bytes_per_step:.4g} bytes"}
+    nb_fire = int(bflag.sum().item())
+    # end to end: host q, k, v, lambda in, o out
+    e2e = None
+    if not args.no_e2e:
+        qh, kh, vh, lh = (x[:4].cpu().pin_memory() for x in (qs, ks, vs, ls))
+        oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+        qd, kd, vd, ld = (torch.empty_like(x[0]) for x in (qs, ks, vs, ls))
+        n_e2e = max(2, min(args.steps, 8))
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for i in range(n_e2e):
+            j = i % 4
+            qd.copy_(qh[j], non_blocking=True)
+            kd.copy_(kh[j], non_blocking=True)
+            vd.copy_(vh[j], non_blocking=True)
+            ld.copy_(lh[j], non_blocking=True)
+            dla.dla_decode_step(p, cache, qd, kd, vd, ld, o, bflag, midx, stream=stream)
+            oh.copy_(o, non_blocking=True)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = dist.reduce(a0.elapsed_time(a1) / n_e2e, "max")
+        e2e = {"value": round(dist.world * B / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
+               "h2d_bytes_per_step": sum(x[0].numel() * x.element_size() for x in (qh, kh, vh, lh)),
+               "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e}
+    res = {"metric": DECODE_METRIC, "value": round(dist.world * B / (ms * 1e-3), 1), "unit": "tokens/s",
+           "ms_per_step": round(ms, 4), "steps": args.steps, "higher_is_better": True,
+           "config": {"workload": f"decode: {B} sequences x H={H}, d={d}, C={C}, fp32 cache after a seeded "
+                                  f"{Tp}-token i.i.d. prefill; bf16 q/k/v N(0,1/128) per step",
+                      "l2": f"cache {cache.buf.numel() / 1e9:.1f} GB >> L2"},
+           "roofline": roof, "kernels": kernel_table(timing, args.steps), "e2e": e2e,
+           "gpu_launches": sum(n for n, _ in timing.values()), "prefill_setup_s": round(prefill_s, 2),
+           "boundaries_last_step": nb_fire}
+    del cache, qs, ks, vs, ls
+    torch.cuda.empty_cache()
+    return res
+
+
+# ---------------------------------------------------------------- oracle timings
+
+def oracle_sample(workload, tokens, heads=None, threads=None):
+    """The fp64 oracle over the first `tokens` tokens of every head of batch
+    row 0 (read-out at every token).  Returns (seconds, threads, token-heads)."""
+    import numpy as np
+    from concurrent.futures import ThreadPoolExecutor
+
+    import oracle
+    from paper_2606_10650_gb300 import workloads as W
+
+    w = W.get(workload)
+    H = w.H if heads is None else heads
+    streams = []
+    for h in range(H):
+        g = W.StreamGen(w, 0, h)
+        q, kk, vv = g.tokens()
+        streams.append((q[:tokens], kk[:tokens], vv[:tokens], g.lam()[:tokens]))
+    n = threads or min(len(streams), os.cpu_count() or 1)
+
+    def one(s):
+        st = oracle.Stream(w.C, w.d, w.d, w.tau, w.eps, w.rms_eps)
+        st.run(*s)
+
+    oracle.lib()
+    t0 = time.time()
+    with ThreadPoolExecutor(n) as ex:
+        list(ex.map(one, streams))
+    return time.time() - t0, n, H * tokens
+
+
+def cpu_baseline(args):
+    secs, n, th = oracle_sample(args.workload, args.cpu_tokens)
+    return {"value": round(args.cpu_tokens / secs, 2), "unit": "tokens/s", "cores": n, "kind": "oracle",
+            "seconds": round(secs, 2),
+            "sample": f"{args.workload} workload, batch row 0, all {th // args.cpu_tokens} heads, first "
+                      f"{args.cpu_tokens} tokens, read-out at every token (a token = all heads of one position)"}
+
+
+def run_reference(args, dist):
+    cfg = config_of(args)
+    if dist.rank != 0:
+        return
+    tok = args.ref_tokens
+    for _ in range(args.warmup):
+        oracle_sample(args.workload, tok)
+    times = []
+    cores = 1
+    for _ in range(args.steps):
+        s, cores, _ = oracle_sample(args.workload, tok)
+        times.append(s)
+    ms = 1e3 * sum(times) / len(times)
+    val = tok / (ms * 1e-3)
+    line = {"impl": "reference", "metric": PREFILL_METRIC, "value": round(val, 2), "unit": "tokens/s", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": cfg,
+            "cpu_baseline": {"value": round(val, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"each step: batch row 0, all heads, first {tok} tokens of the {args.workload} "
+                                       "workload, read-out at every token"},
+            "e2e": {"value": round(val, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def config_of(args):
+    from paper_2606_10650_gb300 import workloads as W
+    w = W.get(args.workload, **({"T": args.T} if args.T else {}))
+    return {"workload": f"{w.name}: B={w.B} H={w.H} T={w.T} d={w.d} C={w.C} {w.dtype} inputs, fp32 states, "
+                        f"tau={w.tau}, lambda U({w.lam_lo},{w.lam_hi})",
+            "global_batch": w.B, "seq_len": w.T, "parallelism": "replicas",
+            "l2": "inputs (q,k,v,lambda: %.0f MB) larger than L2" % (
+                (3 * w.B * w.T * w.H * w.d * (2 if w.dtype == 'bf16' else 4) + 4 * w.B * w.T * w.H * w.C) / 1e6)}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="dla", choices=["dla", "reference"])
+    ap.add_argument("--workload", default="regime")
+    ap.add_argument("--T", type=int, default=0)
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--decode-batch", type=int, default=0)
+    ap.add_argument("--cpu-tokens", type=int, default=8192)
+    ap.add_argument("--ref-tokens", type=int, default=512)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 0)
+    dist = Dist()
+    if args.impl == "reference":
+        run_reference(args, dist)
+        dist.close()
+        return
+    import __graft_entry__
+    __graft_entry__.build()
+    pk = peaks()
+    pre = None if args.no_prefill else bench_prefill(args, dist, pk)
+    dec = None if args.no_decode else bench_decode(args, dist, pk)
+    cpu = cpu_baseline(args) if (dist.rank == 0 and dist.world == 1 and not args.no_cpu) else None
+    if dist.rank == 0:
+        line = {"metric": PREFILL_METRIC, "unit": "tokens/s", "n_gpus": dist.world, "steps": args.steps,
+                "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic (seeded regime-shift streams; no dataset)",
+                "config": config_of(args), "peaks_source": pk["source"]}
+        if pre:
+            line.update(value=round(pre["value"], 1), ms_per_step=round(pre["ms_per_step"], 4),
+                        roofline=pre["roofline"], kernels=pre["kernels"], clocks=pre["clocks"], e2e=pre["e2e"],
+                        gpu_launches=pre["gpu_launches"],
+                        algorithmic_tflops=round(pre["algorithmic_tflops"], 3),
+                        trace={"sum_m": pre["sum_m"], "boundaries": pre["boundaries"], "merges": pre["merges"]})
+        if dec:
+            line["decode"] = dec
+        line["cpu_baseline"] = cpu
+        print(json.dumps(line))
+    dist.close()
+
+
+if __name__ == "__main__":
+    main()

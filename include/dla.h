@@ -148,6 +148,27 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
                            const void* q, const void* k, const void* v, const float* lam,
                            void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
 
+/* Instrumentation (no counterpart in the paper).  Kernel kinds of the
+ * library: K1 scan, K2 read-out, K3 decode, cache init. */
+typedef enum {
+  DLA_K_SCAN = 0,
+  DLA_K_READOUT = 1,
+  DLA_K_DECODE = 2,
+  DLA_K_INIT = 3,
+  DLA_K_COUNT = 4
+} dla_kernel_kind;
+
+/* enable = 1: from now on, every kernel this host thread launches through the
+ * library is bracketed by two CUDA events recorded on its stream (a few
+ * microseconds of host overhead per launch, none on the device).  enable = 0
+ * stops recording.  Returns DLA_ERR_CUDA if events cannot be created. */
+dla_status dla_timing_enable(int enable);
+
+/* Waits for the recorded events, then writes per kernel kind the number of
+ * launches (launches[DLA_K_COUNT], host memory) and their summed device time in
+ * milliseconds (ms[DLA_K_COUNT]).  reset = 1 forgets the records afterwards. */
+dla_status dla_timing_read(int* launches, double* ms, int reset);
+
 /* Message of the last error returned on this host thread ("" if none). */
 const char* dla_last_error(void);
 

@@ -5,6 +5,7 @@
 // kernels of dla_scan.cu / dla_readout_*.cu / dla_decode.cu.
 #include <math.h>
 #include <stdarg.h>
+#include <vector>
 #include <stdio.h>
 #include <string.h>
 
@@ -60,7 +61,10 @@ struct FwdPlan {
   size_t off_status, off_bnd, off_mlog, off_cache, off_m0, off_ids, off_pool, total;
 };
 
-size_t pool_elt(dla_dtype in_dtype) { return in_dtype == DLA_BF16 ? 2 : 4; }
+// Snapshot element size: the CUDA-core read-out keeps fp32 snapshots, since a
+// single bf16 rounding of the states (2^-9 relative) already reaches the 2e-2
+// output tolerance on coherent (regime) streams.
+size_t pool_elt(dla_dtype /*in_dtype*/) { return 4; }
 
 FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
                  bool with_output, bool need_trace, bool need_cache) {
@@ -118,6 +122,39 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
   return fail(DLA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
+// ---- optional per-launch CUDA-event timing (dla_timing_enable / _read)
+struct TimedLaunch {
+  int kind;
+  cudaEvent_t start, stop;
+};
+thread_local bool g_timing = false;
+thread_local std::vector<TimedLaunch> g_records;
+thread_local std::vector<cudaEvent_t> g_free_events;
+
+cudaEvent_t take_event() {
+  if (!g_free_events.empty()) {
+    cudaEvent_t e = g_free_events.back();
+    g_free_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Runs one launch, bracketed by events when timing is enabled.
+template <typename F>
+cudaError_t timed(int kind, cudaStream_t st, F&& launch) {
+  if (!g_timing) return launch();
+  TimedLaunch r{kind, take_event(), take_event()};
+  if (!r.start || !r.stop) return cudaErrorMemoryAllocation;
+  cudaEventRecord(r.start, st);
+  cudaError_t e = launch();
+  cudaEventRecord(r.stop, st);
+  g_records.push_back(r);
+  return e;
+}
+
 }  // namespace
 
 extern "C" {
@@ -134,6 +171,36 @@ void dla_default_params(dla_params* p) {
 }
 
 int dla_version(void) { return DLA_VERSION; }
+
+dla_status dla_timing_enable(int enable) {
+  g_timing = (enable != 0);
+  return ok();
+}
+
+dla_status dla_timing_read(int* launches, double* ms, int reset) {
+  if (!launches || !ms) return fail(DLA_ERR_INVALID_ARG, "launches and ms must be non-NULL");
+  for (int k = 0; k < DLA_K_COUNT; ++k) {
+    launches[k] = 0;
+    ms[k] = 0.0;
+  }
+  for (const TimedLaunch& r : g_records) {
+    cudaError_t e = cudaEventSynchronize(r.stop);
+    if (e != cudaSuccess) return cuda_fail(e, "timing event");
+    float t = 0.f;
+    e = cudaEventElapsedTime(&t, r.start, r.stop);
+    if (e != cudaSuccess) return cuda_fail(e, "timing elapsed");
+    launches[r.kind] += 1;
+    ms[r.kind] += t;
+  }
+  if (reset) {
+    for (const TimedLaunch& r : g_records) {
+      g_free_events.push_back(r.start);
+      g_free_events.push_back(r.stop);
+    }
+    g_records.clear();
+  }
+  return ok();
+}
 
 const char* dla_last_error(void) { return g_err; }
 
@@ -175,8 +242,10 @@ dla_status dla_init_cache(const dla_cache* cache, void* stream) {
   if (!cache) return fail(DLA_ERR_INVALID_ARG, "cache is NULL");
   if (cache->B < 1 || cache->H < 1 || cache->C < 2) return fail(DLA_ERR_INVALID_ARG, "bad cache dims");
   if (!cache->slot || !cache->n || !cache->ibar || !cache->m) return fail(DLA_ERR_INVALID_ARG, "cache has a NULL member");
-  cudaError_t e = dla::launch_init_cache(cache->slot, cache->n, cache->ibar, cache->m, cache->B * cache->H, cache->C,
-                                         (cudaStream_t)stream);
+  cudaError_t e = timed(DLA_K_INIT, (cudaStream_t)stream, [&] {
+    return dla::launch_init_cache(cache->slot, cache->n, cache->ibar, cache->m, cache->B * cache->H, cache->C,
+                                  (cudaStream_t)stream);
+  });
   if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
   return ok();
 }
@@ -253,7 +322,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);
   if (e != cudaSuccess) return cuda_fail(e, "status reset");
   if (!p->from_cache) {
-    e = dla::launch_init_cache(live.slot, live.n, live.ibar, live.m, B * H, C, st);
+    e = timed(DLA_K_INIT, st, [&] { return dla::launch_init_cache(live.slot, live.n, live.ibar, live.m, B * H, C, st); });
     if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
   }
 
@@ -267,11 +336,11 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   sa.boundary = bnd; sa.merge_log = mlog;
   sa.status = status;
   const bool in_bf16 = (in_dtype == DLA_BF16);
-  const bool pool_bf16 = in_bf16;
+  const bool pool_bf16 = false;
   if (!with_output) {
     sa.t_begin = 0; sa.t_end = T;
     sa.pool = nullptr; sa.pool_cap = 0; sa.nsnap = 1; sa.snap_chunks = 1;
-    e = dla::launch_scan(sa, d, in_bf16, pool_bf16, st);
+    e = timed(DLA_K_SCAN, st, [&] { return dla::launch_scan(sa, d, in_bf16, pool_bf16, st); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return ok();
   }
@@ -291,10 +360,10 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     const int t1 = (T - t0 < round_tokens) ? T : t0 + round_tokens;
     sa.t_begin = t0; sa.t_end = t1;
     sa.nsnap = (t1 - t0 + P.interval - 1) / P.interval;
-    e = dla::launch_scan(sa, d, in_bf16, pool_bf16, st);
+    e = timed(DLA_K_SCAN, st, [&] { return dla::launch_scan(sa, d, in_bf16, pool_bf16, st); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
-    e = dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st);
+    e = timed(DLA_K_READOUT, st, [&] { return dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st); });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
   }
   return ok();
@@ -319,7 +388,8 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
   da.sp.tau = p->tau; da.sp.eps = p->eps; da.sp.rms_eps = p->rms_eps; da.sp.score_mode = p->score_mode;
   da.states = cache->states; da.slot = cache->slot; da.n = cache->n; da.ibar = cache->ibar; da.m = cache->m;
   da.boundary = boundary; da.merge_idx = merge_idx;
-  cudaError_t e = dla::launch_decode(da, cache->dk, in_dtype == DLA_BF16, (cudaStream_t)stream);
+  cudaError_t e = timed(DLA_K_DECODE, (cudaStream_t)stream,
+                        [&] { return dla::launch_decode(da, cache->dk, in_dtype == DLA_BF16, (cudaStream_t)stream); });
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   return ok();
 }

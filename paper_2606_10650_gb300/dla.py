@@ -21,7 +21,8 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
-            "dla_last_error", "dla_status_string", "dla_version"]
+            "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read"]
+KERNELS = ["scan", "readout", "decode", "init"]
 
 
 class DLAError(RuntimeError):
@@ -70,6 +71,8 @@ def lib():
         L.dla_status_string.restype = ctypes.c_char_p
         L.dla_status_string.argtypes = [ci]
         L.dla_version.restype = ci
+        L.dla_timing_enable.argtypes = [ci]
+        L.dla_timing_read.argtypes = [ctypes.POINTER(ci), ctypes.POINTER(ctypes.c_double), ci]
         _LIB = L
     return _LIB
 
@@ -108,6 +111,19 @@ def dla_default_params():
     return p
 
 
+def dla_timing_enable(enable=True):
+    _check(lib().dla_timing_enable(int(bool(enable))))
+
+
+def dla_timing_read(reset=True):
+    """{kernel kind: (launches, summed ms)} of the launches recorded since the
+    last reset (see dla_timing_enable)."""
+    n = (ctypes.c_int * 4)()
+    ms = (ctypes.c_double * 4)()
+    _check(lib().dla_timing_read(n, ms, int(bool(reset))))
+    return {KERNELS[i]: (n[i], ms[i]) for i in range(4)}
+
+
 def dla_cache_bytes(B, H, C, dk, dv):
     return lib().dla_cache_bytes(B, H, C, dk, dv)
 
@@ -131,6 +147,20 @@ class Cache:
         self.c = dla_cache()
         _check(lib().dla_cache_carve(ctypes.c_void_p(base), nbytes, B, H, C, d, d, ctypes.byref(self.c)))
         self._base = base
+
+    def sub(self, b0, nb):
+        """A cache object over batch rows [b0, b0 + nb) of this cache (no copy)."""
+        c = dla_cache()
+        B, H, C, d = self.B, self.H, self.C, self.d
+        c.states = self.c.states + b0 * H * C * d * d * 4
+        c.slot = self.c.slot + b0 * H * C * 4
+        c.n = self.c.n + b0 * H * C * 4
+        c.ibar = self.c.ibar + b0 * H * C * 8
+        c.m = self.c.m + b0 * H * 4
+        c.B, c.H, c.C, c.dk, c.dv = nb, H, C, d, d
+        view = object.__new__(Cache)
+        view.B, view.H, view.C, view.d, view.buf, view.c, view._base = nb, H, C, d, self.buf, c, None
+        return view
 
     def view(self, name):
         """torch view of one cache array (states [B,H,C,d,d], slot/n [B,H,C],

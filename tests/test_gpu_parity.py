@@ -137,7 +137,7 @@ def test_decode_steps_match_prefill():
     """dla_forward over T0 tokens, then one dla_decode_step per token, equals
     the oracle over all T tokens (Sec. 3.1 inference rule is the same
     recurrence)."""
-    w = W.get("decode", B=3, H=2, T=300, decode_steps=90, C=16)
+    w = W.get("decode", B=3, H=2, T=300, decode_steps=90, C=4, tau=1.4142)
     Ttot = w.total_tokens
     q, k, v, lam = _safe(w, T=Ttot)
     r = run_oracle(w, q, k, v, lam)
