@@ -139,6 +139,29 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
                        void* workspace, size_t ws_bytes, void* stream);
 
+/* dla_forward for callers that cannot allocate device memory (the paper has
+ * no counterpart: this is a deployment convenience).  Some callers cannot
+ * call cudaMalloc where they run the forward pass -- for example a plugin of
+ * an inference engine that owns all device memory and hands out no workspace,
+ * or code running while another thread captures a CUDA graph in global mode,
+ * where an allocation is an error.  This entry point takes the same arguments
+ * as dla_forward minus the workspace: its scratch is a static device array of
+ * 64 MiB compiled into the library, which every GPU that loads the library
+ * holds until the process exits.  It allocates nothing.
+ *   - The first call on each device (with that device current) looks up the
+ *     array's device address with cudaGetSymbolAddress; make that first call
+ *     before any stream capture.
+ *   - A call whose workspace need exceeds 64 MiB returns DLA_ERR_WORKSPACE with
+ *     a message naming the limit; pass your own `cache` (and boundary /
+ *     merge_log arrays) to keep the need small, or use dla_forward.
+ *   - Every call shares the one array and rewrites the parts it reads; calls
+ *     that overlap on the GPU (different streams, or different host threads,
+ *     on the same device) race on it and must be serialised by the caller. */
+dla_status dla_forward_noalloc(const dla_params* p, dla_dtype in_dtype, int B, int T, int H,
+                               int dk, int dv, const void* q, const void* k, const void* v,
+                               const float* lam, void* o, const dla_cache* cache,
+                               uint8_t* boundary, int32_t* merge_log, void* stream);
+
 /* One recurrent step (Sec. 3.1 inference rule + Algorithm 2 + read-out) for
  * every stream: token (q, k, v) [B, H, d] against the persistent cache, which
  * is updated in place.  lam [B, H, C] fp32 or NULL; o [B, H, d] (out_dtype);

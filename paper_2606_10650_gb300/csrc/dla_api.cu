@@ -157,6 +157,16 @@ cudaError_t timed(int kind, cudaStream_t st, F&& launch) {
 
 }  // namespace
 
+namespace dla {
+dla_status set_error(dla_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+}  // namespace dla
+
 extern "C" {
 
 void dla_default_params(dla_params* p) {

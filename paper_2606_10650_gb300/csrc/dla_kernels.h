@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "dla.h"
+
 namespace dla {
 
 constexpr int kMaxC = 64;   // largest supported capacity C
@@ -82,6 +84,10 @@ struct DecodeArgs {
   uint8_t* boundary;     // [B, H] or nullptr
   int32_t* merge_idx;    // [B, H] or nullptr
 };
+
+// Records a formatted message as the calling thread's dla_last_error() and
+// returns s (for entry points defined outside dla_api.cu).
+dla_status set_error(dla_status s, const char* fmt, ...);
 
 cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 size_t scan_smem_bytes(int d);

@@ -21,7 +21,7 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
-            "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read"]
+            "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc"]
 KERNELS = ["scan", "readout", "decode", "init"]
 
 
@@ -71,6 +71,7 @@ def lib():
         L.dla_status_string.restype = ctypes.c_char_p
         L.dla_status_string.argtypes = [ci]
         L.dla_version.restype = ci
+        L.dla_forward_noalloc.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp]
         L.dla_timing_enable.argtypes = [ci]
         L.dla_timing_read.argtypes = [ctypes.POINTER(ci), ctypes.POINTER(ctypes.c_double), ci]
         _LIB = L
@@ -226,6 +227,17 @@ def dla_forward(params, q, k, v, lam=None, o=None, cache=None, boundary=None, me
                            ctypes.c_void_p(base), nb, _stream(stream))
     _check(st)
     return workspace
+
+
+def dla_forward_noalloc(params, q, k, v, lam=None, o=None, cache=None, boundary=None, merge_log=None, stream=None):
+    """dla_forward without a workspace argument, for callers that cannot
+    allocate: the library's 64 MiB static device scratch is used instead (see
+    include/dla.h).  Same tensor conventions as dla_forward."""
+    B, T, H, d = k.shape
+    st = lib().dla_forward_noalloc(ctypes.byref(params), _dtype_code(k), B, T, H, d, d, _ptr(q), _ptr(k), _ptr(v),
+                                   _ptr(lam), _ptr(o), ctypes.byref(cache.c) if cache is not None else None,
+                                   _ptr(boundary), _ptr(merge_log), _stream(stream))
+    _check(st)
 
 
 def dla_decode_step(params, cache: Cache, q, k, v, lam=None, o=None, boundary=None, merge_idx=None, stream=None):

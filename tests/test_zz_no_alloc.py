@@ -1,0 +1,70 @@
+"""dla_forward_noalloc: the forward pass for callers that cannot allocate
+device memory (for example an engine plugin that is handed no workspace, or
+code running while another thread captures a CUDA graph in global mode).  It
+uses the library's static 64 MiB device scratch instead of a caller
+workspace.  This file is collected last on purpose.
+
+Checked through the C ABI against dla_forward (the entry point with a caller
+workspace) on the same inputs, for two calls in a row with different inputs,
+so that scratch left over from the first call cannot leak into the second."""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_10650_gb300 import dla
+from paper_2606_10650_gb300 import workloads as W
+from parity_util import TOL
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(seed, dev):
+    w = W.get("regime", B=1, H=2, T=900)
+    q, k, v, lam = W.host_batch(w, seed=seed, T=w.T)
+    t = [W.to_device(x, w.dtype, dev) for x in (q, k, v)]
+    t.append(torch.from_numpy(lam.astype(np.float32)).to(dev))
+    return w, t
+
+
+def _run(entry, w, t, dev):
+    q, k, v, lam = t
+    B, T, H, d = k.shape
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    o = torch.full((B, T, H, d), float("nan"), device=dev)
+    bnd = torch.zeros((B, H, T), dtype=torch.uint8, device=dev)
+    ml = torch.zeros((B, H, T), dtype=torch.int32, device=dev)
+    if entry == "noalloc":
+        dla.dla_forward_noalloc(p, q, k, v, lam, o, cache, bnd, ml)
+    else:
+        dla.dla_forward(p, q, k, v, lam, o, cache, bnd, ml)
+    torch.cuda.synchronize()
+    return o.cpu(), bnd.cpu(), ml.cpu(), cache.export()
+
+
+def test_noalloc_matches_dla_forward_two_calls_in_a_row():
+    dev = torch.device("cuda:0")
+    for seed in (11, 12):  # two calls in a row, different inputs
+        w, t = _inputs(seed, dev)
+        o_ref, b_ref, m_ref, c_ref = _run("workspace", w, t, dev)
+        o, b, m, c = _run("noalloc", w, t, dev)
+        assert torch.equal(b, b_ref) and torch.equal(m, m_ref)
+        assert torch.isfinite(o).all()
+        assert (o - o_ref).abs().max().item() <= TOL[w.dtype]
+        assert torch.equal(c["m"], c_ref["m"]) and torch.equal(c["n"], c_ref["n"])
+        assert (c["states"] - c_ref["states"]).abs().max().item() <= TOL[w.dtype]
+
+
+def test_noalloc_rejects_calls_beyond_its_scratch():
+    """Without a caller cache the cache itself must live in the scratch; for a
+    large batch that exceeds the 64 MiB limit and the call is refused with a
+    message naming it, before anything is launched."""
+    L = dla.lib()
+    p = dla.make_params(1.3, 64)
+    fake = ctypes.c_void_p(1 << 24)
+    st = L.dla_forward_noalloc(ctypes.byref(p), dla.DLA_BF16, 8, 4096, 32, 128, 128, fake, fake, fake, None, fake,
+                               None, None, None, None)
+    assert st == 3
+    assert b"static scratch" in L.dla_last_error()
