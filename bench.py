@@ -167,6 +167,8 @@ def bench_prefill(args, dist, pk):
     bnd = torch.empty((B, H, T), dtype=torch.uint8, device=dev)
     ml = torch.empty((B, H, T), dtype=torch.int32, device=dev)
     nb = dla.dla_forward_workspace(p, B, T, H, d, d, in_code, True)
+    if args.ws_gb:
+        nb = max(min(nb, int(args.ws_gb * (1 << 30))), dla.dla_forward_min_workspace(p, B, T, H, d, d, in_code, True))
     buf = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
     ws = (buf, (buf.data_ptr() + 255) // 256 * 256, nb)
     stream = torch.cuda.current_stream()
@@ -203,16 +205,33 @@ def bench_prefill(args, dist, pk):
     flops_readout = 2.0 * d * d * sum_m
     flops_total = 2.0 * d * d * (sum_m + 2 * T * BH)
     kt_tab = kernel_table(timing, args.steps)
+    tc_path = (w.dtype == "bf16" and d == 128)
     ro_n, ro_ms = timing["readout"]
+    sc_n, sc_ms = timing["scan"]
     fp32_peak = pk_fp32(pk)
-    # flops_readout is per step; the launches of a step share it
-    achieved = flops_readout * args.steps / (ro_ms * 1e-3) / 1e12 if ro_n else None
-    roof = {"kernel": "readout", "bound": "alu", "achieved": round(achieved, 3) if achieved else None,
-            "peak": round(fp32_peak, 2), "unit": "TFLOP/s",
-            "frac": round(achieved / fp32_peak, 4) if achieved else None, "traffic": None,
-            "peak_note": "fp32 FFMA peak: 152 SMs x 128 lanes x 2 flop x sm_max_mhz of MEASURED_PEAKS.json",
-            "work_per_launch": f"2*d^2*sum_t m_t / launches per step = "
-                               f"{flops_readout * args.steps / max(1, ro_n):.4g} flop"}
+    rooflines = {}
+    if ro_n:
+        ach = flops_readout * args.steps / (ro_ms * 1e-3) / 1e12  # flops_readout is per step
+        peak = pk["bf16"] if tc_path else fp32_peak
+        rooflines["readout"] = {
+            "kernel": "readout", "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
+            "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
+            "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else
+                          "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
+            "work_per_launch": f"2*d^2*sum_t m_t / launches = {flops_readout * args.steps / ro_n:.4g} flop",
+            "executed_note": ("each state product runs as two bf16 MMAs (hi + lo split of the fp32 state): "
+                              "executed tensor flops are 2x the algorithmic count" if tc_path else "")}
+    if sc_n:
+        flops_scan = 4.0 * d * d * T * BH  # x_t = v^T S k and the state build, 2 d^2 each per token
+        ach = flops_scan * args.steps / (sc_ms * 1e-3) / 1e12
+        rooflines["scan"] = {
+            "kernel": "scan", "bound": "alu", "achieved": round(ach, 3), "peak": round(fp32_peak, 2),
+            "unit": "TFLOP/s", "frac": round(ach / fp32_peak, 4), "traffic": None,
+            "peak_note": "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz",
+            "work_per_launch": f"4*d^2*T*B*H / launches = {flops_scan * args.steps / sc_n:.4g} flop",
+            "note": "sequential per stream: one CTA per (batch, head), B*H CTAs"}
+    dominant = max(rooflines, key=lambda k: timing[k][1]) if rooflines else None
+    roof = rooflines.get(dominant)
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -243,7 +262,7 @@ def bench_prefill(args, dist, pk):
         e2e = {"value": round(dist.world * tokens / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
                "h2d_bytes_per_step": hb, "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e}
     res = {"value": dist.world * tokens / (ms_max * 1e-3), "ms_per_step": ms_max, "tokens_per_step": tokens,
-           "roofline": roof, "kernels": kt_tab, "clocks": clk, "e2e": e2e,
+           "roofline": roof, "rooflines": rooflines, "kernels": kt_tab, "tc_path": tc_path, "clocks": clk, "e2e": e2e,
            "gpu_launches": sum(n for n, _ in timing.values()),
            "algorithmic_tflops": flops_total / (ms_max * 1e-3) / 1e12, "sum_m": sum_m,
            "boundaries": int(bnd.sum().item()), "merges": int((ml >= 0).sum().item())}
@@ -442,6 +461,7 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--decode-batch", type=int, default=0)
+    ap.add_argument("--ws-gb", type=float, default=0.0, help="cap the prefill workspace (GiB)")
     ap.add_argument("--cpu-tokens", type=int, default=8192)
     ap.add_argument("--ref-tokens", type=int, default=512)
     args = ap.parse_args()
@@ -460,11 +480,11 @@ def main():
     if dist.rank == 0:
         line = {"metric": PREFILL_METRIC, "unit": "tokens/s", "n_gpus": dist.world, "steps": args.steps,
                 "warmup": args.warmup, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-                "dtype": "f32", "data": "synthetic (seeded regime-shift streams; no dataset)",
+                "dtype": "bf16" if (pre and pre["tc_path"]) else "f32", "data": "synthetic (seeded regime-shift streams; no dataset)",
                 "config": config_of(args), "peaks_source": pk["source"]}
         if pre:
             line.update(value=round(pre["value"], 1), ms_per_step=round(pre["ms_per_step"], 4),
-                        roofline=pre["roofline"], kernels=pre["kernels"], clocks=pre["clocks"], e2e=pre["e2e"],
+                        roofline=pre["roofline"], rooflines=pre["rooflines"], kernels=pre["kernels"], clocks=pre["clocks"], e2e=pre["e2e"],
                         gpu_launches=pre["gpu_launches"],
                         algorithmic_tflops=round(pre["algorithmic_tflops"], 3),
                         trace={"sum_m": pre["sum_m"], "boundaries": pre["boundaries"], "merges": pre["merges"]})

@@ -133,7 +133,11 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
  *   the final cache; with p->from_cache = 1 it is also the starting cache.
  *   With cache == NULL the cache lives in the workspace and from_cache must
  *   be 0.
- *   workspace: device memory of ws_bytes >= dla_forward_min_workspace(...). */
+ *   workspace: device memory of ws_bytes >= dla_forward_min_workspace(...).
+ *   Its first 4 bytes receive the device status of the call once the work has
+ *   run (int32: 0 ok, DLA_ERR_TIMEOUT when a bounded wait of a kernel gave up,
+ *   DLA_ERR_DEVICE_CHECK when a kernel found an inconsistent cache or pool);
+ *   read them after synchronising the stream. */
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,

@@ -50,8 +50,13 @@ CacheLayout cache_layout(int B, int H, int C, int dk, int dv) {
   return L;
 }
 
-// Read-out interval (tokens per K2 CTA / per snapshot) of a configuration.
-int readout_interval(dla_dtype /*in_dtype*/) { return dla::kReadoutSimtInterval; }
+// The read-out kernel of a configuration: bf16 inputs with d = 128 run on the
+// tensor cores (128-token intervals, bf16 hi/lo snapshots); everything else on
+// CUDA cores (64-token intervals, fp32 snapshots).
+bool use_tc(dla_dtype in_dtype, int d) { return in_dtype == DLA_BF16 && d == 128; }
+int readout_interval(dla_dtype in_dtype, int d) {
+  return use_tc(in_dtype, d) ? dla::kReadoutTcInterval : dla::kReadoutSimtInterval;
+}
 
 struct FwdPlan {
   int interval;      // tokens per snapshot interval
@@ -61,9 +66,10 @@ struct FwdPlan {
   size_t off_status, off_bnd, off_mlog, off_cache, off_m0, off_ids, off_pool, total;
 };
 
-// Snapshot element size: the CUDA-core read-out keeps fp32 snapshots, since a
-// single bf16 rounding of the states (2^-9 relative) already reaches the 2e-2
-// output tolerance on coherent (regime) streams.
+// Bytes per snapshot element: fp32 (CUDA-core read-out) or bf16 hi + lo
+// (tensor-core read-out).  A single bf16 rounding of the states (2^-9
+// relative) already reaches the 2e-2 output tolerance on coherent (regime)
+// streams, hence the hi/lo pair.
 size_t pool_elt(dla_dtype /*in_dtype*/) { return 4; }
 
 FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
@@ -71,7 +77,7 @@ FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dty
   FwdPlan P;
   const size_t BH = (size_t)B * H;
   const int C = p->capacity;
-  P.interval = readout_interval(in_dtype);
+  P.interval = readout_interval(in_dtype, d);
   P.nsnap_total = (T + P.interval - 1) / P.interval;
   P.R = R;
   const int per_snap = C < P.interval + 1 ? C : P.interval + 1;
@@ -262,7 +268,7 @@ dla_status dla_init_cache(const dla_cache* cache, void* stream) {
 
 static FwdPlan choose_plan(const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype, bool with_output,
                            bool need_trace, bool need_cache, size_t budget) {
-  const int nsnap = (T + readout_interval(in_dtype) - 1) / readout_interval(in_dtype);
+  const int nsnap = (T + readout_interval(in_dtype, d) - 1) / readout_interval(in_dtype, d);
   if (!with_output) return plan_for(1, p, B, T, H, d, in_dtype, false, need_trace, need_cache);
   int lo = 1, hi = nsnap;
   FwdPlan best = plan_for(1, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
@@ -346,7 +352,8 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   sa.boundary = bnd; sa.merge_log = mlog;
   sa.status = status;
   const bool in_bf16 = (in_dtype == DLA_BF16);
-  const bool pool_bf16 = false;
+  const bool tc = use_tc(in_dtype, d);
+  const bool pool_bf16 = tc;
   if (!with_output) {
     sa.t_begin = 0; sa.t_end = T;
     sa.pool = nullptr; sa.pool_cap = 0; sa.nsnap = 1; sa.snap_chunks = 1;
@@ -373,7 +380,9 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     e = timed(DLA_K_SCAN, st, [&] { return dla::launch_scan(sa, d, in_bf16, pool_bf16, st); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
-    e = timed(DLA_K_READOUT, st, [&] { return dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st); });
+    e = timed(DLA_K_READOUT, st, [&] {
+      return tc ? dla::launch_readout_tc(ra, status, st) : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st);
+    });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
   }
   return ok();

@@ -14,14 +14,16 @@ namespace dla {
 // N(X) = X / sqrt(||X||^2 / D + rms_eps)):
 //   a = ||s||^2 = ||k||^2 ||v||^2,  beta = <s, S> = v^T S k,  gam = ||S||^2.
 // Mode 0 compares N(s) with N(S) (Algorithm 1); mode 1 compares N(S + s)
-// with N(S) (Eq. importance_score read literally).  Since
-// ||N(A) - N(B)||^2 = |A|^2/ra^2 + |B|^2/rb^2 - 2<A,B>/(ra rb), the score
-// needs no d x d work once a, beta, gam are known.
-__device__ __forceinline__ double info_score(double a, double beta, double gam, double D,
-                                             const ScoreParams& p) {
-  double AA, BB, AB;
+// with N(S) (Eq. importance_score read literally).  With x = ||N(A)||,
+// y = ||N(B)|| and c = <A,B> / (||A|| ||B||),
+//   ||N(A) - N(B)||^2 = (x - y)^2 + 2 x y (1 - c),
+// a form without the cancellation of x^2 + y^2 - 2xyc; it needs no d x d work
+// once a, beta, gam are known.  Evaluated in fp32 (GB300's fp64 rate is a
+// small fraction of its fp32 rate); the inputs carry ~1e-7 relative error.
+__device__ __forceinline__ float info_score(float a, float beta, float gam, float D, const ScoreParams& p) {
+  float AA, BB, AB;
   if (p.score_mode == 1) {
-    AA = gam + 2.0 * beta + a;
+    AA = gam + 2.f * beta + a;
     BB = gam;
     AB = gam + beta;
   } else {
@@ -29,14 +31,15 @@ __device__ __forceinline__ double info_score(double a, double beta, double gam, 
     BB = gam;
     AB = beta;
   }
-  AA = fmax(AA, 0.0);
-  BB = fmax(BB, 0.0);
-  double ra = sqrt(AA / D + p.rms_eps);
-  double rb = sqrt(BB / D + p.rms_eps);
-  double num2 = AA / (ra * ra) + BB / (rb * rb) - 2.0 * AB / (ra * rb);
-  double num = sqrt(fmax(num2, 0.0));
-  double den = sqrt(BB) / rb + p.eps;
-  return num / den;
+  AA = fmaxf(AA, 0.f);
+  BB = fmaxf(BB, 0.f);
+  const float re = (float)p.rms_eps;
+  const float x = sqrtf(AA / (AA / D + re));
+  const float y = sqrtf(BB / (BB / D + re));
+  const float nab = sqrtf(AA) * sqrtf(BB);
+  const float c = nab > 0.f ? fminf(fmaxf(AB / nab, -1.f), 1.f) : 0.f;
+  const float num2 = (x - y) * (x - y) + 2.f * x * y * (1.f - c);
+  return sqrtf(fmaxf(num2, 0.f)) / (y + (float)p.eps);
 }
 
 template <typename T>

@@ -1,17 +1,20 @@
 // dla_decode.cu -- K3: one recurrent DLA step for every (batch, head) stream
 // against its persistent fp32 cache (Sec. 3.1 inference rule, Algorithm 2,
 // Eq. capacity_bounded_output).  Bandwidth-bound: the step reads every live
-// state once and writes one state (plus one more when a merge happens).
+// state once and writes one state (plus the merged one when a merge happens).
 //
-// One CTA (512 threads) per stream.  Thread (row j, part p) owns row j of a
-// state and a contiguous quarter (d = 128) of its columns, so every access is
-// a coalesced 16-byte load / store and per-row reductions stay inside a quad.
+// One CTA (512 threads) per stream.  A state row (d_k floats) is read by
+// LPR = d/4 consecutive lanes, one 16-byte load each, so a warp reads whole
+// rows contiguously; thread (row group rg, lane-in-row li) owns columns
+// 4li..4li+3 of rows rg, rg + NT/LPR, ...  The thread keeps its four q and k
+// values in registers and accumulates a partial o for each of its rows over all
+// states; the lanes of a row are reduced once at the end.
 //   pass A: stream the open state into shared memory while forming
-//           beta = v^T S k, gam = |S|^2 and u = S q;
+//           beta = v^T S k and gam = |S|^2;
 //   decide: score, boundary, and (full cache) the adjacent-pair argmin;
-//   pass B: stream the other states once, accumulating lambda' (S q) with the
-//           post-step logical slot of each state, write the merged state, then
-//           the updated open state (S + v k^T) or the new state v k^T.
+//   pass B: stream every other state once, weighting S q with the post-step
+//           logical slot's lambda; write the merged state, then the updated
+//           open state (S + v k^T) or the new state v k^T.
 #include "dla_common.cuh"
 
 namespace dla {
@@ -23,32 +26,30 @@ constexpr int NT = 512;
 template <int D>
 struct DecSmem {
   float S[D * D];  // open state
-  float q[D], k[D], v[D];
-  float u[D];      // S_open q
+  float v[D];
+  float red[NT / 32][5];
   double ibar[kMaxC];
   int n[kMaxC];
   int slot[kMaxC];
   int newidx[kMaxC];  // post-step logical slot of every pre-step entry
-  double red[NT / 32][2];
-  float qk;
-  double a_norm;
-  double Ival;
-  int m, bflag, jmerge, m_new;
+  float qk, Ival;
+  int m, bflag, jmerge;
 };
 
 }  // namespace
 
 template <int D, typename Tin, typename Tout>
 __global__ void __launch_bounds__(NT, 2) decode_kernel(DecodeArgs a) {
-  constexpr int TPR = NT / D;   // threads per row
-  constexpr int KPT = D / TPR;  // columns per thread
+  constexpr int LPR = D / 4;    // lanes per row
+  constexpr int RG = NT / LPR;  // row groups
+  constexpr int RPT = D / RG;   // rows per thread
   extern __shared__ __align__(16) unsigned char smem_raw[];
   DecSmem<D>& sm = *reinterpret_cast<DecSmem<D>*>(smem_raw);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int bh = blockIdx.x;
   const int C = a.C;
-  const int row = tid / TPR, part = tid % TPR;
-  const int col0 = part * KPT;
+  const int li = tid % LPR, rg = tid / LPR;
+  const int col = 4 * li;
   float* states = a.states + (long long)bh * C * D * D;
 
   if (tid == 0) sm.m = min(max(a.m[bh], 0), C);  // a corrupted cache cannot index out of bounds
@@ -61,81 +62,67 @@ __global__ void __launch_bounds__(NT, 2) decode_kernel(DecodeArgs a) {
   const Tin* qin = reinterpret_cast<const Tin*>(a.q) + (long long)bh * D;
   const Tin* kin = reinterpret_cast<const Tin*>(a.k) + (long long)bh * D;
   const Tin* vin = reinterpret_cast<const Tin*>(a.v) + (long long)bh * D;
-  for (int i = tid; i < D; i += NT) {
-    sm.q[i] = to_f32(qin[i]);
-    sm.k[i] = to_f32(kin[i]);
-    sm.v[i] = to_f32(vin[i]);
-  }
+  const float4 q4 = make_float4(to_f32(qin[col]), to_f32(qin[col + 1]), to_f32(qin[col + 2]), to_f32(qin[col + 3]));
+  const float4 k4 = make_float4(to_f32(kin[col]), to_f32(kin[col + 1]), to_f32(kin[col + 2]), to_f32(kin[col + 3]));
+  for (int i = tid; i < D; i += NT) sm.v[i] = to_f32(vin[i]);
   __syncthreads();
-  if (warp == 0) {  // |k|^2 |v|^2 and q.k
-    float kk = 0.f, vv = 0.f, qk = 0.f;
-    for (int i = lane; i < D; i += 32) {
-      kk += sm.k[i] * sm.k[i];
-      vv += sm.v[i] * sm.v[i];
-      qk += sm.q[i] * sm.k[i];
-    }
-    kk = warp_sum(kk);
-    vv = warp_sum(vv);
-    qk = warp_sum(qk);
-    if (lane == 0) {
-      sm.a_norm = (double)kk * (double)vv;
-      sm.qk = qk;
-    }
-  }
   const int m = sm.m;
   // ---------------------------------------------------------------- pass A
-  double beta_p = 0.0, gam_p = 0.0;
+  float beta_p = 0.f, gam_p = 0.f, kk_p = 0.f, vv_p = 0.f, qk_p = 0.f;
+  if (rg == 0) {  // |k|^2 and q.k: each column block counted once
+    kk_p = k4.x * k4.x + k4.y * k4.y + k4.z * k4.z + k4.w * k4.w;
+    qk_p = q4.x * k4.x + q4.y * k4.y + q4.z * k4.z + q4.w * k4.w;
+  }
+  if (tid < D) vv_p = sm.v[tid] * sm.v[tid];
   if (m > 0) {
-    const float* src = states + (long long)sm.slot[m - 1] * D * D + row * D + col0;
-    float4 r4[KPT / 4];
+    const float* src = states + (long long)sm.slot[m - 1] * D * D;
+    float4 s4[RPT];
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) r4[c] = load4(src + 4 * c);
-    float dk = 0.f, dq = 0.f;
+    for (int r = 0; r < RPT; ++r) s4[r] = load4(src + (rg + r * RG) * D + col);
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) {
-      const int cc = col0 + 4 * c;
-      store4(sm.S + row * D + cc, r4[c]);
-      dk += r4[c].x * sm.k[cc] + r4[c].y * sm.k[cc + 1] + r4[c].z * sm.k[cc + 2] + r4[c].w * sm.k[cc + 3];
-      dq += r4[c].x * sm.q[cc] + r4[c].y * sm.q[cc + 1] + r4[c].z * sm.q[cc + 2] + r4[c].w * sm.q[cc + 3];
-      gam_p += (double)r4[c].x * r4[c].x + (double)r4[c].y * r4[c].y + (double)r4[c].z * r4[c].z +
-               (double)r4[c].w * r4[c].w;
-    }
-#pragma unroll
-    for (int o = 1; o < TPR; o <<= 1) {
-      dk += __shfl_xor_sync(0xffffffffu, dk, o);
-      dq += __shfl_xor_sync(0xffffffffu, dq, o);
-    }
-    if (part == 0) {
-      sm.u[row] = dq;
-      beta_p = (double)sm.v[row] * (double)dk;
+    for (int r = 0; r < RPT; ++r) {
+      const int row = rg + r * RG;
+      store4(sm.S + row * D + col, s4[r]);
+      const float dk = s4[r].x * k4.x + s4[r].y * k4.y + s4[r].z * k4.z + s4[r].w * k4.w;
+      beta_p += sm.v[row] * dk;
+      gam_p += s4[r].x * s4[r].x + s4[r].y * s4[r].y + s4[r].z * s4[r].z + s4[r].w * s4[r].w;
     }
   }
   beta_p = warp_sum(beta_p);
   gam_p = warp_sum(gam_p);
+  kk_p = warp_sum(kk_p);
+  vv_p = warp_sum(vv_p);
+  qk_p = warp_sum(qk_p);
   if (lane == 0) {
     sm.red[warp][0] = beta_p;
     sm.red[warp][1] = gam_p;
+    sm.red[warp][2] = kk_p;
+    sm.red[warp][3] = vv_p;
+    sm.red[warp][4] = qk_p;
   }
   __syncthreads();
   // ---------------------------------------------------------------- decide
   if (warp == 0) {
-    double beta = 0.0, gam = 0.0;
+    float beta = 0.f, gam = 0.f, kk = 0.f, vv = 0.f, qk = 0.f;
     for (int w = 0; w < NT / 32; ++w) {
       beta += sm.red[w][0];
       gam += sm.red[w][1];
+      kk += sm.red[w][2];
+      vv += sm.red[w][3];
+      qk += sm.red[w][4];
     }
     int bflag = 1, j = -1;
-    double I = 0.0;
+    float I = 0.f;
     if (m > 0) {
-      I = info_score(sm.a_norm, beta, gam, (double)D * (double)D, a.sp);
-      bflag = (I >= a.sp.tau) ? 1 : 0;
+      I = info_score(kk * vv, beta, gam, (float)(D * D), a.sp);
+      bflag = ((double)I >= a.sp.tau) ? 1 : 0;
       if (bflag && m == C) j = pair_argmin_warp(sm.n, sm.ibar, m);
     }
-    // post-step logical slot of each pre-step entry
     for (int i = lane; i < m; i += 32) sm.newidx[i] = (j >= 0 && i > j) ? i - 1 : i;
     __syncwarp();
     if (lane == 0) {
       sm.Ival = I;
+      sm.qk = qk;
       sm.bflag = bflag;
       sm.jmerge = j;
     }
@@ -145,86 +132,90 @@ __global__ void __launch_bounds__(NT, 2) decode_kernel(DecodeArgs a) {
   const int bflag = sm.bflag, jm = sm.jmerge;
   const int m_new = bflag ? (jm >= 0 ? m : m + 1) : m;
   const float* lam = a.lam ? a.lam + (long long)bh * C : nullptr;
-  // ---------------------------------------------------------------- pass B
-  float acc = 0.f;  // this thread's share of (sum lambda' S q)_row over its columns
   const int open = m - 1;
+  // ---------------------------------------------------------------- pass B
+  float acc[RPT];
+#pragma unroll
+  for (int r = 0; r < RPT; ++r) acc[r] = 0.f;
   for (int i = 0; i < m; ++i) {
     if (i == open) continue;
     if (jm >= 0 && i == jm + 1) continue;  // consumed with its merge partner
     const float w = lam ? lam[sm.newidx[i]] : 1.f;
-    const float* src = states + (long long)sm.slot[i] * D * D + row * D + col0;
-    float4 r4[KPT / 4];
+    const float* src = states + (long long)sm.slot[i] * D * D;
+    float4 s4[RPT];
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) r4[c] = load4(src + 4 * c);
+    for (int r = 0; r < RPT; ++r) s4[r] = load4(src + (rg + r * RG) * D + col);
     if (jm >= 0 && i == jm) {
-      // merge partner: global state, or the open state in shared memory; the
-      // partner is streamed one 16-byte piece at a time to keep registers low
-      const float* psrc = (jm + 1 == open) ? sm.S + row * D + col0
-                                           : states + (long long)sm.slot[jm + 1] * D * D + row * D + col0;
-      float* dst = states + (long long)sm.slot[jm] * D * D + row * D + col0;
-      float d = 0.f, dp = 0.f;
+      // merge partner: a global state, or the open state in shared memory
+      const bool part_open = (jm + 1 == open);
+      const float* psrc = part_open ? sm.S : states + (long long)sm.slot[jm + 1] * D * D;
+      float* dst = states + (long long)sm.slot[jm] * D * D;
 #pragma unroll
-      for (int c = 0; c < KPT / 4; ++c) {
-        const int cc = col0 + 4 * c;
-        const float4 p4 = load4(psrc + 4 * c);
-        d += r4[c].x * sm.q[cc] + r4[c].y * sm.q[cc + 1] + r4[c].z * sm.q[cc + 2] + r4[c].w * sm.q[cc + 3];
-        dp += p4.x * sm.q[cc] + p4.y * sm.q[cc + 1] + p4.z * sm.q[cc + 2] + p4.w * sm.q[cc + 3];
-        store4(dst + 4 * c, make_float4(r4[c].x + p4.x, r4[c].y + p4.y, r4[c].z + p4.z, r4[c].w + p4.w));
+      for (int r = 0; r < RPT; ++r) {
+        const int off = (rg + r * RG) * D + col;
+        const float4 p4 = load4(psrc + off);
+        float d = s4[r].x * q4.x + s4[r].y * q4.y + s4[r].z * q4.z + s4[r].w * q4.w;
+        if (!part_open) d += p4.x * q4.x + p4.y * q4.y + p4.z * q4.z + p4.w * q4.w;
+        acc[r] += w * d;  // an open partner's share is added below from shared memory
+        store4(dst + off, make_float4(s4[r].x + p4.x, s4[r].y + p4.y, s4[r].z + p4.z, s4[r].w + p4.w));
       }
-      acc += w * d;
-      if (jm + 1 != open) acc += w * dp;  // the open state's share is added below from u
       continue;
     }
-    float d = 0.f;
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) {
-      const int cc = col0 + 4 * c;
-      d += r4[c].x * sm.q[cc] + r4[c].y * sm.q[cc + 1] + r4[c].z * sm.q[cc + 2] + r4[c].w * sm.q[cc + 3];
-    }
-    acc += w * d;
+    for (int r = 0; r < RPT; ++r)
+      acc[r] += w * (s4[r].x * q4.x + s4[r].y * q4.y + s4[r].z * q4.z + s4[r].w * q4.w);
   }
-#pragma unroll
-  for (int o = 1; o < TPR; o <<= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  // open state's read-out (S_open q from pass A) and the token's own term
-  float orow = acc;
-  const float vj = sm.v[row];
+  // the open state's read-out, from its copy in shared memory
   if (m > 0) {
     const float wopen = lam ? lam[sm.newidx[open]] : 1.f;
-    orow += wopen * sm.u[row];
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+      const float4 s4 = load4(sm.S + (rg + r * RG) * D + col);
+      acc[r] += wopen * (s4.x * q4.x + s4.y * q4.y + s4.z * q4.z + s4.w * q4.w);
+    }
   }
-  {
-    // the token state v k^T is read out with the slot it lands in
-    const int slot_tok = bflag ? (m_new - 1) : (m - 1);
-    const float wt = lam ? lam[slot_tok] : 1.f;
-    orow += wt * sm.qk * vj;
-  }
+  // reduce the lanes of each row
+#pragma unroll
+  for (int r = 0; r < RPT; ++r)
+#pragma unroll
+    for (int o = 1; o < LPR; o <<= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+  // the token state v k^T is read out with the slot it lands in
+  const int slot_tok = bflag ? (m_new - 1) : (m - 1);
+  const float wt = lam ? lam[slot_tok] : 1.f;
+  const float qk = sm.qk;
   // ---------------------------------------------------------------- write states
   if (!bflag) {  // S_open += v k^T
-    float* dst = states + (long long)sm.slot[open] * D * D + row * D + col0;
+    float* dst = states + (long long)sm.slot[open] * D * D;
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) {
-      const int cc = col0 + 4 * c;
-      float4 s4 = load4(sm.S + row * D + cc);
-      store4(dst + 4 * c, make_float4(s4.x + vj * sm.k[cc], s4.y + vj * sm.k[cc + 1],
-                                      s4.z + vj * sm.k[cc + 2], s4.w + vj * sm.k[cc + 3]));
+    for (int r = 0; r < RPT; ++r) {
+      const int row = rg + r * RG;
+      const float vj = sm.v[row];
+      const float4 s4 = load4(sm.S + row * D + col);
+      store4(dst + row * D + col,
+             make_float4(s4.x + vj * k4.x, s4.y + vj * k4.y, s4.z + vj * k4.z, s4.w + vj * k4.w));
     }
-  } else {  // new state v k^T in the freed slot (after a merge) or slot m
+  } else {  // the new state v k^T goes to the freed slot (after a merge) or slot m
     const int phys = (jm >= 0) ? sm.slot[jm + 1] : m;
-    float* dst = states + (long long)phys * D * D + row * D + col0;
+    float* dst = states + (long long)phys * D * D;
 #pragma unroll
-    for (int c = 0; c < KPT / 4; ++c) {
-      const int cc = col0 + 4 * c;
-      store4(dst + 4 * c, make_float4(vj * sm.k[cc], vj * sm.k[cc + 1], vj * sm.k[cc + 2], vj * sm.k[cc + 3]));
+    for (int r = 0; r < RPT; ++r) {
+      const int row = rg + r * RG;
+      const float vj = sm.v[row];
+      store4(dst + row * D + col, make_float4(vj * k4.x, vj * k4.y, vj * k4.z, vj * k4.w));
     }
   }
-  if (part == 0) {
+  if (li == 0) {
     Tout* o = reinterpret_cast<Tout*>(a.o) + (long long)bh * D;
-    o[row] = from_f32<Tout>(orow);
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+      const int row = rg + r * RG;
+      o[row] = from_f32<Tout>(acc[r] + wt * qk * sm.v[row]);
+    }
   }
   __syncthreads();
   // ---------------------------------------------------------------- metadata
   if (warp == 0) {
-    const double I = sm.Ival;
+    const double I = (double)sm.Ival;
     if (!bflag) {
       if (lane == 0) {
         sm.n[open] += 1;
@@ -283,6 +274,8 @@ static cudaError_t launch_dec_t(const DecodeArgs& a, cudaStream_t st) {
   const size_t smem = sizeof(DecSmem<D>);
   auto kern = decode_kernel<D, Tin, Tout>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   if (e != cudaSuccess) return e;
   kern<<<a.B * a.H, NT, smem, st>>>(a);
   return cudaGetLastError();

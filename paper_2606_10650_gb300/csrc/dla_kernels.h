@@ -93,6 +93,10 @@ cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, 
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;
+// K2 on tcgen05 / TMEM / TMA (bf16 inputs, d = 128), 128-token intervals,
+// snapshots stored as bf16 hi + lo.
+cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t s);
+constexpr int kReadoutTcInterval = 128;
 cudaError_t launch_decode(const DecodeArgs& a, int d, bool in_bf16, cudaStream_t s);
 cudaError_t launch_init_cache(int32_t* slot, int32_t* n, double* ibar, int32_t* m, int BH, int C,
                               cudaStream_t s);

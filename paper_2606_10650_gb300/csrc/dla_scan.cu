@@ -36,6 +36,7 @@ struct ScanSmem {
   static constexpr int L = kScanL;
   static constexpr int KP = D + 4;  // padded row (floats) of the k / v tiles
   float S[D * D];                   // open state [d_v][d_k]
+  __nv_bfloat16 raw[2][2][L * D];   // bf16 k / v of the next chunk, in flight (bf16 inputs only)
   float K[L * KP];
   float V[L * KP];
   float G[L * (L + 1)];             // G[t][s] = (k_t.k_s)(v_t.v_s), s < t
@@ -43,10 +44,10 @@ struct ScanSmem {
   float a[L];                       // a_t = |k_t|^2 |v_t|^2
   float red[16 * L];                // partial sums
   float wsum[4];
-  double Itok[L];                   // score of every token in the chunk
-  double gpart[NT / 32];            // per-warp partial sums of |S_open|^2
-  double ibar[kMaxC];               // logical metadata of the cache
-  double gam_open;
+  float Itok[L];                    // score of every token in the chunk
+  float gpart[NT / 32];             // per-warp partial sums of |S_open|^2
+  double ibar[kMaxC];               // logical metadata of the cache (summed scores)
+  float gam_open;
   int n[kMaxC];
   int slot[kMaxC];
   int pid[kMaxC];                   // pool id of the entry's latest snapshot
@@ -73,11 +74,44 @@ __device__ __forceinline__ void load_rows(float* dst, const Tin* src, int row_st
   }
 }
 
-// Copies a D x D fp32 state into a pool entry (Tpool), 4 elements per step.
-template <int D, typename Tpool>
-__device__ __forceinline__ void copy_state(Tpool* dst, const float* src) {
+// Starts asynchronous 16-byte copies of `rows` k and v rows (bf16) into the
+// staging buffers; rows >= valid are zero-filled.
+template <int D>
+__device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
+                                            const __nv_bfloat16* vs, int row_stride, int valid) {
+  constexpr int V16 = D / 8;  // 16-byte pieces per row
+  for (int e = threadIdx.x; e < kScanL * V16; e += NT) {
+    const int r = e / V16, c = (e % V16) * 8;
+    const int nbytes = (r < valid) ? 16 : 0;
+    const __nv_bfloat16* sk = (r < valid) ? ks + (long long)r * row_stride + c : ks;
+    const __nv_bfloat16* sv = (r < valid) ? vs + (long long)r * row_stride + c : vs;
+    const uint32_t ak = static_cast<uint32_t>(__cvta_generic_to_shared(dk + r * D + c));
+    const uint32_t av = static_cast<uint32_t>(__cvta_generic_to_shared(dv + r * D + c));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(ak), "l"(sk), "r"(nbytes) : "memory");
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(av), "l"(sv), "r"(nbytes) : "memory");
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+// Copies a D x D fp32 state into a pool entry.  An fp32 pool keeps the value;
+// a bf16 pool stores it as two bf16 matrices hi = bf16(S) and lo = bf16(S - hi)
+// (entry = [hi | lo]), so two bf16 tensor-core products reproduce S q to ~2^-17.
+template <int D>
+__device__ __forceinline__ void copy_state(float* dst, const float* src) {
   for (int e = threadIdx.x * 4; e < D * D; e += NT * 4) store4(dst + e, load4(src + e));
 }
+template <int D>
+__device__ __forceinline__ void copy_state(__nv_bfloat16* dst, const float* src) {
+  for (int e = threadIdx.x * 4; e < D * D; e += NT * 4) {
+    const float4 x = load4(src + e);
+    const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
+    const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+    store4(dst + e, make_float4(f01.x, f01.y, f23.x, f23.y));
+    store4(dst + D * D + e, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
+  }
+}
+template <typename Tpool>
+constexpr int pool_parts() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
 }  // namespace
 
@@ -93,12 +127,13 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   const int bh = blockIdx.x;
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
-  const double Dd = (double)D * (double)D;
+  const float Df = (float)(D * D);
   const Tin* kbase = reinterpret_cast<const Tin*>(a.k) + ((long long)b * a.T * a.H + h) * D;
   const Tin* vbase = reinterpret_cast<const Tin*>(a.v) + ((long long)b * a.T * a.H + h) * D;
   const int row_stride = a.H * D;
   float* states = a.states + (long long)bh * C * D * D;
-  Tpool* pool = a.pool ? reinterpret_cast<Tpool*>(a.pool) + (long long)bh * a.pool_cap * D * D : nullptr;
+  constexpr long long kEntry = (long long)pool_parts<Tpool>() * D * D;  // elements per pool entry
+  Tpool* pool = a.pool ? reinterpret_cast<Tpool*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
   uint8_t* bnd_out = a.boundary + (long long)bh * a.T;
   int32_t* mlog_out = a.merge_log + (long long)bh * a.T;
 
@@ -141,7 +176,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   if (pool) {
     for (int i = 0; i < m_start; ++i) {
       if (i >= a.pool_cap) break;
-      copy_state<D>(pool + (long long)i * D * D, states + (long long)sm.slot[i] * D * D);
+      copy_state<D>(pool + (long long)i * kEntry, states + (long long)sm.slot[i] * D * D);
     }
     if (tid < m_start) sm.pid[tid] = tid;
     if (tid == 0) {
@@ -154,30 +189,54 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
 
   const int ntok = a.t_end - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
+  if constexpr (sizeof(Tin) == 2) {
+    prefetch_kv<D>(sm.raw[0][0], sm.raw[0][1], reinterpret_cast<const __nv_bfloat16*>(kbase) +
+                                                   (long long)a.t_begin * row_stride,
+                   reinterpret_cast<const __nv_bfloat16*>(vbase) + (long long)a.t_begin * row_stride, row_stride,
+                   min(L, ntok));
+  }
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
     const int Lc = min(L, a.t_end - t0);
     // ------------------------------------------------ 1. stage k, v
-    load_rows<D, Tin>(sm.K, kbase + (long long)t0 * row_stride, row_stride, L, Lc);
-    load_rows<D, Tin>(sm.V, vbase + (long long)t0 * row_stride, row_stride, L, Lc);
+    if constexpr (sizeof(Tin) == 2) {
+      // bf16: this chunk was prefetched during the previous one; start the next
+      if (c + 1 < nchunks) {
+        const int t1 = t0 + L;
+        prefetch_kv<D>(sm.raw[(c + 1) & 1][0], sm.raw[(c + 1) & 1][1],
+                       reinterpret_cast<const __nv_bfloat16*>(kbase) + (long long)t1 * row_stride,
+                       reinterpret_cast<const __nv_bfloat16*>(vbase) + (long long)t1 * row_stride, row_stride,
+                       min(L, a.t_end - t1));
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+      } else {
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+      }
+      __syncthreads();
+      load_rows<D, __nv_bfloat16>(sm.K, sm.raw[c & 1][0], D, L, L);
+      load_rows<D, __nv_bfloat16>(sm.V, sm.raw[c & 1][1], D, L, L);
+    } else {
+      load_rows<D, Tin>(sm.K, kbase + (long long)t0 * row_stride, row_stride, L, Lc);
+      load_rows<D, Tin>(sm.V, vbase + (long long)t0 * row_stride, row_stride, L, Lc);
+    }
     if (tid < L) {
       sm.bnd[tid] = 0;
       sm.mlog[tid] = -1;
-      sm.Itok[tid] = 0.0;
+      sm.Itok[tid] = 0.f;
     }
     __syncthreads();
     const int m_chunk = sm.m;
     // ------------------------------------------------ 2. x_t and |S_open|^2
     if (m_chunk > 0) {
-      // gam_open in double: sum of squares of the open state
-      double g = 0.0;
+      // gam_open = |S_open|^2: per-thread partial sums, then a tree (fp32)
+      float g = 0.f;
       for (int e = tid * 4; e < D * D; e += NT * 4) {
         float4 s4 = load4(sm.S + e);
-        g += (double)s4.x * s4.x + (double)s4.y * s4.y + (double)s4.z * s4.z + (double)s4.w * s4.w;
+        g += s4.x * s4.x + s4.y * s4.y + s4.z * s4.z + s4.w * s4.w;
       }
       g = warp_sum(g);
       if (lane == 0) sm.gpart[warp] = g;
-      // x_t: thread = (token block of 4, row block of TJ)
+      // x_t: thread = (tokens tb + 16 i, rows rb*TJ..); rows 16 apart keep the
+      // float4 loads of 16 threads on 8 distinct bank groups
       const int tb = tid % 16, rb = tid / 16;
       float y[4][TJ];
 #pragma unroll
@@ -187,7 +246,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       for (int kk = 0; kk < D; kk += 4) {
         float4 kv[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) kv[i] = load4(sm.K + (tb * 4 + i) * KP + kk);
+        for (int i = 0; i < 4; ++i) kv[i] = load4(sm.K + (tb + 16 * i) * KP + kk);
 #pragma unroll
         for (int r = 0; r < TJ; ++r) {
           float4 s4 = load4(sm.S + (rb * TJ + r) * D + kk);
@@ -200,8 +259,8 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       for (int i = 0; i < 4; ++i) {
         float part = 0.f;
 #pragma unroll
-        for (int r = 0; r < TJ; ++r) part += sm.V[(tb * 4 + i) * KP + rb * TJ + r] * y[i][r];
-        sm.red[rb * L + tb * 4 + i] = part;
+        for (int r = 0; r < TJ; ++r) part += sm.V[(tb + 16 * i) * KP + rb * TJ + r] * y[i][r];
+        sm.red[rb * L + tb + 16 * i] = part;
       }
       __syncthreads();
       if (tid < L) {
@@ -211,17 +270,17 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
         sm.x[tid] = xs;
       }
       if (tid == 0) {
-        double gs = 0.0;
+        float gs = 0.f;
         for (int w = 0; w < NT / 32; ++w) gs += sm.gpart[w];
         sm.gam_open = gs;
       }
     } else {
       if (tid < L) sm.x[tid] = 0.f;
-      if (tid == 0) sm.gam_open = 0.0;
+      if (tid == 0) sm.gam_open = 0.f;
     }
     // ------------------------------------------------ 3. Gram G[t][s] and a_t
     {
-      const int tt = tid / 16, ss = tid % 16;  // 4x4 token tiles
+      const int tt = tid / 16, ss = tid % 16;  // tokens tt + 16 i, ss + 16 j
       float kk4[4][4], vv4[4][4];
 #pragma unroll
       for (int i = 0; i < 4; ++i)
@@ -231,10 +290,10 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
         float4 kt[4], ks[4], vt[4], vs[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          kt[i] = load4(sm.K + (tt * 4 + i) * KP + e);
-          ks[i] = load4(sm.K + (ss * 4 + i) * KP + e);
-          vt[i] = load4(sm.V + (tt * 4 + i) * KP + e);
-          vs[i] = load4(sm.V + (ss * 4 + i) * KP + e);
+          kt[i] = load4(sm.K + (tt + 16 * i) * KP + e);
+          ks[i] = load4(sm.K + (ss + 16 * i) * KP + e);
+          vt[i] = load4(sm.V + (tt + 16 * i) * KP + e);
+          vs[i] = load4(sm.V + (ss + 16 * i) * KP + e);
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i)
@@ -248,7 +307,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          int t = tt * 4 + i, s = ss * 4 + j;
+          int t = tt + 16 * i, s = ss + 16 * j;
           float gv = kk4[i][j] * vv4[i][j];
           sm.G[t * (L + 1) + s] = (s < t) ? gv : 0.f;
           if (s == t) sm.a[t] = gv;
@@ -260,7 +319,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       sm.seg_pre = (m_chunk > 0) ? 1 : 0;
       if (m_chunk == 0) {  // the very first token of an empty cache opens state 0
         sm.bnd[0] = 1;
-        sm.Itok[0] = 0.0;
+        sm.Itok[0] = 0.f;
         sm.cur = 1;
       }
     }
@@ -292,11 +351,10 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
         float excl = inc - w + (warp == 1 ? sm.wsum[0] : 0.f);
         bool fire = false;
         if (t >= cur && t < Lc) {
-          double gam = (pre ? sm.gam_open : 0.0) + (double)excl;
-          ScoreParams sp = a.sp;
-          double I = info_score((double)sm.a[t], (double)beta, gam, Dd, sp);
+          const float gam = (pre ? sm.gam_open : 0.f) + excl;
+          const float I = info_score(sm.a[t], beta, gam, Df, a.sp);
           sm.Itok[t] = I;
-          fire = (I >= sp.tau);
+          fire = ((double)I >= a.sp.tau);
         }
         unsigned bal = __ballot_sync(0xffffffffu, fire);
         if (lane == 0) sm.first_fire[warp] = bal ? (warp * 32 + __ffs(bal) - 1) : L;
@@ -320,15 +378,22 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       int m = sm.m;
       int seg_u0 = 0;
       int nops = 0;
-      for (int t = 0; t < Lc; ++t) {
-        if (!sm.bnd[t]) {
+      int run0 = 0;  // first token of the current run of non-boundary tokens
+      for (int t = 0; t <= Lc; ++t) {
+        if (t < Lc && !sm.bnd[t]) continue;
+        if (t > run0) {  // tokens [run0, t) joined the open state: count and summed score
+          float part = 0.f;
+          for (int u = run0 + lane; u < t; u += 32) part += sm.Itok[u];
+          part = warp_sum(part);
           if (lane == 0) {
-            sm.n[m - 1] += 1;
-            sm.ibar[m - 1] += sm.Itok[t];
+            sm.n[m - 1] += t - run0;
+            sm.ibar[m - 1] += (double)part;
             sm.dirty[m - 1] = 1;
           }
-          continue;
+          __syncwarp();
         }
+        run0 = t + 1;
+        if (t == Lc) break;
         if (m > 0 && lane == 0) {
           sm.ops[nops][0] = OP_CLOSE;
           sm.ops[nops][1] = sm.slot[m - 1];
@@ -375,7 +440,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
         if (lane == 0) {
           sm.slot[m] = phys_new;
           sm.n[m] = 1;
-          sm.ibar[m] = sm.Itok[t];
+          sm.ibar[m] = (double)sm.Itok[t];
           sm.pid[m] = -1;
           sm.dirty[m] = 1;
           sm.mlog[t] = j;
@@ -499,7 +564,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
         const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
         const float* src = srcslot < 0 ? sm.S : states + (long long)srcslot * D * D;
-        copy_state<D>(pool + (long long)p * D * D, src);
+        copy_state<D>(pool + (long long)p * kEntry, src);
       }
       __syncthreads();
     }

@@ -240,6 +240,14 @@ def dla_forward_noalloc(params, q, k, v, lam=None, o=None, cache=None, boundary=
     _check(st)
 
 
+def workspace_status(workspace):
+    """Device status word of the last dla_forward on this workspace (call after
+    synchronising): 0 ok, 5 timeout, 6 device check."""
+    buf, base, _ = workspace
+    off = base - buf.data_ptr()
+    return int(buf[off: off + 4].view(torch.int32).item())
+
+
 def dla_decode_step(params, cache: Cache, q, k, v, lam=None, o=None, boundary=None, merge_idx=None, stream=None):
     """Raw call of dla_decode_step.  q, k, v: [B, H, d]; lam [B, H, C] or None;
     o [B, H, d]; boundary [B, H] uint8; merge_idx [B, H] int32."""

@@ -49,8 +49,9 @@ def run_gpu(w, q, k, v, lam, *, want_o=True, score_mode=0, out_dtype=torch.float
     if ws_bytes is not None:
         buf = torch.empty(ws_bytes + 256, dtype=torch.uint8, device=dev)
         ws = (buf, (buf.data_ptr() + 255) // 256 * 256, ws_bytes)
-    dla.dla_forward(p, qt if want_o else None, kt, vt, lt, o, cache, bnd, ml, workspace=ws)
+    ws = dla.dla_forward(p, qt if want_o else None, kt, vt, lt, o, cache, bnd, ml, workspace=ws)
     torch.cuda.synchronize()
+    assert dla.workspace_status(ws) == 0, "device status word reports a failure"
     return dict(o=None if o is None else o.double().cpu().numpy(), boundary=bnd.cpu().numpy(),
                 merge_log=ml.cpu().numpy(), cache=cache)
 
