@@ -58,12 +58,24 @@ int readout_interval(dla_dtype in_dtype, int d) {
   return use_tc(in_dtype, d) ? dla::kReadoutTcInterval : dla::kReadoutSimtInterval;
 }
 
+// Workspace plan of a forward call.  The read-out needs, for every interval,
+// the list of cache entries at its start (snapshot lists) and a pool holding
+// those entries' states.  Persistent mode: one append-only pool for the whole
+// sequence, so rounds continue it and a scan never waits for a read-out.
+// Reset mode (small workspaces): each round restarts a pool of its own, two
+// pools alternate, and a round copies the live states into its pool first.
 struct FwdPlan {
   int interval;      // tokens per snapshot interval
   int nsnap_total;   // intervals over the whole sequence
   int R;             // intervals per round
-  int pool_cap;      // pool entries per stream per round
-  size_t off_status, off_bnd, off_mlog, off_cache, off_m0, off_ids, off_pool, total;
+  int rounds;
+  int persistent;
+  int nbuf;          // pools (1 persistent, 2 reset with several rounds)
+  int pool_cap;      // pool entries per stream, per pool
+  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram, off_pool,
+      pool_bytes;
+  int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
+  size_t total;
 };
 
 // Bytes per snapshot element: fp32 (CUDA-core read-out) or bf16 hi + lo
@@ -72,7 +84,7 @@ struct FwdPlan {
 // streams, hence the hi/lo pair.
 size_t pool_elt(dla_dtype /*in_dtype*/) { return 4; }
 
-FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
+FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
                  bool with_output, bool need_trace, bool need_cache) {
   FwdPlan P;
   const size_t BH = (size_t)B * H;
@@ -80,21 +92,38 @@ FwdPlan plan_for(int R, const dla_params* p, int B, int T, int H, int d, dla_dty
   P.interval = readout_interval(in_dtype, d);
   P.nsnap_total = (T + P.interval - 1) / P.interval;
   P.R = R;
+  P.rounds = (P.nsnap_total + R - 1) / R;
+  P.persistent = persistent ? 1 : 0;
   const int per_snap = C < P.interval + 1 ? C : P.interval + 1;
-  P.pool_cap = with_output ? C + (R - 1) * per_snap : 0;
+  if (!with_output) {
+    P.nbuf = 0;
+    P.pool_cap = 0;
+  } else if (persistent) {
+    P.nbuf = 1;
+    P.pool_cap = C + (P.nsnap_total - 1) * per_snap;
+  } else {
+    P.nbuf = P.rounds > 1 ? 2 : 1;
+    P.pool_cap = C + (R - 1) * per_snap;
+  }
   size_t off = 0;
-  P.off_status = off; off = align256(off + 256);
-  P.off_bnd = off;    if (need_trace) off = align256(off + BH * T);
-  P.off_mlog = off;   if (need_trace) off = align256(off + BH * T * sizeof(int32_t));
-  P.off_cache = off;  if (need_cache) off = align256(off + cache_layout(B, H, C, d, d).total);
-  P.off_m0 = off;     if (with_output) off = align256(off + BH * R * sizeof(int32_t));
-  P.off_ids = off;    if (with_output) off = align256(off + BH * R * C * sizeof(int32_t));
-  P.off_pool = off;   if (with_output) off = align256(off + BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype));
+  P.off_status = off;    off = align256(off + 256);
+  P.off_bnd = off;       if (need_trace) off = align256(off + BH * T);
+  P.off_mlog = off;      if (need_trace) off = align256(off + BH * T * sizeof(int32_t));
+  P.off_cache = off;     if (need_cache) off = align256(off + cache_layout(B, H, C, d, d).total);
+  P.off_lists_m0 = off;  if (with_output) off = align256(off + BH * P.nsnap_total * sizeof(int32_t));
+  P.off_lists_ids = off; if (with_output) off = align256(off + BH * P.nsnap_total * C * sizeof(int32_t));
+  P.off_pstate = off;    if (with_output) off = align256(off + (BH + BH * C) * sizeof(int32_t));
+  // Gram pre-pass output (bf16 inputs, calls with a read-out): 64x64 + 64 floats per 64-token chunk
+  P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
+  P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * (dla::kScanL * dla::kScanL + dla::kScanL) * 4);
+  P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
+  P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
   return P;
 }
 
-constexpr size_t kPreferredWorkspace = (size_t)8 << 30;  // 8 GiB of read-out staging
+constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
+constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
 
 dla_status check_params(const dla_params* p) {
   if (!p) return fail(DLA_ERR_INVALID_ARG, "params is NULL");
@@ -126,6 +155,39 @@ dla_status check_cache(const dla_cache* c, int B, int H, int C, int d) {
 
 dla_status cuda_fail(cudaError_t e, const char* what) {
   return fail(DLA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// ---- internal streams of the overlapped forward schedule, one set per host
+// thread and device: the scan runs on a high-priority stream, the read-out on
+// a low-priority one, so the scan's few CTAs get SMs first.
+struct StreamSet {
+  cudaStream_t hi = nullptr, lo = nullptr;
+  cudaEvent_t in = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
+  bool ready = false;
+};
+constexpr int kMaxDev = 64;
+thread_local StreamSet g_sets[kMaxDev];
+
+cudaError_t stream_set(StreamSet** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+  StreamSet& S = g_sets[dev];
+  if (!S.ready) {
+    int least = 0, greatest = 0;
+    if ((e = cudaDeviceGetStreamPriorityRange(&least, &greatest)) != cudaSuccess) return e;
+    if ((e = cudaStreamCreateWithPriority(&S.hi, cudaStreamNonBlocking, greatest)) != cudaSuccess) return e;
+    if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
+    for (int i = 0; i < 2; ++i) {
+      if ((e = cudaEventCreateWithFlags(&S.scan_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+      if ((e = cudaEventCreateWithFlags(&S.ro_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
+    S.ready = true;
+  }
+  *out = &S;
+  return cudaSuccess;
 }
 
 // ---- optional per-launch CUDA-event timing (dla_timing_enable / _read)
@@ -269,16 +331,21 @@ dla_status dla_init_cache(const dla_cache* cache, void* stream) {
 static FwdPlan choose_plan(const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype, bool with_output,
                            bool need_trace, bool need_cache, size_t budget) {
   const int nsnap = (T + readout_interval(in_dtype, d) - 1) / readout_interval(in_dtype, d);
-  if (!with_output) return plan_for(1, p, B, T, H, d, in_dtype, false, need_trace, need_cache);
-  int lo = 1, hi = nsnap;
-  FwdPlan best = plan_for(1, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
-  if (best.total > budget) return best;
-  while (lo < hi) {  // largest R whose workspace fits the budget
-    int mid = lo + (hi - lo + 1) / 2;
-    if (plan_for(mid, p, B, T, H, d, in_dtype, true, need_trace, need_cache).total <= budget) lo = mid;
+  if (!with_output) return plan_for(1, false, p, B, T, H, d, in_dtype, false, need_trace, need_cache);
+  // about kTargetRounds rounds, so that all but the last read-out hide behind the scan
+  const int rounds = nsnap < kTargetRounds ? nsnap : kTargetRounds;
+  const int R = (nsnap + rounds - 1) / rounds;
+  FwdPlan pp = plan_for(R, true, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
+  if (pp.total <= budget) return pp;
+  auto reset = [&](int r) { return plan_for(r, false, p, B, T, H, d, in_dtype, true, need_trace, need_cache); };
+  if (reset(R).total <= budget || reset(1).total > budget) return reset(reset(R).total <= budget ? R : 1);
+  int lo = 1, hi = R;  // the largest round that fits
+  while (lo < hi) {
+    const int mid = lo + (hi - lo + 1) / 2;
+    if (reset(mid).total <= budget) lo = mid;
     else hi = mid - 1;
   }
-  return plan_for(lo, p, B, T, H, d, in_dtype, true, need_trace, need_cache);
+  return reset(lo);
 }
 
 size_t dla_forward_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype,
@@ -291,7 +358,7 @@ size_t dla_forward_workspace(const dla_params* p, int B, int T, int H, int dk, i
 size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype,
                                  int with_output) {
   if (!p || B < 1 || T < 1 || H < 1 || dk < 1 || dv < 1) return 0;
-  return plan_for(1, p, B, T, H, dk, in_dtype, with_output != 0, true, true).total;
+  return plan_for(1, false, p, B, T, H, dk, in_dtype, with_output != 0, true, true).total;
 }
 
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv, const void* q,
@@ -357,7 +424,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if (!with_output) {
     sa.t_begin = 0; sa.t_end = T;
     sa.pool = nullptr; sa.pool_cap = 0; sa.nsnap = 1; sa.snap_chunks = 1;
-    e = timed(DLA_K_SCAN, st, [&] { return dla::launch_scan(sa, d, in_bf16, pool_bf16, st); });
+    e = timed(DLA_K_SCAN, st, [&] { return (in_bf16 ? dla::launch_scan_mma(sa, d, pool_bf16, st) : dla::launch_scan(sa, d, false, pool_bf16, st)); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return ok();
   }
@@ -368,23 +435,67 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   ra.B = B; ra.T = T; ra.H = H; ra.C = C;
   ra.boundary = bnd; ra.merge_log = mlog;
   ra.interval = P.interval;
-  sa.pool = ws + P.off_pool; sa.pool_cap = P.pool_cap;
-  sa.snap_m0 = (int32_t*)(ws + P.off_m0); sa.snap_ids = (int32_t*)(ws + P.off_ids);
   sa.snap_chunks = P.interval / dla::kScanL;
-  ra.pool = sa.pool; ra.pool_cap = sa.pool_cap; ra.snap_m0 = sa.snap_m0; ra.snap_ids = sa.snap_ids;
+  sa.pool_cap = P.pool_cap;
+  ra.pool_cap = P.pool_cap;
+  sa.snap_stride = ra.snap_stride = P.nsnap_total;
+  sa.snap_m0 = (int32_t*)(ws + P.off_lists_m0);
+  sa.snap_ids = (int32_t*)(ws + P.off_lists_ids);
+  ra.snap_m0 = sa.snap_m0;
+  ra.snap_ids = sa.snap_ids;
+  sa.pstate = P.persistent ? (int32_t*)(ws + P.off_pstate) : nullptr;
+  sa.gram = P.gram_chunks ? (const float*)(ws + P.off_gram) : nullptr;
+  sa.gram_chunks = P.gram_chunks;
+  // Round r: the scan (high-priority stream) appends to the pool, then the
+  // read-out of round r (low-priority stream) runs while the scan of round
+  // r + 1 proceeds.  In reset mode pool b is reused by round r + 2 only after
+  // the read-out of round r has finished.
+  StreamSet* S = nullptr;
+  if ((e = stream_set(&S)) != cudaSuccess) return cuda_fail(e, "internal streams");
+  if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
+  if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  if (P.gram_chunks) {  // K0: Gram suffix tables of every chunk, on all SMs, ahead of the scan
+    dla::GramArgs ga;
+    ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.out = (float*)(ws + P.off_gram);
+    e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
+    if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+  }
   const int round_tokens = P.R * P.interval;
-  for (int t0 = 0; t0 < T; t0 += round_tokens) {
+  int r = 0;
+  bool used[2] = {false, false};
+  for (int t0 = 0; t0 < T; t0 += round_tokens, ++r) {
     const int t1 = (T - t0 < round_tokens) ? T : t0 + round_tokens;
+    const int bsel = P.persistent ? 0 : (r % 2) % P.nbuf;
+    sa.pool = ws + P.off_pool + (size_t)bsel * P.pool_bytes;
+    ra.pool = sa.pool;
     sa.t_begin = t0; sa.t_end = t1;
     sa.nsnap = (t1 - t0 + P.interval - 1) / P.interval;
-    e = timed(DLA_K_SCAN, st, [&] { return dla::launch_scan(sa, d, in_bf16, pool_bf16, st); });
+    sa.snap_base = ra.snap_base = r * P.R;
+    sa.carry_in = (P.persistent && r > 0) ? 1 : 0;
+    sa.snap_at_end = (P.persistent && t1 < T) ? 1 : 0;
+    if (!P.persistent && used[bsel] && (e = cudaStreamWaitEvent(S->hi, S->ro_done[bsel], 0)) != cudaSuccess)
+      return cuda_fail(e, "stream wait");
+    e = timed(DLA_K_SCAN, S->hi, [&] {
+      return in_bf16 ? dla::launch_scan_mma(sa, d, pool_bf16, S->hi) : dla::launch_scan(sa, d, false, pool_bf16, S->hi);
+    });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    if ((e = cudaEventRecord(S->scan_done[r % 2], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(S->lo, S->scan_done[r % 2], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
-    e = timed(DLA_K_READOUT, st, [&] {
-      return tc ? dla::launch_readout_tc(ra, status, st) : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, st);
+    e = timed(DLA_K_READOUT, S->lo, [&] {
+      return tc ? dla::launch_readout_tc(ra, status, S->lo)
+                : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, S->lo);
     });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+    if ((e = cudaEventRecord(S->ro_done[bsel], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
+    used[bsel] = true;
   }
+  // the caller's stream resumes after the last scan and every read-out
+  if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+  if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  for (int i = 0; i < 2; ++i)
+    if (used[i] && (e = cudaStreamWaitEvent(st, S->ro_done[i], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
   return ok();
 }
 

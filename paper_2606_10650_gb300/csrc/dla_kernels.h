@@ -39,11 +39,27 @@ struct ScanArgs {
   // read-out snapshots (pool == nullptr: no read-out in this call)
   void* pool;
   int pool_cap;          // entries per stream
-  int32_t* snap_m0;      // [B*H][nsnap]
-  int32_t* snap_ids;     // [B*H][nsnap][C]
+  int32_t* snap_m0;      // [B*H][snap_stride]     live entries at each interval start
+  int32_t* snap_ids;     // [B*H][snap_stride][C]  their pool ids (logical order)
+  int snap_stride;       // intervals of the whole sequence
+  int snap_base;         // global index of this round's first interval
   int nsnap;             // snapshot intervals in this round
   int snap_chunks;       // scan chunks per snapshot interval
+  int carry_in;          // 1: the pool continues from the previous round (pstate holds its counters)
+  int snap_at_end;       // 1: also snapshot at this round's last interval end (for the next round)
+  int32_t* pstate;       // [B*H] next free pool entry, then [B*H][C] pool ids of the live entries
+  const float* gram;     // Gram pre-pass output [B*H][gram_chunks][64*64 + 64], or nullptr
+  int gram_chunks;       // 64-token chunks of the whole sequence
   int32_t* status;       // device status word (0 = ok)
+};
+
+// K0: Gram pre-pass over every 64-token chunk of every stream (bf16 inputs).
+struct GramArgs {
+  const void* k;
+  const void* v;
+  int B, T, H;
+  int nchunks;
+  float* out;            // [B*H][nchunks][64*64 + 64]
 };
 
 // K2: read-out of one round, one CTA per (snapshot interval, stream).
@@ -62,6 +78,8 @@ struct ReadoutArgs {
   int pool_cap;
   const int32_t* snap_m0;
   const int32_t* snap_ids;
+  int snap_stride;       // intervals of the whole sequence
+  int snap_base;         // global index of this round's first interval
   int nsnap;
   int interval;          // tokens per snapshot interval
 };
@@ -90,6 +108,9 @@ struct DecodeArgs {
 dla_status set_error(dla_status s, const char* fmt, ...);
 
 cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
+// K1 for bf16 inputs with its contractions on mma.sync (dla_scan_mma.cu).
+cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s);
+cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s);
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;

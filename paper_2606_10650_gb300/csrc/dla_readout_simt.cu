@@ -68,14 +68,14 @@ __global__ void __launch_bounds__(NT, 1) readout_simt_kernel(ReadoutArgs a) {
   const int Lc = min(L, a.t_end - c0);
   const int row_stride = a.H * D;
   const long long tok0 = ((long long)b * a.T + c0) * a.H + h;  // row index of token c0
-  const int m0 = a.snap_m0[(long long)bh * a.nsnap + s];
+  const int m0 = a.snap_m0[(long long)bh * a.snap_stride + a.snap_base + s];
   const uint8_t* bnd = a.boundary + (long long)bh * a.T + c0;
   const int32_t* mlog = a.merge_log + (long long)bh * a.T + c0;
 
   load_rows<D, Tin>(sm.Q, reinterpret_cast<const Tin*>(a.q) + tok0 * D, row_stride, Lc);
   load_rows<D, Tin>(sm.K, reinterpret_cast<const Tin*>(a.k) + tok0 * D, row_stride, Lc);
   load_rows<D, Tin>(sm.V, reinterpret_cast<const Tin*>(a.v) + tok0 * D, row_stride, Lc);
-  for (int i = tid; i < m0; i += NT) sm.ids[i] = a.snap_ids[((long long)bh * a.nsnap + s) * C + i];
+  for (int i = tid; i < m0; i += NT) sm.ids[i] = a.snap_ids[((long long)bh * a.snap_stride + a.snap_base + s) * C + i];
 
   // ---- logical slot of every entry at every token (warp 0)
   if (warp == 0) {

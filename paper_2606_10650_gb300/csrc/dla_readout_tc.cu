@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(NT, 1)
   const int C = a.C;
   const int c0 = a.t_begin + s * L;
   const int Lc = min(L, a.t_end - c0);
-  const int m0 = a.snap_m0[(long long)bh * a.nsnap + s];
+  const int m0 = a.snap_m0[(long long)bh * a.snap_stride + a.snap_base + s];
   volatile int* abort = &sm.abort_flag;
 
   if (tid == 0) {
@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(NT, 1)
     sm.abort_flag = 0;
     fence_mbar_init();
   }
-  for (int i = tid; i < m0; i += NT) sm.ids[i] = a.snap_ids[((long long)bh * a.nsnap + s) * C + i];
+  for (int i = tid; i < m0; i += NT) sm.ids[i] = a.snap_ids[((long long)bh * a.snap_stride + a.snap_base + s) * C + i];
   if (warp == 1) tmem_alloc(&sm.tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();

@@ -172,18 +172,23 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   } else {
     for (int e = tid * 4; e < D * D; e += NT * 4) store4(sm.S + e, make_float4(0.f, 0.f, 0.f, 0.f));
   }
-  // snapshot 0: every live entry as it stands at the start of the round
   if (pool) {
-    for (int i = 0; i < m_start; ++i) {
-      if (i >= a.pool_cap) break;
-      copy_state<D>(pool + (long long)i * kEntry, states + (long long)sm.slot[i] * D * D);
+    const long long lst = (long long)bh * a.snap_stride + a.snap_base;  // list row of this round's first interval
+    if (a.carry_in) {  // the pool continues: the previous round wrote this interval's list
+      if (tid == 0) sm.pool_next = a.pstate[bh];
+      for (int i = tid; i < m_start; i += NT) sm.pid[i] = a.pstate[a.B * a.H + (long long)bh * C + i];
+    } else {  // snapshot 0: every live entry as it stands at the start of the round
+      for (int i = 0; i < m_start; ++i) {
+        if (i >= a.pool_cap) break;
+        copy_state<D>(pool + (long long)i * kEntry, states + (long long)sm.slot[i] * D * D);
+      }
+      if (tid < m_start) sm.pid[tid] = tid;
+      if (tid == 0) {
+        sm.pool_next = m_start;
+        a.snap_m0[lst] = m_start;
+      }
+      for (int i = tid; i < m_start; i += NT) a.snap_ids[lst * C + i] = i;
     }
-    if (tid < m_start) sm.pid[tid] = tid;
-    if (tid == 0) {
-      sm.pool_next = m_start;
-      a.snap_m0[(long long)bh * a.nsnap] = m_start;
-    }
-    for (int i = tid; i < m_start; i += NT) a.snap_ids[((long long)bh * a.nsnap) * C + i] = i;
   }
   __syncthreads();
 
@@ -536,7 +541,8 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
     // ------------------------------------------------ 7. read-out snapshot
     const bool interval_end = ((c + 1) % a.snap_chunks) == 0;
     const int snap_idx = (c + 1) / a.snap_chunks;
-    if (pool && interval_end && snap_idx < a.nsnap) {
+    const long long lrow = (long long)bh * a.snap_stride + a.snap_base + snap_idx;
+    if (pool && interval_end && (snap_idx < a.nsnap || a.snap_at_end)) {
       if (tid == 0) {
         int nj = 0;
         const int m = sm.m;
@@ -555,12 +561,12 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
           }
         }
         sm.nsnapjobs = nj;
-        a.snap_m0[(long long)bh * a.nsnap + snap_idx] = m;
+        a.snap_m0[lrow] = m;
       }
       __syncthreads();
       const int m = sm.m;
       for (int i = tid; i < m; i += NT)
-        a.snap_ids[((long long)bh * a.nsnap + snap_idx) * C + i] = sm.pid[i];
+        a.snap_ids[lrow * C + i] = sm.pid[i];
       for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
         const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
         const float* src = srcslot < 0 ? sm.S : states + (long long)srcslot * D * D;
@@ -582,6 +588,10 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
       a.ibar[(long long)bh * C + i] = (i < m) ? sm.ibar[i] : 0.0;
     }
     if (tid == 0) a.m[bh] = m;
+    if (pool && a.pstate) {  // counters for a following round that continues this pool
+      if (tid == 0) a.pstate[bh] = sm.pool_next;
+      for (int i = tid; i < m; i += NT) a.pstate[a.B * a.H + (long long)bh * C + i] = sm.pid[i];
+    }
   }
 }
 

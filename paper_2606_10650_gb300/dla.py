@@ -22,7 +22,7 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
             "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc"]
-KERNELS = ["scan", "readout", "decode", "init"]
+KERNELS = ["scan", "readout", "decode", "init", "gram"]
 
 
 class DLAError(RuntimeError):
@@ -119,10 +119,11 @@ def dla_timing_enable(enable=True):
 def dla_timing_read(reset=True):
     """{kernel kind: (launches, summed ms)} of the launches recorded since the
     last reset (see dla_timing_enable)."""
-    n = (ctypes.c_int * 4)()
-    ms = (ctypes.c_double * 4)()
+    k = len(KERNELS)
+    n = (ctypes.c_int * k)()
+    ms = (ctypes.c_double * k)()
     _check(lib().dla_timing_read(n, ms, int(bool(reset))))
-    return {KERNELS[i]: (n[i], ms[i]) for i in range(4)}
+    return {KERNELS[i]: (n[i], ms[i]) for i in range(k)}
 
 
 def dla_cache_bytes(B, H, C, dk, dv):
