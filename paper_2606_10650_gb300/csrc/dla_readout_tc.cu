@@ -44,8 +44,11 @@ struct TcSmem {
   uint8_t Q[2][kTile];         // A operand, two k-halves                      32 KB
   uint8_t st[2][2][2][kTile];  // [stage][hi/lo][k-half]; stage 0 = A, 1 = B  128 KB
   uint8_t Pt[2][kTile];        // lambda-weighted P, A operand [t][s]           32 KB
-  unsigned char tab[L * MAXE];  // logical slot of entry x at token t           24 KB
+  unsigned char tab[(L + 1) * MAXE];  // logical slot of entry x after event e    24 KB
   int ent[L];                   // entry holding token s
+  int evt[L];                   // events (boundaries) at or before token t
+  uint8_t bnd[L];               // the interval's boundary flags
+  int mlog[L];                  // and merge indices
   int ids[kMaxC];               // pool ids of the snapshot entries
   uint64_t bar_qk, bar_p, bar_pt, bar_o, bar_done;
   uint64_t full[2], empty[2], acc_full[2], acc_empty[2];
@@ -178,47 +181,88 @@ __global__ void __launch_bounds__(NT, 1)
     const long long rowbase = ((long long)b * a.T + c0) * a.H + h;  // row index of token c0
     const __nv_bfloat16* vg = reinterpret_cast<const __nv_bfloat16*>(a.v);
 
-    // V^T into stage A, part 1, as the K-major B operand [j][s] (s = K index)
-    for (int e = etid; e < L * (D / 8); e += NEPI * 32) {
-      const int ss = e / (D / 8), j0 = (e % (D / 8)) * 8;
-      uint4 raw = make_uint4(0, 0, 0, 0);
-      if (ss < Lc) raw = *reinterpret_cast<const uint4*>(vg + (rowbase + (long long)ss * a.H) * D + j0);
-      const __nv_bfloat16* vv = reinterpret_cast<const __nv_bfloat16*>(&raw);
-      uint8_t* tile = sm.st[0][1][ss >> 6];
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        *reinterpret_cast<__nv_bfloat16*>(tile + sw128_offset(j0 + i, ss & 63)) = vv[i];
+    // the interval's boundary flags and merge indices, staged once
+    if (etid < L) {
+      const bool in = etid < Lc;
+      sm.bnd[etid] = in ? a.boundary[(long long)bh * a.T + c0 + etid] : (uint8_t)0;
+      sm.mlog[etid] = in ? a.merge_log[(long long)bh * a.T + c0 + etid] : -1;
     }
-    // logical slot table (one warp, in token order)
-    if (ew == 0) {
-      int* logi = reinterpret_cast<int*>(sm.Pt[0]);  // scratch until Pt is written
-      for (int x = lane; x < MAXE; x += 32) logi[x] = (x < m0) ? x : -1;
-      __syncwarp();
-      const uint8_t* bnd = a.boundary + (long long)bh * a.T + c0;
-      const int32_t* mlog = a.merge_log + (long long)bh * a.T + c0;
-      int nent = m0, cnt = m0, open = m0 - 1;
-      for (int tt = 0; tt < Lc; ++tt) {
-        if (bnd[tt]) {
-          const int j = mlog[tt];
-          if (j >= 0) {
-            for (int x = lane; x < nent; x += 32)
-              if (logi[x] > j) logi[x] -= 1;
-            cnt -= 1;
-          }
-          __syncwarp();
-          if (lane == 0) logi[nent] = cnt;
-          open = nent;
-          nent += 1;
-          cnt += 1;
-          __syncwarp();
-        }
-        if (lane == 0) sm.ent[tt] = open;
-        for (int x = lane; x < nent; x += 32) sm.tab[tt * MAXE + x] = (unsigned char)logi[x];
-        __syncwarp();
+    // V^T into stage A, part 1, as the K-major B operand [j][s] (s = K index);
+    // each thread issues its eight 16-byte loads before any store
+    {
+      constexpr int PER = L * (D / 8) / (NEPI * 32);
+      uint4 raw[PER];
+#pragma unroll
+      for (int i = 0; i < PER; ++i) {
+        const int e = etid + i * NEPI * 32;
+        const int ss = e / (D / 8), j0 = (e % (D / 8)) * 8;
+        raw[i] = make_uint4(0, 0, 0, 0);
+        if (ss < Lc) raw[i] = *reinterpret_cast<const uint4*>(vg + (rowbase + (long long)ss * a.H) * D + j0);
+      }
+#pragma unroll
+      for (int i = 0; i < PER; ++i) {
+        const int e = etid + i * NEPI * 32;
+        const int ss = e / (D / 8), j0 = (e % (D / 8)) * 8;
+        const __nv_bfloat16* vv = reinterpret_cast<const __nv_bfloat16*>(&raw[i]);
+        uint8_t* tile = sm.st[0][1][ss >> 6];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          *reinterpret_cast<__nv_bfloat16*>(tile + sw128_offset(j0 + u, ss & 63)) = vv[u];
       }
     }
     asm volatile("bar.sync 1, 256;" ::: "memory");
+    // logical slot table, one row per boundary event (one warp): row e holds
+    // L(x) after the first e events of the interval; token t reads row evt[t]
+    if (ew == 0) {
+      int* logi = reinterpret_cast<int*>(sm.Pt[0]);  // scratch until Pt is written
+      for (int x = lane; x < MAXE; x += 32) {
+        logi[x] = (x < m0) ? x : -1;
+        if (x < m0) sm.tab[x] = (unsigned char)x;
+      }
+      __syncwarp();
+      unsigned long long lo64 = 0, hi64 = 0;
+#pragma unroll
+      for (int w4 = 0; w4 < 4; ++w4) {
+        const unsigned m = __ballot_sync(0xffffffffu, sm.bnd[32 * w4 + lane] != 0);
+        if (w4 < 2) lo64 |= (unsigned long long)m << (32 * w4);
+        else hi64 |= (unsigned long long)m << (32 * (w4 - 2));
+      }
+      int nent = m0, cnt = m0, ev = 0;
+      while (lo64 | hi64) {
+        const int tt = lo64 ? (__ffsll((long long)lo64) - 1) : (64 + __ffsll((long long)hi64) - 1);
+        if (lo64) lo64 &= lo64 - 1; else hi64 &= hi64 - 1;
+        const int j = sm.mlog[tt];
+        if (j >= 0) {
+          for (int x = lane; x < nent; x += 32)
+            if (logi[x] > j) logi[x] -= 1;
+          cnt -= 1;
+        }
+        __syncwarp();
+        if (lane == 0) logi[nent] = cnt;
+        nent += 1;
+        cnt += 1;
+        ev += 1;
+        __syncwarp();
+        for (int x = lane; x < nent; x += 32) sm.tab[ev * MAXE + x] = (unsigned char)logi[x];
+        __syncwarp();
+      }
+    }
+    // events at or before each token, and the entry holding it
+    if (etid < L) {  // warps 2..5, one token per lane
+      const int tt = etid;
+      int e = 0;
+#pragma unroll
+      for (int w4 = 0; w4 < 4; ++w4) {
+        const unsigned m = __ballot_sync(0xffffffffu, sm.bnd[32 * w4 + lane] != 0);
+        if (32 * w4 + 31 <= tt) e += __popc(m);
+        else if (32 * w4 <= tt) e += __popc(m & (0xffffffffu >> (31 - (tt - 32 * w4))));
+      }
+      sm.evt[tt] = e;
+      sm.ent[tt] = (e == 0) ? m0 - 1 : m0 + e - 1;
+    }
+    asm volatile("bar.sync 1, 256;" ::: "memory");
     const float* lam_t = (a.lam && t < Lc) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
+    const int evt_t = sm.evt[t];
     // ---- Pt = P * lambda_{t, L_t(e(s))} for s <= t (bf16), s in this warp's half
     if (mbar_wait(&sm.bar_p, 0, abort, status)) {
       tc_fence_after();
@@ -238,7 +282,7 @@ __global__ void __launch_bounds__(NT, 1)
             const int ss = 64 * ch + sl;
             float w = 0.f;
             if (ss <= t && t < Lc) {
-              const int li = sm.tab[t * MAXE + sm.ent[ss]];
+              const int li = sm.tab[evt_t * MAXE + sm.ent[ss]];
               w = lam_t ? lam_t[li] : 1.f;
             }
             w2[u] = p[sl] * w;
@@ -263,12 +307,18 @@ __global__ void __launch_bounds__(NT, 1)
       tmem_ld32(lane_addr + COL_O + 64 * ch, o);
       tmem_ld32(lane_addr + COL_O + 64 * ch + 32, o + 32);
     }
+    // weight of state x for this token; fetched one state ahead of its use
+    auto weight = [&](int x) -> float {
+      if (t >= Lc || x >= m0) return 0.f;
+      return lam_t ? lam_t[sm.tab[evt_t * MAXE + x]] : 1.f;
+    };
+    float w_next = weight(0);
     for (int x = 0; x < m0; ++x) {
       const int buf = x & 1, kb = x >> 1;
+      const float w = w_next;
+      w_next = weight(x + 1);
       if (!mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status)) break;
       tc_fence_after();
-      float w = 0.f;
-      if (t < Lc) w = lam_t ? lam_t[sm.tab[t * MAXE + x]] : 1.f;
       float dv[32];
       const uint32_t base = lane_addr + COL_S + 128u * buf + 64 * ch;
       tmem_ld32(base, dv);
