@@ -72,8 +72,8 @@ struct FwdPlan {
   int persistent;
   int nbuf;          // pools (1 persistent, 2 reset with several rounds)
   int pool_cap;      // pool entries per stream, per pool
-  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram, off_pool,
-      pool_bytes;
+  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram, off_ointra,
+      off_pool, pool_bytes;
   int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
   size_t total;
 };
@@ -116,6 +116,8 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // Gram pre-pass output (bf16 inputs, calls with a read-out): 64x64 + 64 floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * (dla::kScanL * dla::kScanL + dla::kScanL) * 4);
+  // intra-interval read-out part of one round (tensor-core read-out), fp32
+  P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + BH * (size_t)R * P.interval * d * 4);
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
@@ -446,6 +448,8 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   sa.pstate = P.persistent ? (int32_t*)(ws + P.off_pstate) : nullptr;
   sa.gram = P.gram_chunks ? (const float*)(ws + P.off_gram) : nullptr;
   sa.gram_chunks = P.gram_chunks;
+  ra.ointra = tc ? (float*)(ws + P.off_ointra) : nullptr;
+  ra.ointra_T = P.R * P.interval;
   // Round r: the scan (high-priority stream) appends to the pool, then the
   // read-out of round r (low-priority stream) runs while the scan of round
   // r + 1 proceeds.  In reset mode pool b is reused by round r + 2 only after
@@ -483,6 +487,10 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     if ((e = cudaEventRecord(S->scan_done[r % 2], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(S->lo, S->scan_done[r % 2], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
+    if (tc) {  // K2a, then K2b on the same stream (K2b starts from K2a's output)
+      e = timed(DLA_K_READOUT_INTRA, S->lo, [&] { return dla::launch_readout_intra(ra, S->lo); });
+      if (e != cudaSuccess) return cuda_fail(e, "intra read-out launch");
+    }
     e = timed(DLA_K_READOUT, S->lo, [&] {
       return tc ? dla::launch_readout_tc(ra, status, S->lo)
                 : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, S->lo);

@@ -82,6 +82,8 @@ struct ReadoutArgs {
   int snap_base;         // global index of this round's first interval
   int nsnap;
   int interval;          // tokens per snapshot interval
+  float* ointra;         // [B*H][ointra_T][d] fp32 intra-interval part (tensor-core path), token t - t_begin
+  int ointra_T;          // tokens per stream in ointra (one round)
 };
 
 // K3: one decode step of every stream.
@@ -114,8 +116,11 @@ cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s);
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;
-// K2 on tcgen05 / TMEM / TMA (bf16 inputs, d = 128), 128-token intervals,
-// snapshots stored as bf16 hi + lo.
+// K2 for bf16 inputs, d = 128, 128-token intervals, in two launches:
+// K2a (mma.sync) writes the intra-interval part to a.ointra; K2b (tcgen05 /
+// TMEM / TMA, snapshots stored as bf16 hi + lo) adds the snapshot part and
+// writes o.
+cudaError_t launch_readout_intra(const ReadoutArgs& a, cudaStream_t s);
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t s);
 constexpr int kReadoutTcInterval = 128;
 cudaError_t launch_decode(const DecodeArgs& a, int d, bool in_bf16, cudaStream_t s);

@@ -12,6 +12,7 @@
 // Shapes per 64-token chunk: X is 64 x d x d, the Grams 2 x 64 x 64 x d and the
 // build d x d x 64, i.e. about 6 d^2 * 64 flop, a few thousand mma per CTA.
 #include "dla_common.cuh"
+#include "dla_mma.cuh"
 
 namespace dla {
 
@@ -52,30 +53,6 @@ struct MmaSmem {
   int nops, nsnapjobs;
   int m, cur, js, seg_pre, pool_next;
 };
-
-__device__ __forceinline__ uint32_t su32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
-
-__device__ __forceinline__ void ldsm4(uint32_t* r, const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(su32(p)));
-}
-__device__ __forceinline__ void ldsm4t(uint32_t* r, const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(su32(p)));
-}
-__device__ __forceinline__ void ldsm2(uint32_t* r, const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(su32(p)));
-}
-// c (16x8 fp32) += a (16x16 bf16, row) * b (16x8 bf16, col)
-__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 
 // Keep the bf16 halves of a packed pair whose token index lies in [u0, u1).
 __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1) {
