@@ -4,6 +4,7 @@
 // the forward pass and the kernel launches.  Every compute step runs in the
 // kernels of dla_scan.cu / dla_readout_*.cu / dla_decode.cu.
 #include <math.h>
+#include <algorithm>
 #include <stdarg.h>
 #include <vector>
 #include <stdio.h>
@@ -124,6 +125,23 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   return P;
 }
 
+// Interval counts of the rounds, in order.  Rounds of at most R intervals,
+// balanced; in persistent mode followed by a taper of R/2, R/4, R/8 intervals,
+// so that the read-out left to run after the last scan is short.
+std::vector<int> round_sizes(const FwdPlan& P) {
+  std::vector<int> out, tail;
+  int left = P.nsnap_total;
+  if (P.persistent)
+    for (int s = P.R / 2; s >= 1 && s >= P.R / 8 && left - s >= P.R; s /= 2) {
+      tail.push_back(s);
+      left -= s;
+    }
+  const int n = (left + P.R - 1) / P.R;
+  for (int i = 0; i < n; ++i) out.push_back(left / n + (i < left % n ? 1 : 0));
+  out.insert(out.end(), tail.begin(), tail.end());
+  return out;
+}
+
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
 
@@ -164,7 +182,7 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
 // a low-priority one, so the scan's few CTAs get SMs first.
 struct StreamSet {
   cudaStream_t hi = nullptr, lo = nullptr;
-  cudaEvent_t in = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
+  cudaEvent_t in = nullptr, gram_done = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
   bool ready = false;
 };
 constexpr int kMaxDev = 64;
@@ -182,6 +200,7 @@ cudaError_t stream_set(StreamSet** out) {
     if ((e = cudaStreamCreateWithPriority(&S.hi, cudaStreamNonBlocking, greatest)) != cudaSuccess) return e;
     if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&S.gram_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     for (int i = 0; i < 2; ++i) {
       if ((e = cudaEventCreateWithFlags(&S.scan_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
       if ((e = cudaEventCreateWithFlags(&S.ro_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
@@ -458,27 +477,43 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = stream_set(&S)) != cudaSuccess) return cuda_fail(e, "internal streams");
   if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
   if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
-  if (P.gram_chunks) {  // K0: Gram suffix tables of every chunk, on all SMs, ahead of the scan
+  const std::vector<int> sizes = round_sizes(P);
+  bool gram_rest = false;  // the scan of round 1 waits for the Gram tables of rounds 1..
+  if (P.gram_chunks) {
+    // K0: Gram suffix tables.  Round 0's chunks run ahead of the first scan on
+    // the scan stream; the rest run on the read-out stream while that scan goes.
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
     ga.out = (float*)(ws + P.off_gram);
+    const int first = std::min(P.gram_chunks, sizes[0] * P.interval / dla::kScanL);
+    ga.chunk0 = 0; ga.count = first;
     e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+    if (first < P.gram_chunks) {
+      ga.chunk0 = first; ga.count = P.gram_chunks - first;
+      if ((e = cudaStreamWaitEvent(S->lo, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+      e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
+      if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+      if ((e = cudaEventRecord(S->gram_done, S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
+      gram_rest = true;
+    }
   }
-  const int round_tokens = P.R * P.interval;
-  int r = 0;
   bool used[2] = {false, false};
-  for (int t0 = 0; t0 < T; t0 += round_tokens, ++r) {
-    const int t1 = (T - t0 < round_tokens) ? T : t0 + round_tokens;
+  int snap0 = 0;  // global index of the round's first interval
+  for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
+    const int t0 = snap0 * P.interval;
+    const int t1 = std::min(T, t0 + sizes[r] * P.interval);
     const int bsel = P.persistent ? 0 : (r % 2) % P.nbuf;
     sa.pool = ws + P.off_pool + (size_t)bsel * P.pool_bytes;
     ra.pool = sa.pool;
     sa.t_begin = t0; sa.t_end = t1;
     sa.nsnap = (t1 - t0 + P.interval - 1) / P.interval;
-    sa.snap_base = ra.snap_base = r * P.R;
+    sa.snap_base = ra.snap_base = snap0;
     sa.carry_in = (P.persistent && r > 0) ? 1 : 0;
     sa.snap_at_end = (P.persistent && t1 < T) ? 1 : 0;
     if (!P.persistent && used[bsel] && (e = cudaStreamWaitEvent(S->hi, S->ro_done[bsel], 0)) != cudaSuccess)
+      return cuda_fail(e, "stream wait");
+    if (r == 1 && gram_rest && (e = cudaStreamWaitEvent(S->hi, S->gram_done, 0)) != cudaSuccess)
       return cuda_fail(e, "stream wait");
     e = timed(DLA_K_SCAN, S->hi, [&] {
       return in_bf16 ? dla::launch_scan_mma(sa, d, pool_bf16, S->hi) : dla::launch_scan(sa, d, false, pool_bf16, S->hi);

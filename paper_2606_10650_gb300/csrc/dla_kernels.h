@@ -58,7 +58,8 @@ struct GramArgs {
   const void* k;
   const void* v;
   int B, T, H;
-  int nchunks;
+  int nchunks;           // chunks of the whole sequence
+  int chunk0, count;     // this launch: chunks chunk0 .. chunk0 + count - 1
   float* out;            // [B*H][nchunks][64*64 + 64]
 };
 

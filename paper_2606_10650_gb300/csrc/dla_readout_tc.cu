@@ -154,14 +154,15 @@ __global__ void __launch_bounds__(NT, 1)
       sm.bnd[etid] = in ? a.boundary[(long long)bh * a.T + c0 + etid] : (uint8_t)0;
       sm.mlog[etid] = in ? a.merge_log[(long long)bh * a.T + c0 + etid] : -1;
     }
-    // o starts from the intra-interval part (K2a)
+    // o starts from the intra-interval part (K2a; column-quad order, so a warp
+    // reads 512 contiguous bytes per load)
     float o[64];
     {
-      const float* src = a.ointra + ((long long)bh * a.ointra_T + (c0 - a.t_begin) + t) * D + 64 * ch;
+      const float* src = a.ointra + ((long long)bh * a.ointra_T + (c0 - a.t_begin)) * D + (16 * ch * L + t) * 4;
 #pragma unroll
       for (int i = 0; i < 64; i += 4) {
         float4 v4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (t < Lc) v4 = *reinterpret_cast<const float4*>(src + i);
+        if (t < Lc) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
         o[i] = v4.x; o[i + 1] = v4.y; o[i + 2] = v4.z; o[i + 3] = v4.w;
       }
     }

@@ -26,21 +26,21 @@ constexpr int kGramBlock = L * L + L;  // floats per chunk of the Gram pre-pass 
 
 enum : int { OP_CLOSE = 0, OP_MERGE = 1 };
 
-template <int D>
+template <int D, int CL>
 struct MmaSmem {
   static constexpr int RP = D + 8;  // padded bf16 row: 8 rows of a ldmatrix hit 8 bank groups
   static constexpr int GS = L + 4;  // suffix-table row (16-byte aligned for cp.async)
   __nv_bfloat16 kv[2][2][L * RP];   // [stage][k / v][t][RP]
-  __nv_bfloat16 S2[2][D * RP];      // open state as bf16 hi / lo, [j][RP]
+  __nv_bfloat16 S2[2][D / CL * RP]; // this CTA's rows of the open state as bf16 hi / lo, [j][RP]
   float gs[2][L * GS];              // [stage] suffix table sg[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s)
   float as[2][L];                   // [stage] a_t = |k_t|^2 |v_t|^2
   float G[L * (L + 1)];             // Gram rows, when the scan forms them itself
   float red[NW][L];
+  float xs[2][L + 4];               // [chunk parity] this CTA's part of x_t (t < L) and of |S_open|^2 (at L)
   float gred[NW];
   float wsum[4];
   float Itok[L];
   double ibar[kMaxC];
-  float gam_open;
   int n[kMaxC];
   int slot[kMaxC];
   int pid[kMaxC];
@@ -150,12 +150,14 @@ __device__ __forceinline__ void suffix_rows(float* G) {
   }
 }
 
-// State copies move D*D/4/NT float4 per thread; loads are issued in batches of
-// four before their stores so that a copy costs a few memory latencies, not one
-// per element (the compiler cannot reorder a load past a possibly aliasing store).
-template <int D>
+// State copies (NR rows of a D x D state) move NR*D/4/NT float4 per thread;
+// loads are issued in batches of four before their stores so that a copy costs
+// a few memory latencies, not one per element (the compiler cannot reorder a
+// load past a possibly aliasing store).  A bf16 pool entry is hi rows [D][D]
+// followed by lo rows [D][D]: dst points at this CTA's first hi row.
+template <int D, int NR = D>
 __device__ __forceinline__ void copy_state_g(float* dst, const float* src) {
-  constexpr int PER = D * D / 4 / NT;
+  constexpr int PER = NR * D / 4 / NT;
   for (int base = 0; base < PER; base += 4) {
     float4 v[4];
 #pragma unroll
@@ -164,9 +166,9 @@ __device__ __forceinline__ void copy_state_g(float* dst, const float* src) {
     for (int i = 0; i < 4; ++i) store4(dst + ((base + i) * NT + threadIdx.x) * 4, v[i]);
   }
 }
-template <int D>
+template <int D, int NR = D>
 __device__ __forceinline__ void copy_state_g(__nv_bfloat16* dst, const float* src) {
-  constexpr int PER = D * D / 4 / NT;
+  constexpr int PER = NR * D / 4 / NT;
   for (int base = 0; base < PER; base += 4) {
     float4 v[4];
 #pragma unroll
@@ -183,9 +185,9 @@ __device__ __forceinline__ void copy_state_g(__nv_bfloat16* dst, const float* sr
   }
 }
 // dst += src over one D x D state, batched like copy_state_g.
-template <int D>
+template <int D, int NR = D>
 __device__ __forceinline__ void add_state_g(float* dst, const float* src) {
-  constexpr int PER = D * D / 4 / NT;
+  constexpr int PER = NR * D / 4 / NT;
   for (int base = 0; base < PER; base += 4) {
     float4 x[4], y[4];
 #pragma unroll
@@ -201,15 +203,9 @@ __device__ __forceinline__ void add_state_g(float* dst, const float* src) {
   }
 }
 
-// One pair of adjacent state elements (k, k+1 of row j) into a pool entry.
+// One pair of adjacent state elements (k, k+1 of row j) into an fp32 pool entry.
 __device__ __forceinline__ void put_pair(float* entry, int D, int j, int k, float v0, float v1) {
   *reinterpret_cast<float2*>(entry + j * D + k) = make_float2(v0, v1);
-}
-__device__ __forceinline__ void put_pair(__nv_bfloat16* entry, int D, int j, int k, float v0, float v1) {
-  const __nv_bfloat162 hi = __floats2bfloat162_rn(v0, v1);
-  const float2 f = __bfloat1622float2(hi);
-  *reinterpret_cast<__nv_bfloat162*>(entry + j * D + k) = hi;
-  *reinterpret_cast<__nv_bfloat162*>(entry + D * D + j * D + k) = __floats2bfloat162_rn(v0 - f.x, v1 - f.y);
 }
 
 template <typename Tpool>
@@ -217,34 +213,49 @@ constexpr int parts_of() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
 }  // namespace
 
-template <int D, typename Tpool>
+// One stream per CTA (CL = 1) or per CTA pair (CL = 2, a thread-block
+// cluster): with a pair, each CTA owns d/2 rows of the open state (and of every
+// state it copies or adds), forms its part of x_t and |S_open|^2, and the two
+// parts meet through distributed shared memory once per chunk; both CTAs then
+// take the same decisions from the same sums (x = part of rank 0 + part of
+// rank 1 in both), and rank 0 writes the trace, the lists and the metadata.
+template <int D, typename Tpool, int CL>
 __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   constexpr int RP = D + 8;
-  constexpr int MT = D / 16;          // 16-row bands of the state
-  constexpr int WPM = NW / MT;        // warps per band (1 for d = 128, 2 for d = 64)
+  constexpr int R = D / CL;           // state rows of this CTA
+  constexpr int MT = R / 16;          // 16-row bands of those rows
+  constexpr int WPM = NW / MT;        // warps per band
   constexpr int KC = D / WPM;         // state columns per warp
   constexpr int NT8 = KC / 8;         // n8 tiles per warp in the state build
-  constexpr int NJ8 = D / 8 / NW;     // n8 tiles per warp in the x GEMM
+  constexpr int NJ8 = R / 8 / NW;     // n8 tiles per warp in the x GEMM
+  static_assert(NJ8 == 1 || NJ8 == 2, "x GEMM tiling");
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  MmaSmem<D>& sm = *reinterpret_cast<MmaSmem<D>*>(smem_raw);
+  MmaSmem<D, CL>& sm = *reinterpret_cast<MmaSmem<D, CL>*>(smem_raw);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g = lane >> 2, tg = lane & 3;
-  const int bh = blockIdx.x;
+  const int rank = (CL > 1) ? (int)cluster_rank() : 0;
+  const bool lead = (rank == 0);      // writes what both CTAs of a pair hold
+  const int bh = blockIdx.x / CL;
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const float Df = (float)(D * D);
   const __nv_bfloat16* kbase = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
   const __nv_bfloat16* vbase = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
   const int row_stride = a.H * D;
+  const int rbase = rank * R;         // first state row of this CTA
   float* states = a.states + (long long)bh * C * D * D;
   constexpr long long kEntry = (long long)parts_of<Tpool>() * D * D;
   Tpool* pool = a.pool ? reinterpret_cast<Tpool*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
   uint8_t* bnd_out = a.boundary + (long long)bh * a.T;
   int32_t* mlog_out = a.merge_log + (long long)bh * a.T;
+  // this CTA's rows of state slot p
+  auto srows = [&](int p) { return states + (long long)p * D * D + (long long)rbase * D; };
 
-  // this warp's band of the open state: rows j0 .. j0+15, columns k0 .. k0+KC-1
+  // this warp's band of the open state: local rows j0 .. j0+15 (global rbase + j0 ..),
+  // columns k0 .. k0+KC-1
   const int j0 = 16 * (warp % MT), k0 = KC * (warp / MT);
+  const int jg0 = rbase + j0;
   float acc[NT8][4];
 
   // ---------------------------------------------------------------- round start
@@ -279,8 +290,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const int k = k0 + 8 * n + 2 * tg;
       float2 lo = make_float2(0.f, 0.f), hi = make_float2(0.f, 0.f);
       if (src) {
-        lo = *reinterpret_cast<const float2*>(src + (j0 + g) * D + k);
-        hi = *reinterpret_cast<const float2*>(src + (j0 + g + 8) * D + k);
+        lo = *reinterpret_cast<const float2*>(src + (jg0 + g) * D + k);
+        hi = *reinterpret_cast<const float2*>(src + (jg0 + g + 8) * D + k);
       }
       acc[n][0] = lo.x; acc[n][1] = lo.y; acc[n][2] = hi.x; acc[n][3] = hi.y;
     }
@@ -292,18 +303,19 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       for (int i = tid; i < m_start; i += NT) sm.pid[i] = a.pstate[a.B * a.H + (long long)bh * C + i];
     } else {  // snapshot 0: every live entry at the start of the round
       for (int i = 0; i < m_start && i < a.pool_cap; ++i)
-        copy_state_g<D>(pool + (long long)i * kEntry, states + (long long)sm.slot[i] * D * D);
+        copy_state_g<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]));
       if (tid < m_start) sm.pid[tid] = tid;
-      if (tid == 0) {
-        sm.pool_next = m_start;
-        a.snap_m0[lst] = m_start;
+      if (tid == 0) sm.pool_next = m_start;
+      if (lead) {
+        if (tid == 0) a.snap_m0[lst] = m_start;
+        for (int i = tid; i < m_start; i += NT) a.snap_ids[lst * C + i] = i;
       }
-      for (int i = tid; i < m_start; i += NT) a.snap_ids[lst * C + i] = i;
     }
   }
 
-  // open state -> bf16 hi / lo operand and |S_open|^2, from the accumulators
-  auto publish_state = [&]() {
+  // this CTA's rows of the open state -> bf16 hi / lo operand, and its part of
+  // |S_open|^2 into xs[buf][L]
+  auto publish_state = [&](int buf) {
     float gp = 0.f;
 #pragma unroll
     for (int n = 0; n < NT8; ++n) {
@@ -325,7 +337,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     if (tid == 0) {
       float gs = 0.f;
       for (int w = 0; w < NW; ++w) gs += sm.gred[w];
-      sm.gam_open = gs;
+      sm.xs[buf][L] = gs;
     }
   };
   // acc += V^T K over chunk tokens [u0, u1) of stage st
@@ -337,7 +349,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const int t0 = 16 * ks;
       if (t0 >= u1 || t0 + 16 <= u0) continue;
       uint32_t af[4];
-      ldsm4t(af, Vs + (t0 + (q >> 1) * 8 + r8) * RP + j0 + (q & 1) * 8);
+      ldsm4t(af, Vs + (t0 + (q >> 1) * 8 + r8) * RP + jg0 + (q & 1) * 8);
       af[0] = mask_pair(af[0], t0 + 2 * tg, u0, u1);
       af[1] = mask_pair(af[1], t0 + 2 * tg, u0, u1);
       af[2] = mask_pair(af[2], t0 + 8 + 2 * tg, u0, u1);
@@ -351,8 +363,16 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
   };
+  // x_t or |S_open|^2 of the whole state: the CTAs' parts added in rank order
+  auto whole = [&](const float* p) -> float {
+    if constexpr (CL == 1) {
+      return *p;
+    } else {
+      return dsmem_ld(p, 0) + dsmem_ld(p, 1);
+    }
+  };
 
-  publish_state();
+  publish_state(0);
   __syncthreads();
 
   const int ntok = a.t_end - a.t_begin;
@@ -385,7 +405,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     const __nv_bfloat16* Ks = sm.kv[st][0];
     const __nv_bfloat16* Vs = sm.kv[st][1];
     const int q = lane >> 3, r8 = lane & 7;
-    // ------------------------------------------------ 2. x_t = v_t^T S_open k_t
+    // ------------------------------------------------ 2. x_t = v_t^T S_open k_t (this CTA's rows)
     if (m_chunk > 0) {
       float X[4][NJ8][4];
 #pragma unroll
@@ -394,7 +414,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         for (int nj = 0; nj < NJ8; ++nj)
 #pragma unroll
           for (int e = 0; e < 4; ++e) X[mt][nj][e] = 0.f;
-      const int jb = warp * 8 * NJ8;
+      const int jb = warp * 8 * NJ8;  // local rows of this warp
       for (int kk = 0; kk < D; kk += 16) {
         uint32_t bh_[4], bl_[4];
         if constexpr (NJ8 == 2) {
@@ -415,13 +435,13 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           }
         }
       }
-      // x partial over this warp's j columns: sum_j v_t[j] X[t][j]
+      // x partial over this warp's j rows: sum_j v_t[j] X[t][j]
 #pragma unroll
       for (int mt = 0; mt < 4; ++mt) {
         float p0 = 0.f, p1 = 0.f;  // rows g and g + 8 of the tile
 #pragma unroll
         for (int nj = 0; nj < NJ8; ++nj) {
-          const int j = jb + 8 * nj + 2 * tg;
+          const int j = rbase + jb + 8 * nj + 2 * tg;
           const int ta = 16 * mt + g, tb8 = ta + 8;
           const float2 va = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Vs + ta * RP + j));
           const float2 vb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Vs + tb8 * RP + j));
@@ -452,6 +472,18 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
     __syncthreads();
+    if (tid < L) {  // this CTA's part of x_t
+      float x = 0.f;
+      if (m_chunk > 0)
+#pragma unroll
+        for (int w8 = 0; w8 < NW; ++w8) x += sm.red[w8][tid];
+      sm.xs[st][tid] = x;
+    }
+    if constexpr (CL > 1) {
+      cluster_sync();
+    } else {
+      __syncthreads();
+    }
     // ------------------------------------------------ 4. boundary passes (warps 0-1, token t = tid)
     // Each pass scores every undecided token as if the open segment ran to it,
     // takes the first that fires, and restarts the segment there.  Only the
@@ -466,10 +498,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         }
         cur = 1;
       }
-      float xt = 0.f;
-      if (m_chunk > 0)
-#pragma unroll
-        for (int w8 = 0; w8 < NW; ++w8) xt += sm.red[w8][t];
+      const float xt = (m_chunk > 0) ? whole(&sm.xs[st][t]) : 0.f;
+      const float gam_open = (m_chunk > 0) ? whole(&sm.xs[st][L]) : 0.f;
       const float at = sm.as[st][t];
       const float* gst = sm.gs[st];
       while (cur < Lc) {
@@ -489,7 +519,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         const float excl = inc - w + (warp == 1 ? sm.wsum[0] : 0.f);
         bool fire = false;
         if (t >= cur && t < Lc) {
-          const float gam = (pre ? sm.gam_open : 0.f) + excl;
+          const float gam = (pre ? gam_open : 0.f) + excl;
           const float I = info_score(at, beta, gam, Df, a.sp);
           sm.Itok[t] = I;
           fire = ((double)I >= a.sp.tau);
@@ -593,7 +623,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
     __syncthreads();
-    // ------------------------------------------------ 6. state updates
+    // ------------------------------------------------ 6. state updates (this CTA's rows)
     {
       const int nops = sm.nops;
       for (int op = 0; op < nops; ++op) {
@@ -604,22 +634,22 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 #pragma unroll
           for (int n = 0; n < NT8; ++n) {
             const int k = k0 + 8 * n + 2 * tg;
-            *reinterpret_cast<float2*>(dst + (j0 + g) * D + k) = make_float2(acc[n][0], acc[n][1]);
-            *reinterpret_cast<float2*>(dst + (j0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
+            *reinterpret_cast<float2*>(dst + (jg0 + g) * D + k) = make_float2(acc[n][0], acc[n][1]);
+            *reinterpret_cast<float2*>(dst + (jg0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
             acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
           }
         } else {
-          add_state_g<D>(states + (long long)sm.ops[op][1] * D * D, states + (long long)sm.ops[op][2] * D * D);
+          add_state_g<D, R>(srows(sm.ops[op][1]), srows(sm.ops[op][2]));
         }
         __syncthreads();
       }
       build(st, sm.js, Lc);  // the chunk's tail joins the open state
     }
-    if (tid < Lc) {
+    if (lead && tid < Lc) {
       bnd_out[t0 + tid] = (uint8_t)sm.bnd[tid];
       mlog_out[t0 + tid] = sm.mlog[tid];
     }
-    publish_state();  // operand of the next chunk's x GEMM and |S_open|^2
+    publish_state(st ^ 1);  // operand of the next chunk's x GEMM and |S_open|^2
     __syncthreads();
     // ------------------------------------------------ 7. read-out snapshot
     const bool interval_end = ((c + 1) % a.snap_chunks) == 0;
@@ -634,16 +664,16 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           const bool need = (i < m) && (sm.dirty[i] || sm.pid[i] < 0);
           const unsigned bal = __ballot_sync(0xffffffffu, need);
           if (need) {
-            const int rank = nj + __popc(bal & ((1u << lane) - 1u));
-            int p = sm.pool_next + rank;
+            const int rank_ = nj + __popc(bal & ((1u << lane) - 1u));
+            int p = sm.pool_next + rank_;
             if (p >= a.pool_cap) {  // cannot happen with a correctly sized workspace
               atomicExch(a.status, 6);
               p = a.pool_cap - 1;
             }
             sm.pid[i] = p;
             sm.dirty[i] = 0;
-            sm.snap_src[rank][0] = p;
-            sm.snap_src[rank][1] = (i == m - 1) ? -1 : sm.slot[i];
+            sm.snap_src[rank_][0] = p;
+            sm.snap_src[rank_][1] = (i == m - 1) ? -1 : sm.slot[i];
           }
           nj += __popc(bal);
         }
@@ -651,34 +681,35 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         if (lane == 0) {
           sm.pool_next += nj;
           sm.nsnapjobs = nj;
-          a.snap_m0[lrow] = m;
+          if (lead) a.snap_m0[lrow] = m;
         }
       }
       __syncthreads();
       const int m = sm.m;
-      for (int i = tid; i < m; i += NT) a.snap_ids[lrow * C + i] = sm.pid[i];
+      if (lead)
+        for (int i = tid; i < m; i += NT) a.snap_ids[lrow * C + i] = sm.pid[i];
       for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
         const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
         Tpool* entry = pool + (long long)p * kEntry;
         if (srcslot < 0) {  // the open state
           if constexpr (sizeof(Tpool) == 2) {
             // bf16 hi / lo are already staged in shared memory: coalesced 16-byte copies
-            for (int e = tid; e < 2 * D * (D / 8); e += NT) {
-              const int part = e / (D * (D / 8)), rem = e % (D * (D / 8));
+            for (int e = tid; e < 2 * R * (D / 8); e += NT) {
+              const int part = e / (R * (D / 8)), rem = e % (R * (D / 8));
               const int j = rem / (D / 8), k8 = (rem % (D / 8)) * 8;
-              *reinterpret_cast<uint4*>(entry + part * D * D + j * D + k8) =
+              *reinterpret_cast<uint4*>(entry + part * D * D + (rbase + j) * D + k8) =
                   *reinterpret_cast<const uint4*>(&sm.S2[part][j * RP + k8]);
             }
           } else {  // fp32 pool: straight from the accumulators
 #pragma unroll
             for (int n = 0; n < NT8; ++n) {
               const int k = k0 + 8 * n + 2 * tg;
-              put_pair(entry, D, j0 + g, k, acc[n][0], acc[n][1]);
-              put_pair(entry, D, j0 + g + 8, k, acc[n][2], acc[n][3]);
+              put_pair(entry, D, jg0 + g, k, acc[n][0], acc[n][1]);
+              put_pair(entry, D, jg0 + g + 8, k, acc[n][2], acc[n][3]);
             }
           }
         } else {
-          copy_state_g<D>(entry, states + (long long)srcslot * D * D);
+          copy_state_g<D, R>(entry + (long long)rbase * D, srows(srcslot));
         }
       }
       __syncthreads();
@@ -692,21 +723,24 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 #pragma unroll
       for (int n = 0; n < NT8; ++n) {
         const int k = k0 + 8 * n + 2 * tg;
-        *reinterpret_cast<float2*>(dst + (j0 + g) * D + k) = make_float2(acc[n][0], acc[n][1]);
-        *reinterpret_cast<float2*>(dst + (j0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
+        *reinterpret_cast<float2*>(dst + (jg0 + g) * D + k) = make_float2(acc[n][0], acc[n][1]);
+        *reinterpret_cast<float2*>(dst + (jg0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
       }
     }
-    for (int i = tid; i < C; i += NT) {
-      a.slot[(long long)bh * C + i] = sm.slot[i];
-      a.n[(long long)bh * C + i] = (i < m) ? sm.n[i] : 0;
-      a.ibar[(long long)bh * C + i] = (i < m) ? sm.ibar[i] : 0.0;
-    }
-    if (tid == 0) a.m[bh] = m;
-    if (pool && a.pstate) {  // counters for a following round that continues this pool
-      if (tid == 0) a.pstate[bh] = sm.pool_next;
-      for (int i = tid; i < m; i += NT) a.pstate[a.B * a.H + (long long)bh * C + i] = sm.pid[i];
+    if (lead) {
+      for (int i = tid; i < C; i += NT) {
+        a.slot[(long long)bh * C + i] = sm.slot[i];
+        a.n[(long long)bh * C + i] = (i < m) ? sm.n[i] : 0;
+        a.ibar[(long long)bh * C + i] = (i < m) ? sm.ibar[i] : 0.0;
+      }
+      if (tid == 0) a.m[bh] = m;
+      if (pool && a.pstate) {  // counters for a following round that continues this pool
+        if (tid == 0) a.pstate[bh] = sm.pool_next;
+        for (int i = tid; i < m; i += NT) a.pstate[a.B * a.H + (long long)bh * C + i] = sm.pid[i];
+      }
     }
   }
+  if constexpr (CL > 1) cluster_sync();  // the partner may still read this CTA's shared memory
 }
 
 // K0: Gram pre-pass.  One CTA per (64-token chunk, stream): the suffix table
@@ -727,7 +761,7 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   constexpr int RP = D + 8;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   GramSmem<D>& sm = *reinterpret_cast<GramSmem<D>*>(smem_raw);
-  const int c = blockIdx.x, bh = blockIdx.y;
+  const int c = a.chunk0 + blockIdx.x, bh = blockIdx.y;
   const int b = bh / a.H, h = bh % a.H;
   const int t0 = c * L;
   const int valid = min(L, a.T - t0);
@@ -766,7 +800,7 @@ static cudaError_t launch_gram_t(const GramArgs& a, cudaStream_t s) {
   auto kern = gram_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid(a.nchunks, a.B * a.H);
+  dim3 grid(a.count, a.B * a.H);
   kern<<<grid, NT, smem, s>>>(a);
   return cudaGetLastError();
 }
@@ -775,19 +809,42 @@ cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s) {
   return d == 128 ? launch_gram_t<128>(a, s) : launch_gram_t<64>(a, s);
 }
 
-template <int D, typename Tpool>
+template <int D, typename Tpool, int CL>
 static cudaError_t launch_scan_mma_t(const ScanArgs& a, cudaStream_t s) {
-  const size_t smem = sizeof(MmaSmem<D>);
-  auto kern = scan_mma_kernel<D, Tpool>;
+  const size_t smem = sizeof(MmaSmem<D, CL>);
+  auto kern = scan_mma_kernel<D, Tpool, CL>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<a.B * a.H, NT, smem, s>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B * a.H * CL);
+  cfg.blockDim = dim3(NT);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = CL > 1 ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+// CTA pairs when two CTAs per stream still fit on the device in one wave.
+static bool use_pairs(const ScanArgs& a) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  return 2LL * a.B * a.H <= sms;
 }
 
 cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s) {
-  if (d == 128) return pool_bf16 ? launch_scan_mma_t<128, __nv_bfloat16>(a, s) : launch_scan_mma_t<128, float>(a, s);
-  return pool_bf16 ? launch_scan_mma_t<64, __nv_bfloat16>(a, s) : launch_scan_mma_t<64, float>(a, s);
+  if (d == 128) {
+    if (use_pairs(a))
+      return pool_bf16 ? launch_scan_mma_t<128, __nv_bfloat16, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);
+    return pool_bf16 ? launch_scan_mma_t<128, __nv_bfloat16, 1>(a, s) : launch_scan_mma_t<128, float, 1>(a, s);
+  }
+  return pool_bf16 ? launch_scan_mma_t<64, __nv_bfloat16, 1>(a, s) : launch_scan_mma_t<64, float, 1>(a, s);
 }
 
 }  // namespace dla

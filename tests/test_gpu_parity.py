@@ -35,6 +35,8 @@ CASES = {
     "long_churn_bf16": ("long", dict(B=1, H=2, T=1500, block=256)),
     "d64_bf16": ("standard", dict(B=2, H=2, T=700, d=64, C=8, tau=1.4215)),
     "d128_fp32": ("tiny", dict(B=1, H=2, T=300, d=128, C=6, tau=1.4142)),
+    # more streams than CTA pairs fit on the device: one scan CTA per stream
+    "many_streams_bf16": ("regime", dict(B=3, H=27, T=300, C=3, tau=1.2)),
 }
 
 
