@@ -114,9 +114,9 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   P.off_lists_m0 = off;  if (with_output) off = align256(off + BH * P.nsnap_total * sizeof(int32_t));
   P.off_lists_ids = off; if (with_output) off = align256(off + BH * P.nsnap_total * C * sizeof(int32_t));
   P.off_pstate = off;    if (with_output) off = align256(off + (BH + BH * C) * sizeof(int32_t));
-  // Gram pre-pass output (bf16 inputs, calls with a read-out): 64x64 + 64 floats per 64-token chunk
+  // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramBlock floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
-  P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * (dla::kScanL * dla::kScanL + dla::kScanL) * 4);
+  P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
   // intra-interval read-out part of one round (tensor-core read-out), fp32
   P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + BH * (size_t)R * P.interval * d * 4);
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
@@ -141,6 +141,20 @@ std::vector<int> round_sizes(const FwdPlan& P) {
   out.insert(out.end(), tail.begin(), tail.end());
   return out;
 }
+
+}  // namespace
+
+namespace dla {
+void finish_score_params(ScoreParams& sp) {
+  float t = (float)sp.tau;
+  if ((double)t < sp.tau) t = nextafterf(t, INFINITY);
+  sp.tau_f = t;
+  sp.eps_f = (float)sp.eps;
+  sp.rms_eps_f = (float)sp.rms_eps;
+}
+}  // namespace dla
+
+namespace {
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
@@ -435,6 +449,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   sa.k = k; sa.v = v;
   sa.B = B; sa.T = T; sa.H = H;
   sa.sp.tau = p->tau; sa.sp.eps = p->eps; sa.sp.rms_eps = p->rms_eps; sa.sp.score_mode = p->score_mode;
+  dla::finish_score_params(sa.sp);
   sa.C = C;
   sa.states = live.states; sa.slot = live.slot; sa.n = live.n; sa.ibar = live.ibar; sa.m = live.m;
   sa.boundary = bnd; sa.merge_log = mlog;
@@ -559,6 +574,7 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
   da.out_bf16 = (p->out_dtype == DLA_BF16);
   da.B = cache->B; da.H = cache->H; da.C = cache->C;
   da.sp.tau = p->tau; da.sp.eps = p->eps; da.sp.rms_eps = p->rms_eps; da.sp.score_mode = p->score_mode;
+  dla::finish_score_params(da.sp);
   da.states = cache->states; da.slot = cache->slot; da.n = cache->n; da.ibar = cache->ibar; da.m = cache->m;
   da.boundary = boundary; da.merge_idx = merge_idx;
   cudaError_t e = timed(DLA_K_DECODE, (cudaStream_t)stream,

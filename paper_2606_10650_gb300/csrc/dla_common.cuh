@@ -42,6 +42,34 @@ __device__ __forceinline__ float info_score(float a, float beta, float gam, floa
   return sqrtf(fmaxf(num2, 0.f)) / (y + (float)p.eps);
 }
 
+// The same score as info_score, from hardware reciprocal square roots and an
+// approximate divide (a few ulp; invD = 1 / D).  For the latency-bound
+// boundary passes of the scan: each pass waits on one score per token.
+__device__ __forceinline__ float info_score_fast(float a, float beta, float gam, float invD, const ScoreParams& p) {
+  float AA, BB, AB;
+  if (p.score_mode == 1) {
+    AA = gam + 2.f * beta + a;
+    BB = gam;
+    AB = gam + beta;
+  } else {
+    AA = a;
+    BB = gam;
+    AB = beta;
+  }
+  AA = fmaxf(AA, 0.f);
+  BB = fmaxf(BB, 0.f);
+  const float re = p.rms_eps_f;
+  const float rA = rsqrtf(AA), rB = rsqrtf(BB);
+  const float sA = rsqrtf(fmaf(AA, invD, re)), sB = rsqrtf(fmaf(BB, invD, re));
+  // |N(A)| = sqrt(AA) / sqrt(AA / D + re), likewise for B; c = <A, B> / (|A| |B|)
+  const float x = (AA > 0.f) ? AA * rA * sA : 0.f;
+  const float y = (BB > 0.f) ? BB * rB * sB : 0.f;
+  const float c = (AA > 0.f && BB > 0.f) ? fminf(fmaxf(AB * rA * rB, -1.f), 1.f) : 0.f;
+  const float num2 = fmaxf((x - y) * (x - y) + 2.f * x * y * (1.f - c), 0.f);
+  const float nrm = (num2 > 0.f) ? num2 * rsqrtf(num2) : 0.f;
+  return __fdividef(nrm, y + p.eps_f);
+}
+
 template <typename T>
 __device__ __forceinline__ float to_f32(T x);
 template <>

@@ -12,12 +12,21 @@ namespace dla {
 
 constexpr int kMaxC = 64;   // largest supported capacity C
 constexpr int kScanL = 64;  // tokens per scan chunk (K1)
+// Floats per chunk of the Gram pre-pass output: suffix table gs[j][t], its
+// prefix table Q[j][t] and a_t (see GramArgs).
+constexpr int kGramBlock = 2 * kScanL * kScanL + kScanL;
 
 // Method parameters of the score / boundary test (Sec. 3.1).
 struct ScoreParams {
   double tau, eps, rms_eps;
   int score_mode;
+  // fp32 copies: tau_f is the smallest float >= tau, so that for a float score
+  // I >= tau_f exactly when (double) I >= tau; eps_f, rms_eps_f rounded to nearest
+  float tau_f, eps_f, rms_eps_f;
 };
+
+// Fills the fp32 fields of sp from its fp64 ones (host).
+void finish_score_params(ScoreParams& sp);
 
 // K1: sequential scan of one round [t_begin, t_end) of every stream.
 struct ScanArgs {
@@ -48,19 +57,23 @@ struct ScanArgs {
   int carry_in;          // 1: the pool continues from the previous round (pstate holds its counters)
   int snap_at_end;       // 1: also snapshot at this round's last interval end (for the next round)
   int32_t* pstate;       // [B*H] next free pool entry, then [B*H][C] pool ids of the live entries
-  const float* gram;     // Gram pre-pass output [B*H][gram_chunks][64*64 + 64], or nullptr
+  const float* gram;     // Gram pre-pass output [B*H][gram_chunks][kGramBlock], or nullptr
   int gram_chunks;       // 64-token chunks of the whole sequence
   int32_t* status;       // device status word (0 = ok)
 };
 
 // K0: Gram pre-pass over every 64-token chunk of every stream (bf16 inputs).
+// Per chunk, with G_ts = (k_t.k_s)(v_t.v_s):
+//   gs[j][t] = sum_{j <= s < t} G_ts       (beta_t of a segment opened at j, without S)
+//   Q[j][t]  = sum_{j <= u < t} gs[j][u]   (their running sum over the segment)
+//   a_t      = G_tt
 struct GramArgs {
   const void* k;
   const void* v;
   int B, T, H;
   int nchunks;           // chunks of the whole sequence
   int chunk0, count;     // this launch: chunks chunk0 .. chunk0 + count - 1
-  float* out;            // [B*H][nchunks][64*64 + 64]
+  float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64)
 };
 
 // K2: read-out of one round, one CTA per (snapshot interval, stream).

@@ -42,13 +42,18 @@ __device__ __forceinline__ uint32_t cluster_rank() {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-// The float at the same shared-memory offset as p in the CTA of the cluster with rank r.
-__device__ __forceinline__ float dsmem_ld(const float* p, uint32_t r) {
-  uint32_t remote;
-  float v;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(su32(p)), "r"(r));
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
-  return v;
+// Address of the same shared-memory location as p in the CTA of the cluster with rank r.
+__device__ __forceinline__ uint32_t mapa_u32(const void* p, uint32_t r) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(su32(p)), "r"(r));
+  return a;
+}
+// Asynchronous store of v into another CTA's shared memory (cluster address
+// raddr); completes 4 bytes of transactions on that CTA's mbarrier rbar.
+__device__ __forceinline__ void st_async_f32(uint32_t raddr, float v, uint32_t rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+               "r"(__float_as_uint(v)), "r"(rbar)
+               : "memory");
 }
 
 }  // namespace dla

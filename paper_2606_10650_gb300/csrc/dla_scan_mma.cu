@@ -13,6 +13,7 @@
 // build d x d x 64, i.e. about 6 d^2 * 64 flop, a few thousand mma per CTA.
 #include "dla_common.cuh"
 #include "dla_mma.cuh"
+#include "dla_sm100.cuh"
 
 namespace dla {
 
@@ -22,7 +23,6 @@ constexpr int NT = 256;
 constexpr int NW = NT / 32;
 constexpr int L = kScanL;
 constexpr int GS = L + 4;          // row of a suffix table in shared memory
-constexpr int kGramBlock = L * L + L;  // floats per chunk of the Gram pre-pass output
 
 enum : int { OP_CLOSE = 0, OP_MERGE = 1 };
 
@@ -32,24 +32,20 @@ struct MmaSmem {
   static constexpr int GS = L + 4;  // suffix-table row (16-byte aligned for cp.async)
   __nv_bfloat16 kv[2][2][L * RP];   // [stage][k / v][t][RP]
   __nv_bfloat16 S2[2][D / CL * RP]; // this CTA's rows of the open state as bf16 hi / lo, [j][RP]
-  float gs[2][L * GS];              // [stage] suffix table sg[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s)
+  float gs[2][L * GS];              // [stage] suffix table gs[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s)
+  float Qs[2][L * GS];              // [stage] prefix table Q[j][t] = sum_{j <= u < t} gs[j][u]
   float as[2][L];                   // [stage] a_t = |k_t|^2 |v_t|^2
-  float G[L * (L + 1)];             // Gram rows, when the scan forms them itself
   float red[NW][L];
-  float xs[2][L + 4];               // [chunk parity] this CTA's part of x_t (t < L) and of |S_open|^2 (at L)
+  float xs[2][CL][L + 4];           // [chunk parity][CTA] parts of x_t (t < L) and of |S_open|^2 (at L)
+  uint64_t xbar[2];                 // [chunk parity] the partner's parts have arrived (CTA pairs)
+  int abort_flag;                   // a wait for the partner gave up
   float gred[NW];
-  float wsum[4];
-  float Itok[L];
-  double ibar[kMaxC];
-  int n[kMaxC];
-  int slot[kMaxC];
-  int pid[kMaxC];
-  int dirty[kMaxC];
+  int slot[kMaxC];                  // physical slots at the round start
+  int open_slot;                    // physical slot of the open entry (m - 1) after the last replay
   int bnd[L];
   int mlog[L];
   int ops[3 * L + 4][4];
   int snap_src[kMaxC][2];
-  int first_fire[2];
   int nops, nsnapjobs;
   int m, cur, js, seg_pre, pool_next;
 };
@@ -64,7 +60,7 @@ __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1)
 template <int D>
 __device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
                                             const __nv_bfloat16* vs, int row_stride, int valid, float* dgs,
-                                            float* das, const float* gsrc) {
+                                            float* dqs, float* das, const float* gsrc) {
   constexpr int RP = D + 8;
   constexpr int V16 = D / 8;
   for (int e = threadIdx.x; e < L * V16; e += NT) {
@@ -77,12 +73,14 @@ __device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dv + r * RP + c)), "l"(sv), "r"(nbytes)
                  : "memory");
   }
-  if (gsrc) {  // suffix table [j][t] (64 x 64) and a_t of this chunk from the Gram pre-pass
-    for (int e = threadIdx.x; e < L * (L / 4) + L / 4; e += NT) {
-      const bool is_a = e >= L * (L / 4);
-      const int r = is_a ? 0 : e / (L / 4), c4 = is_a ? (e - L * (L / 4)) * 4 : (e % (L / 4)) * 4;
-      float* dst = is_a ? das + c4 : dgs + r * GS + c4;
-      const float* src = is_a ? gsrc + L * L + c4 : gsrc + r * L + c4;
+  if (gsrc) {  // suffix table gs, prefix table Q (64 x 64 each, [j][t]) and a_t from the Gram pre-pass
+    constexpr int R4 = L / 4;  // 16-byte pieces per row
+    for (int e = threadIdx.x; e < 2 * L * R4 + R4; e += NT) {
+      const int tab = e / (L * R4);  // 0: gs, 1: Q, 2: a
+      const int rem = e - tab * L * R4;
+      const int r = rem / R4, c4 = (rem % R4) * 4;
+      float* dst = (tab == 2) ? das + c4 : (tab == 0 ? dgs : dqs) + r * GS + c4;
+      const float* src = gsrc + tab * L * L + r * L + c4;
       asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(su32(dst)), "l"(src) : "memory");
     }
   }
@@ -150,6 +148,25 @@ __device__ __forceinline__ void suffix_rows(float* G) {
   }
 }
 
+// Exclusive prefix sums along rows: dst[j * ds + t] = sum_{u < t} src[j * rs + u * cs]
+// (a warp per row j, two elements per lane).
+__device__ __forceinline__ void prefix_rows(const float* src, int rs, int cs, float* dst, int ds) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int j = warp; j < L; j += NW) {
+    const float g0 = src[j * rs + (2 * lane) * cs], g1 = src[j * rs + (2 * lane + 1) * cs];
+    float inc = g0 + g1;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float up = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += up;
+    }
+    float ex = __shfl_up_sync(0xffffffffu, inc, 1);
+    if (lane == 0) ex = 0.f;
+    dst[j * ds + 2 * lane] = ex;
+    dst[j * ds + 2 * lane + 1] = ex + g0;
+  }
+}
+
 // State copies (NR rows of a D x D state) move NR*D/4/NT float4 per thread;
 // loads are issued in batches of four before their stores so that a copy costs
 // a few memory latencies, not one per element (the compiler cannot reorder a
@@ -211,6 +228,27 @@ __device__ __forceinline__ void put_pair(float* entry, int D, int j, int k, floa
 template <typename Tpool>
 constexpr int parts_of() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
+// Cache metadata of the live entries, held in registers by one warp: entry i
+// in lane i % 32, element i / 32 (C <= 64).  i is warp-uniform.
+template <typename T>
+__device__ __forceinline__ T entry_get(const T (&f)[2], int i) {
+  return __shfl_sync(0xffffffffu, (i < 32) ? f[0] : f[1], i & 31);
+}
+template <typename T>
+__device__ __forceinline__ void entry_set(T (&f)[2], int i, T v) {
+  if ((i & 31) == (int)(threadIdx.x & 31)) {
+    if (i < 32) f[0] = v;
+    else f[1] = v;
+  }
+}
+// Entry i + 1's field for both of this lane's entries (i = lane, lane + 32).
+template <typename T>
+__device__ __forceinline__ void entry_next(const T (&f)[2], T (&nx)[2]) {
+  const int lane = threadIdx.x & 31;
+  nx[0] = __shfl_sync(0xffffffffu, lane == 0 ? f[1] : f[0], (lane + 1) & 31);
+  nx[1] = __shfl_down_sync(0xffffffffu, f[1], 1);
+}
+
 }  // namespace
 
 // One stream per CTA (CL = 1) or per CTA pair (CL = 2, a thread-block
@@ -267,6 +305,12 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     }
     sm.m = m0;
     sm.pool_next = 0;
+    sm.abort_flag = 0;
+    if constexpr (CL > 1) {
+      sm100::mbar_init(&sm.xbar[0], 1);
+      sm100::mbar_init(&sm.xbar[1], 1);
+      sm100::fence_mbar_init();
+    }
   }
   __syncthreads();
   for (int i = tid; i < C; i += NT) {
@@ -276,13 +320,25 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       sl = i;
     }
     sm.slot[i] = sl;
-    sm.n[i] = a.n[(long long)bh * C + i];
-    sm.ibar[i] = a.ibar[(long long)bh * C + i];
-    sm.pid[i] = -1;
-    sm.dirty[i] = 0;
   }
   __syncthreads();
   const int m_start = sm.m;
+  if (tid == 0) sm.open_slot = (m_start > 0) ? sm.slot[m_start - 1] : 0;  // rewritten by every replay
+  // Warp 0 keeps n, Ibar, physical slot, pool id and "changed since the last
+  // snapshot" of every entry in registers (entry i: lane i % 32, element i / 32).
+  int e_n[2] = {0, 0}, e_slot[2] = {0, 0}, e_pid[2] = {-1, -1}, e_dirty[2] = {0, 0};
+  double e_ib[2] = {0.0, 0.0};
+  if (warp == 0) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int i = lane + 32 * r;
+      if (i < C) {
+        e_n[r] = a.n[(long long)bh * C + i];
+        e_ib[r] = a.ibar[(long long)bh * C + i];
+        e_slot[r] = sm.slot[i];
+      }
+    }
+  }
   {
     const float* src = m_start > 0 ? states + (long long)sm.slot[m_start - 1] * D * D : nullptr;
 #pragma unroll
@@ -300,11 +356,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     const long long lst = (long long)bh * a.snap_stride + a.snap_base;  // list row of this round's first interval
     if (a.carry_in) {  // the pool continues: the previous round wrote this interval's list
       if (tid == 0) sm.pool_next = a.pstate[bh];
-      for (int i = tid; i < m_start; i += NT) sm.pid[i] = a.pstate[a.B * a.H + (long long)bh * C + i];
+      if (warp == 0)
+#pragma unroll
+        for (int r = 0; r < 2; ++r)
+          if (lane + 32 * r < m_start) e_pid[r] = a.pstate[a.B * a.H + (long long)bh * C + lane + 32 * r];
     } else {  // snapshot 0: every live entry at the start of the round
       for (int i = 0; i < m_start && i < a.pool_cap; ++i)
         copy_state_g<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]));
-      if (tid < m_start) sm.pid[tid] = tid;
+      if (warp == 0)
+#pragma unroll
+        for (int r = 0; r < 2; ++r)
+          if (lane + 32 * r < m_start) e_pid[r] = lane + 32 * r;
       if (tid == 0) sm.pool_next = m_start;
       if (lead) {
         if (tid == 0) a.snap_m0[lst] = m_start;
@@ -314,7 +376,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   }
 
   // this CTA's rows of the open state -> bf16 hi / lo operand, and its part of
-  // |S_open|^2 into xs[buf][L]
+  // |S_open|^2 into xs[buf][rank][L]
   auto publish_state = [&](int buf) {
     float gp = 0.f;
 #pragma unroll
@@ -337,7 +399,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     if (tid == 0) {
       float gs = 0.f;
       for (int w = 0; w < NW; ++w) gs += sm.gred[w];
-      sm.xs[buf][L] = gs;
+      sm.xs[buf][rank][L] = gs;
     }
   };
   // acc += V^T K over chunk tokens [u0, u1) of stage st
@@ -363,15 +425,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
   };
-  // x_t or |S_open|^2 of the whole state: the CTAs' parts added in rank order
-  auto whole = [&](const float* p) -> float {
+  // x_t or |S_open|^2 of the whole state (index i of xs[buf][.]): the CTAs'
+  // parts added in rank order
+  auto whole = [&](int buf, int i) -> float {
     if constexpr (CL == 1) {
-      return *p;
+      return sm.xs[buf][0][i];
     } else {
-      return dsmem_ld(p, 0) + dsmem_ld(p, 1);
+      return sm.xs[buf][0][i] + sm.xs[buf][1][i];
     }
   };
 
+  if constexpr (CL > 1) cluster_sync();  // both CTAs run (barriers initialised) before the first exchange
   publish_state(0);
   __syncthreads();
 
@@ -379,7 +443,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const int nchunks = (ntok + L - 1) / L;
   const long long gchunk0 = (long long)bh * a.gram_chunks + a.t_begin / L;  // Gram block of the round's first chunk
   prefetch_kv<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
-                 vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gs[0], sm.as[0],
+                 vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gs[0], sm.Qs[0], sm.as[0],
                  a.gram ? a.gram + gchunk0 * kGramBlock : nullptr);
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
@@ -390,16 +454,12 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const int t1 = t0 + L;
       prefetch_kv<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
                      vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gs[st ^ 1],
-                     sm.as[st ^ 1], a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr);
+                     sm.Qs[st ^ 1], sm.as[st ^ 1], a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr);
       asm volatile("cp.async.wait_group 1;" ::: "memory");
     } else {
       asm volatile("cp.async.wait_group 0;" ::: "memory");
     }
-    if (tid < L) {
-      sm.bnd[tid] = 0;
-      sm.mlog[tid] = -1;
-      sm.Itok[tid] = 0.f;
-    }
+    if (tid < L) sm.mlog[tid] = -1;
     __syncthreads();
     const int m_chunk = sm.m;
     const __nv_bfloat16* Ks = sm.kv[st][0];
@@ -462,14 +522,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     // Normally prefetched from the Gram pre-pass; formed here when the call has
     // no room for the pre-pass output (scan-only calls).
     if (!a.gram) {
-      gram_tile<D>(Ks, Vs, sm.G, sm.as[st]);
+      float* G = sm.Qs[st ^ 1];  // scratch: nothing is prefetched into the other stage here
+      gram_tile<D>(Ks, Vs, G, sm.as[st]);
       __syncthreads();
-      suffix_rows(sm.G);
+      suffix_rows(G);
       __syncthreads();
       for (int e = tid; e < L * L; e += NT) {  // transpose to the [j][t] layout the passes read
         const int t = e % L, j = e / L;
-        sm.gs[st][j * GS + t] = sm.G[t * (L + 1) + j];
+        sm.gs[st][j * GS + t] = G[t * (L + 1) + j];
       }
+      __syncthreads();
+      prefix_rows(sm.gs[st], GS, 1, sm.Qs[st], GS);
     }
     __syncthreads();
     if (tid < L) {  // this CTA's part of x_t
@@ -477,149 +540,192 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       if (m_chunk > 0)
 #pragma unroll
         for (int w8 = 0; w8 < NW; ++w8) x += sm.red[w8][tid];
-      sm.xs[st][tid] = x;
-    }
-    if constexpr (CL > 1) {
-      cluster_sync();
-    } else {
-      __syncthreads();
-    }
-    // ------------------------------------------------ 4. boundary passes (warps 0-1, token t = tid)
-    // Each pass scores every undecided token as if the open segment ran to it,
-    // takes the first that fires, and restarts the segment there.  Only the
-    // two warps that own the tokens take part (64-thread named barrier).
-    if (warp < 2) {
-      const int t = tid;
-      int cur = 0, js = 0, pre = (m_chunk > 0) ? 1 : 0;
-      if (m_chunk == 0) {  // the very first token of an empty cache opens state 0
-        if (t == 0) {
-          sm.bnd[0] = 1;
-          sm.Itok[0] = 0.f;
-        }
-        cur = 1;
+      sm.xs[st][rank][tid] = x;
+      if constexpr (CL > 1) {  // this CTA's parts of x_t and |S_open|^2 into the partner's copy
+        const uint32_t peer = (uint32_t)(rank ^ 1);
+        const uint32_t rbar = mapa_u32(&sm.xbar[st], peer);
+        st_async_f32(mapa_u32(&sm.xs[st][rank][tid], peer), x, rbar);
+        if (tid == 0) st_async_f32(mapa_u32(&sm.xs[st][rank][L], peer), sm.xs[st][rank][L], rbar);
       }
-      const float xt = (m_chunk > 0) ? whole(&sm.xs[st][t]) : 0.f;
-      const float gam_open = (m_chunk > 0) ? whole(&sm.xs[st][L]) : 0.f;
-      const float at = sm.as[st][t];
+    }
+    __syncthreads();
+    // ------------------------------------------------ 4. boundary passes (warp 0, tokens 2 lane, 2 lane + 1)
+    // Each pass scores every undecided token as if the open segment ran to it,
+    // takes the first that fires, and restarts the segment there.
+    // ------------------------------------------------ 5. replay of the decisions (Algorithm 2, warp 0)
+    if (warp == 0) {
+      if constexpr (CL > 1) {  // the partner's parts (L + 1 floats) for this chunk
+        if (lane == 0) sm100::mbar_expect_tx(&sm.xbar[st], (L + 1) * 4);
+        __syncwarp();
+        sm100::mbar_wait_cluster(&sm.xbar[st], (uint32_t)((c >> 1) & 1), &sm.abort_flag, a.status);
+      }
+      const int ta = 2 * lane, tb = ta + 1;
+      const float xa = (m_chunk > 0) ? whole(st, ta) : 0.f;
+      const float xb = (m_chunk > 0) ? whole(st, tb) : 0.f;
+      const float gam_open = (m_chunk > 0) ? whole(st, L) : 0.f;
+      const float aa = sm.as[st][ta], ab = sm.as[st][tb];
       const float* gst = sm.gs[st];
-      while (cur < Lc) {
-        float beta = 0.f, w = 0.f;
-        if (t >= js && t < Lc) {
-          beta = (pre ? xt : 0.f) + gst[js * GS + t];
-          w = 2.f * beta + at;
-        }
-        float inc = w;
+      const float* qst = sm.Qs[st];
+      // exclusive prefix sums of x_t and a_t over the chunk: with the table Q,
+      // sum_{js <= u < t} (2 beta_u + a_u) = 2 (X(t) - X(js)) [open state] + 2 Q[js][t] + A(t) - A(js)
+      float xpa, xpb, apa, apb;
+      {
+        float ix = xa + xb, ia = aa + ab;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          const float up = __shfl_up_sync(0xffffffffu, inc, o);
-          if (lane >= o) inc += up;
+          const float ux = __shfl_up_sync(0xffffffffu, ix, o);
+          const float ua = __shfl_up_sync(0xffffffffu, ia, o);
+          if (lane >= o) {
+            ix += ux;
+            ia += ua;
+          }
         }
-        if (lane == 31) sm.wsum[warp] = inc;
-        asm volatile("bar.sync 1, 64;" ::: "memory");
-        const float excl = inc - w + (warp == 1 ? sm.wsum[0] : 0.f);
-        bool fire = false;
-        if (t >= cur && t < Lc) {
-          const float gam = (pre ? gam_open : 0.f) + excl;
-          const float I = info_score(at, beta, gam, Df, a.sp);
-          sm.Itok[t] = I;
-          fire = ((double)I >= a.sp.tau);
+        xpa = __shfl_up_sync(0xffffffffu, ix, 1);
+        apa = __shfl_up_sync(0xffffffffu, ia, 1);
+        if (lane == 0) xpa = apa = 0.f;
+        xpb = xpa + xa;
+        apb = apa + aa;
+      }
+      const float invDf = 1.f / Df;
+      float Ia = 0.f, Ib = 0.f;  // final scores of tokens ta, tb
+      int cur = 0, js = 0, pre = (m_chunk > 0) ? 1 : 0;
+      unsigned long long bmask = 0;
+      if (m_chunk == 0) {  // the very first token of an empty cache opens state 0 (score 0)
+        bmask = 1;
+        cur = 1;
+      }
+      while (cur < Lc) {
+        const float xpj = __shfl_sync(0xffffffffu, (js & 1) ? xpb : xpa, js >> 1);
+        const float apj = __shfl_sync(0xffffffffu, (js & 1) ? apb : apa, js >> 1);
+        const float g0 = pre ? gam_open : 0.f;
+        bool fa = false, fb = false;
+        if (ta >= cur && ta < Lc) {
+          const float ba = (pre ? xa : 0.f) + gst[js * GS + ta];
+          const float ea = (pre ? 2.f * (xpa - xpj) : 0.f) + 2.f * qst[js * GS + ta] + (apa - apj);
+          Ia = info_score_fast(aa, ba, g0 + ea, invDf, a.sp);
+          fa = (Ia >= a.sp.tau_f);
         }
-        const unsigned bal = __ballot_sync(0xffffffffu, fire);
-        if (lane == 0) sm.first_fire[warp] = bal ? (warp * 32 + __ffs(bal) - 1) : L;
-        asm volatile("bar.sync 1, 64;" ::: "memory");
-        const int ts = min(sm.first_fire[0], sm.first_fire[1]);
-        if (ts >= Lc) break;
-        if (t == ts) sm.bnd[ts] = 1;
+        if (tb >= cur && tb < Lc) {
+          const float bb = (pre ? xb : 0.f) + gst[js * GS + tb];
+          const float eb = (pre ? 2.f * (xpb - xpj) : 0.f) + 2.f * qst[js * GS + tb] + (apb - apj);
+          Ib = info_score_fast(ab, bb, g0 + eb, invDf, a.sp);
+          fb = (Ib >= a.sp.tau_f);
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, fa || fb);
+        if (!bal) break;
+        const int src = __ffs(bal) - 1;
+        const int ts = 2 * src + (__shfl_sync(0xffffffffu, (int)fa, src) ? 0 : 1);
+        bmask |= 1ull << ts;
         js = ts;
         pre = 0;
         cur = ts + 1;
       }
-    }
-    __syncthreads();
-    // ------------------------------------------------ 5. replay decisions (warp 0)
-    if (warp == 0) {
-      int m = sm.m;
-      int seg_u0 = 0;
-      int nops = 0;
-      int run0 = 0;
-      // boundary tokens of the chunk as a bit mask (Lc <= 64)
-      const unsigned lo = __ballot_sync(0xffffffffu, sm.bnd[lane] != 0);
-      const unsigned hi = __ballot_sync(0xffffffffu, sm.bnd[lane + 32] != 0);
-      unsigned long long pend = ((unsigned long long)hi << 32) | lo;
+      sm.bnd[ta] = (int)((bmask >> ta) & 1);
+      sm.bnd[tb] = (int)((bmask >> tb) & 1);
+      // score sum of the tokens [u0, u1) of the chunk (fp32 warp sum; Ibar itself is fp64)
+      auto run_sum = [&](int u0, int u1) -> float {
+        const float v = ((ta >= u0 && ta < u1) ? Ia : 0.f) + ((tb >= u0 && tb < u1) ? Ib : 0.f);
+        return warp_sum(v);
+      };
+      int m = m_chunk;
+      int seg_u0 = 0, nops = 0, run0 = 0;
+      unsigned long long pend = bmask;
       while (true) {
         const int t = pend ? (__ffsll((long long)pend) - 1) : Lc;
         pend &= pend - 1;
-        if (t > run0) {  // tokens [run0, t) joined the open state
-          float part = 0.f;
-          for (int u = run0 + lane; u < t; u += 32) part += sm.Itok[u];
-          part = warp_sum(part);
-          if (lane == 0) {
-            sm.n[m - 1] += t - run0;
-            sm.ibar[m - 1] += (double)part;
-            sm.dirty[m - 1] = 1;
+        if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
+          const double part = (double)run_sum(run0, t);
+          const int e = m - 1;
+          if ((e & 31) == lane) {
+            if (e < 32) {
+              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1;
+            } else {
+              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1;
+            }
           }
-          __syncwarp();
         }
         run0 = t + 1;
         if (t >= Lc) break;
-        if (m > 0 && lane == 0) {
-          sm.ops[nops][0] = OP_CLOSE;
-          sm.ops[nops][1] = sm.slot[m - 1];
-          sm.ops[nops][2] = seg_u0;
-          sm.ops[nops][3] = t;
+        if (m > 0) {
+          const int sl = entry_get(e_slot, m - 1);
+          if (lane == 0) {
+            sm.ops[nops][0] = OP_CLOSE;
+            sm.ops[nops][1] = sl;
+            sm.ops[nops][2] = seg_u0;
+            sm.ops[nops][3] = t;
+          }
+          ++nops;
         }
-        if (m > 0) ++nops;
         int j = -1, phys_new = m;
-        __syncwarp();
         if (m == C) {
-          j = pair_argmin_warp(sm.n, sm.ibar, m);
-          const int dst = sm.slot[j], src = sm.slot[j + 1];
-          __syncwarp();
+          // pair densities (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}): fp64 sums, compared in fp32
+          int nn[2], ns[2], np_[2], nd[2];
+          double nb[2];
+          entry_next(e_n, nn);
+          entry_next(e_ib, nb);
+          entry_next(e_slot, ns);
+          entry_next(e_pid, np_);
+          entry_next(e_dirty, nd);
+          float best = __int_as_float(0x7f800000);
+          int bi = 0x7fffffff;
+          if (lane + 1 < m) {
+            best = (float)(e_ib[0] + nb[0]) / (float)(e_n[0] + nn[0]);
+            bi = lane;
+          }
+          if (lane + 33 < m) {
+            const float d1 = (float)(e_ib[1] + nb[1]) / (float)(e_n[1] + nn[1]);
+            if (d1 < best) {
+              best = d1;
+              bi = lane + 32;
+            }
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+            if (ov < best || (ov == best && oi < bi)) {
+              best = ov;
+              bi = oi;
+            }
+          }
+          j = bi;
+          const int dst = entry_get(e_slot, j), srcs = entry_get(e_slot, j + 1);
           if (lane == 0) {
             sm.ops[nops][0] = OP_MERGE;
             sm.ops[nops][1] = dst;
-            sm.ops[nops][2] = src;
+            sm.ops[nops][2] = srcs;
             sm.ops[nops][3] = 0;
-            sm.n[j] += sm.n[j + 1];
-            sm.ibar[j] += sm.ibar[j + 1];
-            sm.dirty[j] = 1;
-            sm.pid[j] = -1;
           }
           ++nops;
-          __syncwarp();
-          for (int base = j + 1; base < m - 1; base += 32) {
-            const int i = base + lane;
-            int nv = 0, sv = 0, pv = 0, dv = 0;
-            double iv = 0.0;
-            if (i < m - 1) {
-              nv = sm.n[i + 1]; sv = sm.slot[i + 1]; pv = sm.pid[i + 1]; dv = sm.dirty[i + 1];
-              iv = sm.ibar[i + 1];
+          // entry j absorbs j + 1; entries j + 2 .. m - 1 move down by one
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int i = lane + 32 * r;
+            if (i == j) {
+              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1;
+            } else if (i > j && i < m - 1) {
+              e_n[r] = nn[r]; e_ib[r] = nb[r]; e_slot[r] = ns[r]; e_pid[r] = np_[r]; e_dirty[r] = nd[r];
             }
-            __syncwarp();
-            if (i < m - 1) {
-              sm.n[i] = nv; sm.slot[i] = sv; sm.pid[i] = pv; sm.dirty[i] = dv; sm.ibar[i] = iv;
-            }
-            __syncwarp();
           }
-          phys_new = src;
+          phys_new = srcs;
           m -= 1;
         }
-        if (lane == 0) {
-          sm.slot[m] = phys_new;
-          sm.n[m] = 1;
-          sm.ibar[m] = (double)sm.Itok[t];
-          sm.pid[m] = -1;
-          sm.dirty[m] = 1;
-          sm.mlog[t] = j;
-        }
-        __syncwarp();
+        const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
+        entry_set(e_slot, m, phys_new);
+        entry_set(e_n, m, 1);
+        entry_set(e_ib, m, (double)it);
+        entry_set(e_pid, m, -1);
+        entry_set(e_dirty, m, 1);
+        if (lane == 0) sm.mlog[t] = j;
         m += 1;
         seg_u0 = t;
       }
+      const int oslot = (m > 0) ? entry_get(e_slot, m - 1) : 0;
       if (lane == 0) {
         sm.m = m;
         sm.nops = nops;
         sm.js = seg_u0;
+        sm.open_slot = oslot;
       }
     }
     __syncthreads();
@@ -659,9 +765,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       if (warp == 0) {  // entries whose state changed get a fresh pool entry
         const int m = sm.m;
         int nj = 0;
-        for (int base = 0; base < m; base += 32) {
-          const int i = base + lane;
-          const bool need = (i < m) && (sm.dirty[i] || sm.pid[i] < 0);
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int i = lane + 32 * r;
+          const bool need = (i < m) && (e_dirty[r] || e_pid[r] < 0);
           const unsigned bal = __ballot_sync(0xffffffffu, need);
           if (need) {
             const int rank_ = nj + __popc(bal & ((1u << lane) - 1u));
@@ -670,12 +777,13 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
               atomicExch(a.status, 6);
               p = a.pool_cap - 1;
             }
-            sm.pid[i] = p;
-            sm.dirty[i] = 0;
+            e_pid[r] = p;
+            e_dirty[r] = 0;
             sm.snap_src[rank_][0] = p;
-            sm.snap_src[rank_][1] = (i == m - 1) ? -1 : sm.slot[i];
+            sm.snap_src[rank_][1] = (i == m - 1) ? -1 : e_slot[r];
           }
           nj += __popc(bal);
+          if (lead && i < m) a.snap_ids[lrow * C + i] = e_pid[r];
         }
         __syncwarp();
         if (lane == 0) {
@@ -685,9 +793,6 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         }
       }
       __syncthreads();
-      const int m = sm.m;
-      if (lead)
-        for (int i = tid; i < m; i += NT) a.snap_ids[lrow * C + i] = sm.pid[i];
       for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
         const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
         Tpool* entry = pool + (long long)p * kEntry;
@@ -719,7 +824,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   {
     const int m = sm.m;
     if (m > 0) {
-      float* dst = states + (long long)sm.slot[m - 1] * D * D;
+      float* dst = states + (long long)sm.open_slot * D * D;
 #pragma unroll
       for (int n = 0; n < NT8; ++n) {
         const int k = k0 + 8 * n + 2 * tg;
@@ -727,16 +832,20 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         *reinterpret_cast<float2*>(dst + (jg0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
       }
     }
-    if (lead) {
-      for (int i = tid; i < C; i += NT) {
-        a.slot[(long long)bh * C + i] = sm.slot[i];
-        a.n[(long long)bh * C + i] = (i < m) ? sm.n[i] : 0;
-        a.ibar[(long long)bh * C + i] = (i < m) ? sm.ibar[i] : 0.0;
+    if (lead && warp == 0) {
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const int i = lane + 32 * r;
+        if (i < C) {
+          a.slot[(long long)bh * C + i] = e_slot[r];
+          a.n[(long long)bh * C + i] = (i < m) ? e_n[r] : 0;
+          a.ibar[(long long)bh * C + i] = (i < m) ? e_ib[r] : 0.0;
+        }
+        if (pool && a.pstate && i < m) a.pstate[a.B * a.H + (long long)bh * C + i] = e_pid[r];
       }
-      if (tid == 0) a.m[bh] = m;
-      if (pool && a.pstate) {  // counters for a following round that continues this pool
-        if (tid == 0) a.pstate[bh] = sm.pool_next;
-        for (int i = tid; i < m; i += NT) a.pstate[a.B * a.H + (long long)bh * C + i] = sm.pid[i];
+      if (lane == 0) {
+        a.m[bh] = m;
+        if (pool && a.pstate) a.pstate[bh] = sm.pool_next;  // counters for a following round that continues this pool
       }
     }
   }
@@ -744,15 +853,18 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 }
 
 // K0: Gram pre-pass.  One CTA per (64-token chunk, stream): the suffix table
-// sg[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s) and a_t of every chunk, so the
-// sequential scan reads beta_t of any segment start with one load.  Depends on
-// k and v only, so it runs on every SM ahead of the scan.
+// gs[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s), its running sums
+// Q[j][t] = sum_{j <= u < t} gs[j][u] and a_t of every chunk, so that the
+// sequential scan reads beta_t and the segment's sum of 2 beta_u + a_u for any
+// segment start with two loads.  Depends on k and v only, so it runs on the
+// other SMs ahead of the scan.
 template <int D>
 struct GramSmem {
   static constexpr int RP = D + 8;
   __nv_bfloat16 k[L * RP];
   __nv_bfloat16 v[L * RP];
   float G[L * (L + 1)];
+  float Q[L * (L + 1)];
   float a[L];
 };
 
@@ -784,14 +896,17 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   __syncthreads();
   gram_tile<D>(sm.k, sm.v, sm.G, sm.a);
   __syncthreads();
-  suffix_rows(sm.G);
+  suffix_rows(sm.G);  // G[t][j] = gs[j][t]
+  __syncthreads();
+  prefix_rows(sm.G, 1, L + 1, sm.Q, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u]
   __syncthreads();
   float* out = a.out + ((long long)bh * a.nchunks + c) * kGramBlock;
   for (int e = threadIdx.x; e < L * L; e += NT) {
     const int t = e % L, j = e / L;
     out[j * L + t] = sm.G[t * (L + 1) + j];
+    out[L * L + j * L + t] = sm.Q[j * (L + 1) + t];
   }
-  if (threadIdx.x < L) out[L * L + threadIdx.x] = sm.a[threadIdx.x];
+  if (threadIdx.x < L) out[2 * L * L + threadIdx.x] = sm.a[threadIdx.x];
 }
 
 template <int D>
