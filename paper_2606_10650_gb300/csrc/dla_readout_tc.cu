@@ -1,20 +1,27 @@
 // dla_readout_tc.cu -- K2b on the 5th-generation tensor cores (tcgen05 + TMEM
 // + TMA): the snapshot part of the read-out of Eq. (capacity_bounded_output)
 //   o_t = o_intra[t] + sum_{x < m0} lambda_{t, L_t(x)} (S_x q_t)
-// for one 128-token interval of one stream per CTA, bf16 inputs, d = 128.
-// o_intra (the interval's own tokens, fp32) comes from K2a.  The cache seen by
-// token t is the snapshot taken by K1 at the interval start (m0 states,
-// logical order) regrouped by the merges decided inside the interval: merges
-// only add states, so snapshot entry x contributes with the lambda of its
-// logical slot L_t(x) after the interval's events up to t.
-// Per state x: D_x = Q S_x^T = Q (S_hi + S_lo)^T (M = 128 tokens, N = 128,
-// K = 128), the fp32 snapshot split into bf16 hi + lo parts by K1 (two MMAs per
-// state keep the state rounding near 2^-17 instead of 2^-9).
-// Roles: warp 0 issues TMA loads into five 32 KB half-stages (the hi or lo part
-// of one state each), warp 1 issues tcgen05.mma (one thread) into four TMEM
-// accumulators of 128 columns, warps 2..9 read TMEM, weight by lambda and
-// accumulate o in registers (warp w reads TMEM lane quadrant w % 4; warps 2-5
-// own columns 0-63, warps 6-9 own 64-127).
+// for bf16 inputs, d = 128.  o_intra (the interval's own tokens, fp32) comes
+// from K2a.  The cache seen by token t is the snapshot taken by K1 at the start
+// of t's 128-token interval (m0 states, logical order) regrouped by the merges
+// decided inside the interval: merges only add states, so snapshot entry x
+// contributes with the lambda of its logical slot L_t(x) after the interval's
+// events up to t.
+//
+// One CTA per (pair of consecutive intervals A, B, stream).  Consecutive
+// snapshot lists share most of their states (only entries that changed get new
+// pool entries), so the CTA loads the union of the two lists once and applies
+// each state to the tokens of both intervals: D_x^A = Q_A S_x^T and
+// D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128), with
+// S_x = S_hi + S_lo, the fp32 snapshot split into bf16 parts by K1 (two MMAs
+// per state and interval keep the state rounding near 2^-17 instead of 2^-9).
+// An interval's MMAs are skipped for a state that is not in its list.
+// Roles: warp 0 issues TMA loads (the two Q tiles, then the hi and lo parts of
+// each union state into four 32 KB half-stages), warp 1 issues tcgen05.mma (one
+// thread) into two TMEM buffers of two 128-column accumulators (A, B), warps
+// 2..9 read TMEM, weight by lambda and accumulate both intervals' o in registers
+// (warp w reads TMEM lane quadrant w % 4; warps 2-5 own columns 0-63, warps 6-9
+// own 64-127).
 #include <cudaTypedefs.h>
 
 #include "dla_common.cuh"
@@ -26,29 +33,78 @@ namespace {
 
 using namespace sm100;
 
-constexpr int L = 128;   // tokens per CTA
+constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
 constexpr int NT = 320;  // 10 warps
 constexpr int NEPI = 8;  // epilogue warps
-constexpr int NHS = 5;   // shared-memory half-stages
-constexpr int NACC = 4;  // TMEM accumulators
+constexpr int NHS = 4;   // shared-memory half-stages
+constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
+constexpr int MAXU = 2 * kMaxC;  // union of two lists
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTile = L * 128;  // one K-major 128B-swizzled tile: 128 rows x 64 bf16
 
-struct TcSmem {
-  uint8_t Q[2][kTile];                 // A operand, two k-halves              32 KB
-  uint8_t hs[NHS][2][kTile];           // [half-stage][k-half]                160 KB
+struct Side {                          // per interval of the pair
   unsigned char tab[(L + 1) * kMaxC];  // L(x) of snapshot entry x after event e
-  int logi[kMaxC];
   int evt[L];                          // events (boundaries) at or before token t
-  int mlog[L];                         // the interval's merge indices
-  uint8_t bnd[L];                      // and boundary flags
-  int ids[kMaxC];                      // pool ids of the snapshot entries
+  int mlog[L];                         // merge indices
+  uint8_t bnd[L];                      // boundary flags
+};
+
+struct TcSmem {
+  uint8_t Q[2][2][kTile];      // [interval][k-half], A operands        64 KB
+  uint8_t hs[NHS][2][kTile];   // [half-stage][k-half]                 128 KB
+  Side side[2];
+  int ids[2][kMaxC];           // pool ids of the two lists
+  int uid[MAXU];               // union: pool id
+  int uxa[MAXU], uxb[MAXU];    // union: index in list A / list B, or -1
+  int logi[kMaxC];
+  int nu;                      // union size
   uint64_t bar_q, bar_done;
-  uint64_t full[NHS], empty[NHS], acc_full[NACC], acc_empty[NACC];
+  uint64_t full[NHS], empty[NHS], acc_full[NBUF], acc_empty[NBUF];
   uint32_t tmem_base;
   int abort_flag;
 };
+
+// Slot table of one interval (one warp): row e holds L(x) of snapshot entry x
+// after the interval's first e boundary events.
+__device__ __forceinline__ void build_table(Side& sd, int* logi, int m0, int lane) {
+  for (int x = lane; x < m0; x += 32) {
+    logi[x] = x;
+    sd.tab[x] = (unsigned char)x;
+  }
+  __syncwarp();
+  unsigned long long lo64 = 0, hi64 = 0;
+#pragma unroll
+  for (int w4 = 0; w4 < 4; ++w4) {
+    const unsigned m = __ballot_sync(0xffffffffu, sd.bnd[32 * w4 + lane] != 0);
+    if (w4 < 2) lo64 |= (unsigned long long)m << (32 * w4);
+    else hi64 |= (unsigned long long)m << (32 * (w4 - 2));
+  }
+  int ev = 0;
+  while (lo64 | hi64) {
+    const int tt = lo64 ? (__ffsll((long long)lo64) - 1) : (64 + __ffsll((long long)hi64) - 1);
+    if (lo64) lo64 &= lo64 - 1; else hi64 &= hi64 - 1;
+    const int j = sd.mlog[tt];
+    ev += 1;
+    for (int x = lane; x < m0; x += 32) {
+      int li = logi[x];
+      if (j >= 0 && li > j) logi[x] = --li;
+      sd.tab[ev * kMaxC + x] = (unsigned char)li;
+    }
+  }
+}
+
+// Events at or before token tt of an interval (one warp, one token per lane).
+__device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
+  int e = 0;
+#pragma unroll
+  for (int w4 = 0; w4 < 4; ++w4) {
+    const unsigned m = __ballot_sync(0xffffffffu, sd.bnd[32 * w4 + lane] != 0);
+    if (32 * w4 + 31 <= tt) e += __popc(m);
+    else if (32 * w4 <= tt) e += __popc(m & (0xffffffffu >> (31 - (tt - 32 * w4))));
+  }
+  return e;
+}
 
 }  // namespace
 
@@ -58,13 +114,18 @@ __global__ void __launch_bounds__(NT, 1)
   extern __shared__ uint8_t smem_raw[];
   TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int s = blockIdx.x, bh = blockIdx.y;
+  const int pair = blockIdx.x, bh = blockIdx.y;
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
-  const int c0 = a.t_begin + s * L;
-  const int Lc = min(L, a.t_end - c0);
-  const long long lrow = (long long)bh * a.snap_stride + a.snap_base + s;
-  const int m0 = a.snap_m0[lrow];
+  const int sA = 2 * pair;
+  const bool hasB = (sA + 1) < a.nsnap;
+  // interval A (side 0) and B (side 1) of the pair
+  const int c0A = a.t_begin + sA * L, c0B = c0A + L;
+  const int LcA = min(L, a.t_end - c0A), LcB = hasB ? min(L, a.t_end - c0B) : 0;
+  const long long lrowA = (long long)bh * a.snap_stride + a.snap_base + sA, lrowB = lrowA + 1;
+  const int m0A = a.snap_m0[lrowA], m0B = hasB ? a.snap_m0[lrowB] : 0;
+  auto c0_of = [&](int side) { return side ? c0B : c0A; };
+  auto Lc_of = [&](int side) { return side ? LcB : LcA; };
   volatile int* abort = &sm.abort_flag;
 
   if (tid == 0) {
@@ -74,43 +135,87 @@ __global__ void __launch_bounds__(NT, 1)
       mbar_init(&sm.full[i], 1);
       mbar_init(&sm.empty[i], 1);
     }
-    for (int i = 0; i < NACC; ++i) {
+    for (int i = 0; i < NBUF; ++i) {
       mbar_init(&sm.acc_full[i], 1);
       mbar_init(&sm.acc_empty[i], NEPI);
     }
     sm.abort_flag = 0;
     fence_mbar_init();
+    // the Q tiles go out first; they depend on nothing
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmS);
+    mbar_expect_tx(&sm.bar_q, (hasB ? 4 : 2) * kTile);
+    tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, c0A, b);
+    tma_load_4d(sm.Q[0][1], &tmQ, &sm.bar_q, 64, h, c0A, b);
+    if (hasB) {
+      tma_load_4d(sm.Q[1][0], &tmQ, &sm.bar_q, 0, h, c0B, b);
+      tma_load_4d(sm.Q[1][1], &tmQ, &sm.bar_q, 64, h, c0B, b);
+    }
   }
-  for (int i = tid; i < m0; i += NT) sm.ids[i] = a.snap_ids[lrow * C + i];
+  for (int i = tid; i < 2 * kMaxC; i += NT) {
+    const int side = i / kMaxC, x = i % kMaxC;
+    sm.ids[side][x] = (x < (side ? m0B : m0A)) ? a.snap_ids[(side ? lrowB : lrowA) * C + x] : -1;
+  }
   if (warp == 1) tmem_alloc(&sm.tmem_base, kTmemCols);
+  __syncthreads();
+  if (warp == 0) {
+    // union of the two lists: list A in order, then the entries of list B not in A
+    for (int x = lane; x < kMaxC; x += 32) {
+      if (x < m0A) {
+        sm.uid[x] = sm.ids[0][x];
+        sm.uxa[x] = x;
+        sm.uxb[x] = -1;
+      }
+    }
+    __syncwarp();
+    int nb_only = 0;
+    for (int base = 0; base < m0B; base += 32) {
+      const int x = base + lane;
+      int match = -1;
+      if (x < m0B) {
+        const int id = sm.ids[1][x];
+        for (int y = 0; y < m0A; ++y)
+          if (sm.ids[0][y] == id) match = y;
+      }
+      const unsigned only = __ballot_sync(0xffffffffu, x < m0B && match < 0);
+      if (x < m0B) {
+        if (match >= 0) {
+          sm.uxb[match] = x;
+        } else {
+          const int u = m0A + nb_only + __popc(only & ((1u << lane) - 1u));
+          sm.uid[u] = sm.ids[1][x];
+          sm.uxa[u] = -1;
+          sm.uxb[u] = x;
+        }
+      }
+      nb_only += __popc(only);
+    }
+    if (lane == 0) sm.nu = m0A + nb_only;
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
+  const int nu = sm.nu;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      prefetch_tmap(&tmQ);
-      prefetch_tmap(&tmS);
-      mbar_expect_tx(&sm.bar_q, 2 * kTile);
-      tma_load_4d(sm.Q[0], &tmQ, &sm.bar_q, 0, h, c0, b);
-      tma_load_4d(sm.Q[1], &tmQ, &sm.bar_q, 64, h, c0, b);
       int issued[NHS];  // uses of each half-stage so far
       for (int i = 0; i < NHS; ++i) issued[i] = 0;
-      for (int u = 0; u < 2 * m0; ++u) {  // unit u: part u & 1 (hi, lo) of state u >> 1
+      for (int u = 0; u < 2 * nu; ++u) {  // unit u: part u & 1 (hi, lo) of union state u >> 1
         const int hsi = u % NHS, k = u / NHS;
         if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
-        const int row = (int)((((long long)bh * a.pool_cap + sm.ids[u >> 1]) * 2 + (u & 1)) * D);
+        const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
         tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
         tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
         issued[hsi] = k + 1;
       }
       if (*abort) {  // let copies in flight land before the CTA exits
         for (int i = 0; i < NHS; ++i)
-          if (issued[i] > 0) mbar_wait(&sm.full[i], (uint32_t)((issued[i] - 1) & 1), abort, nullptr);
-        mbar_wait(&sm.bar_q, 0, abort, nullptr);
+          if (issued[i] > 0) mbar_wait_drain(&sm.full[i], (uint32_t)((issued[i] - 1) & 1));
+        mbar_wait_drain(&sm.bar_q, 0);
       }
     }
   } else if (warp == 1) {
@@ -118,131 +223,130 @@ __global__ void __launch_bounds__(NT, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(L, D);
       bool ok = mbar_wait(&sm.bar_q, 0, abort, status);
-      for (int x = 0; ok && x < m0; ++x) {
-        const int buf = x % NACC, kb = x / NACC;
+      for (int x = 0; ok && x < nu; ++x) {
+        const int buf = x % NBUF, kb = x / NBUF;
+        const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
         if (!mbar_wait(&sm.acc_empty[buf], (uint32_t)((kb & 1) ^ 1), abort, status)) break;
         tc_fence_after();
-        const uint32_t dcol = tmem + 128u * buf;
+        const uint32_t dA = tmem + 256u * buf, dB = dA + 128u;
         for (int part = 0; part < 2; ++part) {
           const int u = 2 * x + part, hsi = u % NHS, k = u / NHS;
           if (!(ok = mbar_wait(&sm.full[hsi], (uint32_t)(k & 1), abort, status))) break;
           tc_fence_after();
           for (int kk = 0; kk < 8; ++kk) {
             const uint32_t off = (uint32_t)(kk & 3) * 32;
-            mma_bf16(dcol, desc_kmajor_sw128(smem_u32(sm.Q[kk >> 2]) + off),
-                     desc_kmajor_sw128(smem_u32(sm.hs[hsi][kk >> 2]) + off), idesc, (part | kk) > 0);
+            const uint64_t bdesc = desc_kmajor_sw128(smem_u32(sm.hs[hsi][kk >> 2]) + off);
+            if (inA) mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off), bdesc, idesc, (part | kk) > 0);
+            if (inB) mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off), bdesc, idesc, (part | kk) > 0);
           }
           mma_commit(&sm.empty[hsi]);
         }
         if (ok) mma_commit(&sm.acc_full[buf]);
       }
       mma_commit(&sm.bar_done);  // every MMA issued above has completed once this fires
-      mbar_wait(&sm.bar_done, 0, abort, nullptr);
+      mbar_wait_drain(&sm.bar_done, 0);
     }
   } else {
     // ------------------------------------------------------------ epilogue warps
     const int ew = warp - 2;            // 0..7
     const int quad = warp & 3;          // TMEM lane quadrant of this warp
     const int ch = (warp < 6) ? 0 : 1;  // column half
-    const int t = quad * 32 + lane;     // token row of this thread
+    const int t = quad * 32 + lane;     // token row of this thread (in both intervals)
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
     const int etid = ew * 32 + lane;    // 0..255
-    const long long rowbase = ((long long)b * a.T + c0) * a.H + h;  // row index of token c0
 
-    if (etid < L) {  // the interval's boundary flags and merge indices, staged once
-      const bool in = etid < Lc;
-      sm.bnd[etid] = in ? a.boundary[(long long)bh * a.T + c0 + etid] : (uint8_t)0;
-      sm.mlog[etid] = in ? a.merge_log[(long long)bh * a.T + c0 + etid] : -1;
+    {  // both intervals' boundary flags and merge indices (thread etid: interval etid / L, token etid % L)
+      const int side = etid / L, tt = etid % L;
+      const bool in = tt < Lc_of(side);
+      const long long tr = (long long)bh * a.T + c0_of(side) + tt;
+      sm.side[side].bnd[tt] = in ? a.boundary[tr] : (uint8_t)0;
+      sm.side[side].mlog[tt] = in ? a.merge_log[tr] : -1;
     }
-    // o starts from the intra-interval part (K2a; column-quad order, so a warp
+    // o starts from the intra-interval parts (K2a; column-quad order, so a warp
     // reads 512 contiguous bytes per load)
-    float o[64];
-    {
-      const float* src = a.ointra + ((long long)bh * a.ointra_T + (c0 - a.t_begin)) * D + (16 * ch * L + t) * 4;
+    float o[2][64];
+#pragma unroll
+    for (int side = 0; side < 2; ++side) {
+      const float* src =
+          a.ointra + ((long long)bh * a.ointra_T + (c0_of(side) - a.t_begin)) * D + (16 * ch * L + t) * 4;
 #pragma unroll
       for (int i = 0; i < 64; i += 4) {
         float4 v4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (t < Lc) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
-        o[i] = v4.x; o[i + 1] = v4.y; o[i + 2] = v4.z; o[i + 3] = v4.w;
+        if (t < Lc_of(side)) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
+        o[side][i] = v4.x; o[side][i + 1] = v4.y; o[side][i + 2] = v4.z; o[side][i + 3] = v4.w;
       }
     }
     asm volatile("bar.sync 1, 256;" ::: "memory");
-    // logical slots of the snapshot entries, one table row per boundary event
-    // (one warp): row e holds L(x) after the first e events of the interval
-    if (ew == 0) {
-      for (int x = lane; x < m0; x += 32) {
-        sm.logi[x] = x;
-        sm.tab[x] = (unsigned char)x;
-      }
-      __syncwarp();
-      unsigned long long lo64 = 0, hi64 = 0;
-#pragma unroll
-      for (int w4 = 0; w4 < 4; ++w4) {
-        const unsigned m = __ballot_sync(0xffffffffu, sm.bnd[32 * w4 + lane] != 0);
-        if (w4 < 2) lo64 |= (unsigned long long)m << (32 * w4);
-        else hi64 |= (unsigned long long)m << (32 * (w4 - 2));
-      }
-      int ev = 0;
-      while (lo64 | hi64) {
-        const int tt = lo64 ? (__ffsll((long long)lo64) - 1) : (64 + __ffsll((long long)hi64) - 1);
-        if (lo64) lo64 &= lo64 - 1; else hi64 &= hi64 - 1;
-        const int j = sm.mlog[tt];
-        ev += 1;
-        for (int x = lane; x < m0; x += 32) {
-          int li = sm.logi[x];
-          if (j >= 0 && li > j) sm.logi[x] = --li;
-          sm.tab[ev * kMaxC + x] = (unsigned char)li;
-        }
-      }
-    }
-    if (etid < L) {  // events at or before each token (warps 2..5, one token per lane)
-      const int tt = etid;
-      int e = 0;
-#pragma unroll
-      for (int w4 = 0; w4 < 4; ++w4) {
-        const unsigned m = __ballot_sync(0xffffffffu, sm.bnd[32 * w4 + lane] != 0);
-        if (32 * w4 + 31 <= tt) e += __popc(m);
-        else if (32 * w4 <= tt) e += __popc(m & (0xffffffffu >> (31 - (tt - 32 * w4))));
-      }
-      sm.evt[tt] = e;
+    if (ew == 0) build_table(sm.side[0], sm.logi, m0A, lane);
+    asm volatile("bar.sync 1, 256;" ::: "memory");  // logi is shared by the two builds
+    if (ew == 0) build_table(sm.side[1], sm.logi, m0B, lane);
+    {
+      const int side = etid / L, tt = etid % L;  // warps 2-5: interval A, 6-9: interval B
+      sm.side[side].evt[tt] = events_before(sm.side[side], tt, lane);
     }
     asm volatile("bar.sync 1, 256;" ::: "memory");
-    const float* lam_t = (a.lam && t < Lc) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
-    const unsigned char* tab_t = sm.tab + sm.evt[t] * kMaxC;
-    // weight of state x for this token; fetched one state ahead of its use
-    auto weight = [&](int x) -> float {
-      if (t >= Lc || x >= m0) return 0.f;
-      return lam_t ? lam_t[tab_t[x]] : 1.f;
+    const float* lam[2];
+    const unsigned char* tabt[2];
+#pragma unroll
+    for (int side = 0; side < 2; ++side) {
+      const long long rowbase = ((long long)b * a.T + c0_of(side)) * a.H + h;
+      lam[side] = (a.lam && t < Lc_of(side)) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
+      tabt[side] = sm.side[side].tab + sm.side[side].evt[t] * kMaxC;
+    }
+    // weight of union state x for this token in interval side (0 when not in its list)
+    auto weight = [&](int side, int x) -> float {
+      if (x >= nu || t >= Lc_of(side)) return 0.f;
+      const int xi = side ? sm.uxb[x] : sm.uxa[x];
+      if (xi < 0) return 0.f;
+      return lam[side] ? lam[side][tabt[side][xi]] : 1.f;
     };
-    float w_next = weight(0);
-    for (int x = 0; x < m0; ++x) {
-      const int buf = x % NACC, kb = x / NACC;
-      const float w = w_next;
-      w_next = weight(x + 1);
+    float wnA = weight(0, 0), wnB = weight(1, 0);
+    for (int x = 0; x < nu; ++x) {
+      const int buf = x % NBUF, kb = x / NBUF;
+      const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
+      const float wA = wnA, wB = wnB;
+      wnA = weight(0, x + 1);
+      wnB = weight(1, x + 1);
       if (!mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status)) break;
       tc_fence_after();
-      float dv[32];
-      const uint32_t base = lane_addr + 128u * buf + 64 * ch;
-      tmem_ld32(base, dv);
+      float dv[16];
+      const uint32_t base = lane_addr + 256u * buf + 64 * ch;
+      if (inA) {
 #pragma unroll
-      for (int i = 0; i < 32; ++i) o[i] += w * dv[i];
-      tmem_ld32(base + 32, dv);
+        for (int c = 0; c < 64; c += 16) {
+          tmem_ld16(base + c, dv);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) o[32 + i] += w * dv[i];
+          for (int i = 0; i < 16; ++i) o[0][c + i] += wA * dv[i];
+        }
+      }
+      if (inB) {
+#pragma unroll
+        for (int c = 0; c < 64; c += 16) {
+          tmem_ld16(base + 128 + c, dv);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o[1][c + i] += wB * dv[i];
+        }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
     }
-    if (t < Lc && !*abort) {
-      const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
-      if (a.out_bf16) {
-        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
+    if (!*abort) {
 #pragma unroll
-        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-      } else {
-        float* out = reinterpret_cast<float*>(a.o) + orow;
+      for (int side = 0; side < 2; ++side) {
+        if (t >= Lc_of(side)) continue;
+        const long long orow = (((long long)b * a.T + c0_of(side) + t) * a.H + h) * D + 64 * ch;
+        if (a.out_bf16) {
+          __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
 #pragma unroll
-        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+          for (int i = 0; i < 64; i += 4)
+            store4(out + i, make_float4(o[side][i], o[side][i + 1], o[side][i + 2], o[side][i + 3]));
+        } else {
+          float* out = reinterpret_cast<float*>(a.o) + orow;
+#pragma unroll
+          for (int i = 0; i < 64; i += 4)
+            store4(out + i, make_float4(o[side][i], o[side][i + 1], o[side][i + 2], o[side][i + 3]));
+        }
       }
     }
   }
@@ -303,7 +407,7 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
   const size_t smem = sizeof(TcSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid(a.nsnap, a.B * a.H);
+  dim3 grid((a.nsnap + 1) / 2, a.B * a.H);  // pairs of intervals
   readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, ms, status);
   return cudaGetLastError();
 }

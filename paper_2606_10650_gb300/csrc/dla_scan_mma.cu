@@ -22,19 +22,20 @@ namespace {
 constexpr int NT = 256;
 constexpr int NW = NT / 32;
 constexpr int L = kScanL;
-constexpr int GS = L + 4;          // row of a suffix table in shared memory
+constexpr int GS = L;              // row of a Gram table in shared memory (the pre-pass block, verbatim)
 
 enum : int { OP_CLOSE = 0, OP_MERGE = 1 };
 
 template <int D, int CL>
 struct MmaSmem {
   static constexpr int RP = D + 8;  // padded bf16 row: 8 rows of a ldmatrix hit 8 bank groups
-  static constexpr int GS = L + 4;  // suffix-table row (16-byte aligned for cp.async)
   __nv_bfloat16 kv[2][2][L * RP];   // [stage][k / v][t][RP]
   __nv_bfloat16 S2[2][D / CL * RP]; // this CTA's rows of the open state as bf16 hi / lo, [j][RP]
-  float gs[2][L * GS];              // [stage] suffix table gs[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s)
-  float Qs[2][L * GS];              // [stage] prefix table Q[j][t] = sum_{j <= u < t} gs[j][u]
-  float as[2][L];                   // [stage] a_t = |k_t|^2 |v_t|^2
+  // [stage] the chunk's Gram block, as the pre-pass writes it: suffix table
+  // gs[j][t] = sum_{j <= s < t} (k_t.k_s)(v_t.v_s), prefix table
+  // Q[j][t] = sum_{j <= u < t} gs[j][u], then a_t = |k_t|^2 |v_t|^2
+  float gq[2][kGramBlock];
+  uint64_t kvbar[2];                // [stage] the stage's Gram block has landed
   float red[NW][L];
   float xs[2][CL][L + 4];           // [chunk parity][CTA] parts of x_t (t < L) and of |S_open|^2 (at L)
   uint64_t xbar[2];                 // [chunk parity] the partner's parts have arrived (CTA pairs)
@@ -57,12 +58,20 @@ __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1)
   return v & (lo | hi);
 }
 
+// Next chunk's k and v rows (cp.async by every thread, zero-filled past the
+// sequence end) and its Gram block (one bulk copy by thread 0, completing on
+// `bar`).  The k, v copies are waited for with cp.async.wait_group, the Gram
+// block with the mbarrier.
 template <int D>
-__device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
-                                            const __nv_bfloat16* vs, int row_stride, int valid, float* dgs,
-                                            float* dqs, float* das, const float* gsrc) {
+__device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
+                                               const __nv_bfloat16* vs, int row_stride, int valid, float* dgq,
+                                               const float* gsrc, uint64_t* bar) {
   constexpr int RP = D + 8;
   constexpr int V16 = D / 8;
+  if (threadIdx.x == 0 && gsrc) {
+    sm100::mbar_expect_tx(bar, (uint32_t)kGramBlock * 4u);
+    sm100::bulk_g2s(dgq, gsrc, (uint32_t)kGramBlock * 4u, bar);
+  }
   for (int e = threadIdx.x; e < L * V16; e += NT) {
     const int r = e / V16, c = (e % V16) * 8;
     const int nbytes = (r < valid) ? 16 : 0;
@@ -72,17 +81,6 @@ __device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv
                  : "memory");
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dv + r * RP + c)), "l"(sv), "r"(nbytes)
                  : "memory");
-  }
-  if (gsrc) {  // suffix table gs, prefix table Q (64 x 64 each, [j][t]) and a_t from the Gram pre-pass
-    constexpr int R4 = L / 4;  // 16-byte pieces per row
-    for (int e = threadIdx.x; e < 2 * L * R4 + R4; e += NT) {
-      const int tab = e / (L * R4);  // 0: gs, 1: Q, 2: a
-      const int rem = e - tab * L * R4;
-      const int r = rem / R4, c4 = (rem % R4) * 4;
-      float* dst = (tab == 2) ? das + c4 : (tab == 0 ? dgs : dqs) + r * GS + c4;
-      const float* src = gsrc + tab * L * L + r * L + c4;
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(su32(dst)), "l"(src) : "memory");
-    }
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
@@ -306,11 +304,13 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     sm.m = m0;
     sm.pool_next = 0;
     sm.abort_flag = 0;
+    sm100::mbar_init(&sm.kvbar[0], 1);
+    sm100::mbar_init(&sm.kvbar[1], 1);
     if constexpr (CL > 1) {
       sm100::mbar_init(&sm.xbar[0], 1);
       sm100::mbar_init(&sm.xbar[1], 1);
-      sm100::fence_mbar_init();
     }
+    sm100::fence_mbar_init();
   }
   __syncthreads();
   for (int i = tid; i < C; i += NT) {
@@ -442,9 +442,9 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const int ntok = a.t_end - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
   const long long gchunk0 = (long long)bh * a.gram_chunks + a.t_begin / L;  // Gram block of the round's first chunk
-  prefetch_kv<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
-                 vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gs[0], sm.Qs[0], sm.as[0],
-                 a.gram ? a.gram + gchunk0 * kGramBlock : nullptr);
+  prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
+                      vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
+                      a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0]);
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
     const int Lc = min(L, a.t_end - t0);
@@ -452,13 +452,14 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     // ------------------------------------------------ 1. k, v of this chunk; prefetch the next
     if (c + 1 < nchunks) {
       const int t1 = t0 + L;
-      prefetch_kv<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
-                     vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gs[st ^ 1],
-                     sm.Qs[st ^ 1], sm.as[st ^ 1], a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr);
+      prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
+                        vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
+                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1]);
       asm volatile("cp.async.wait_group 1;" ::: "memory");
     } else {
       asm volatile("cp.async.wait_group 0;" ::: "memory");
     }
+    if (a.gram) sm100::mbar_wait(&sm.kvbar[st], (uint32_t)((c >> 1) & 1), &sm.abort_flag, a.status);
     if (tid < L) sm.mlog[tid] = -1;
     __syncthreads();
     const int m_chunk = sm.m;
@@ -522,17 +523,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     // Normally prefetched from the Gram pre-pass; formed here when the call has
     // no room for the pre-pass output (scan-only calls).
     if (!a.gram) {
-      float* G = sm.Qs[st ^ 1];  // scratch: nothing is prefetched into the other stage here
-      gram_tile<D>(Ks, Vs, G, sm.as[st]);
+      float* G = sm.gq[st ^ 1];  // scratch: no Gram block is prefetched into the other stage here
+      gram_tile<D>(Ks, Vs, G, sm.gq[st] + 2 * L * L);
       __syncthreads();
       suffix_rows(G);
       __syncthreads();
       for (int e = tid; e < L * L; e += NT) {  // transpose to the [j][t] layout the passes read
         const int t = e % L, j = e / L;
-        sm.gs[st][j * GS + t] = G[t * (L + 1) + j];
+        sm.gq[st][j * GS + t] = G[t * (L + 1) + j];
       }
       __syncthreads();
-      prefix_rows(sm.gs[st], GS, 1, sm.Qs[st], GS);
+      prefix_rows(sm.gq[st], GS, 1, sm.gq[st] + L * L, GS);
     }
     __syncthreads();
     if (tid < L) {  // this CTA's part of x_t
@@ -563,9 +564,9 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const float xa = (m_chunk > 0) ? whole(st, ta) : 0.f;
       const float xb = (m_chunk > 0) ? whole(st, tb) : 0.f;
       const float gam_open = (m_chunk > 0) ? whole(st, L) : 0.f;
-      const float aa = sm.as[st][ta], ab = sm.as[st][tb];
-      const float* gst = sm.gs[st];
-      const float* qst = sm.Qs[st];
+      const float* gst = sm.gq[st];
+      const float* qst = gst + L * L;
+      const float aa = gst[2 * L * L + ta], ab = gst[2 * L * L + tb];
       // exclusive prefix sums of x_t and a_t over the chunk: with the table Q,
       // sum_{js <= u < t} (2 beta_u + a_u) = 2 (X(t) - X(js)) [open state] + 2 Q[js][t] + A(t) - A(js)
       float xpa, xpb, apa, apb;
