@@ -48,6 +48,7 @@ struct MmaSmem {
   int ops[3 * L + 4][4];
   int snap_src[kMaxC][2];
   int nops, nsnapjobs;
+  int pend;                         // snapshot copies waiting for the next chunk's idle warps (bf16 pool)
   int m, cur, js, seg_pre, pool_next;
 };
 
@@ -199,6 +200,31 @@ __device__ __forceinline__ void copy_state_g(__nv_bfloat16* dst, const float* sr
     }
   }
 }
+// The same conversion by threads i0, i0 + ni, ... (any count: the deferred
+// snapshot copies run on the warps that idle during the boundary passes).
+template <int D, int NR>
+__device__ __forceinline__ void copy_state_split(__nv_bfloat16* dst, const float* src, int i0, int ni) {
+  constexpr int N4 = NR * D / 4;
+  for (int base = i0; base < N4; base += 4 * ni) {
+    float4 v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int e4 = base + i * ni;
+      v[i] = (e4 < N4) ? load4(src + e4 * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int e4 = base + i * ni;
+      if (e4 < N4) {
+        const float4 x = v[i];
+        const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
+        const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+        store4(dst + e4 * 4, make_float4(f01.x, f01.y, f23.x, f23.y));
+        store4(dst + D * D + e4 * 4, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
+      }
+    }
+  }
+}
 // dst += src over one D x D state, batched like copy_state_g.
 template <int D, int NR = D>
 __device__ __forceinline__ void add_state_g(float* dst, const float* src) {
@@ -303,6 +329,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     }
     sm.m = m0;
     sm.pool_next = 0;
+    sm.pend = 0;
     sm.abort_flag = 0;
     sm100::mbar_init(&sm.kvbar[0], 1);
     sm100::mbar_init(&sm.kvbar[1], 1);
@@ -422,6 +449,27 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         ldsm4t(bf, Ks + (t0 + (q & 1) * 8 + r8) * RP + k0 + 16 * np + (q >> 1) * 8);
         mma16816(acc[2 * np], af, bf[0], bf[1]);
         mma16816(acc[2 * np + 1], af, bf[2], bf[3]);
+      }
+    }
+  };
+  // The snapshot copies listed in sm.snap_src[0 .. n): the open state from its
+  // bf16 hi / lo operand in shared memory, closed states from their fp32 slots.
+  // Threads i0, i0 + ni, ...
+  auto snapshot_copies = [&](int n, int i0, int ni) {
+    for (int jj = 0; jj < n; ++jj) {
+      const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
+      Tpool* entry = pool + (long long)p * kEntry;
+      if constexpr (sizeof(Tpool) == 2) {
+        if (srcslot < 0) {  // coalesced 16-byte copies of the staged hi / lo rows
+          for (int e = i0; e < 2 * R * (D / 8); e += ni) {
+            const int part = e / (R * (D / 8)), rem = e % (R * (D / 8));
+            const int j = rem / (D / 8), k8 = (rem % (D / 8)) * 8;
+            *reinterpret_cast<uint4*>(entry + part * D * D + (rbase + j) * D + k8) =
+                *reinterpret_cast<const uint4*>(&sm.S2[part][j * RP + k8]);
+          }
+        } else {
+          copy_state_split<D, R>(entry + (long long)rbase * D, srows(srcslot), i0, ni);
+        }
       }
     }
   };
@@ -550,6 +598,11 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
     __syncthreads();
+    // ------------------------------------------------ 3b. the previous interval's snapshot copies (warps 1..)
+    // They read the staged open state and closed slots, which only the state
+    // updates and the publish below change, so they overlap warp 0's passes.
+    if constexpr (sizeof(Tpool) == 2)
+      if (warp != 0 && sm.pend > 0) snapshot_copies(sm.pend, tid - 32, NT - 32);
     // ------------------------------------------------ 4. boundary passes (warp 0, tokens 2 lane, 2 lane + 1)
     // Each pass scores every undecided token as if the open segment ran to it,
     // takes the first that fires, and restarts the segment there.
@@ -730,6 +783,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
     __syncthreads();
+    if (tid == 0) sm.pend = 0;  // every warp is past the deferred copies (read before this barrier)
     // ------------------------------------------------ 6. state updates (this CTA's rows)
     {
       const int nops = sm.nops;
@@ -793,31 +847,32 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           if (lead) a.snap_m0[lrow] = m;
         }
       }
-      __syncthreads();
-      for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
-        const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
-        Tpool* entry = pool + (long long)p * kEntry;
-        if (srcslot < 0) {  // the open state
-          if constexpr (sizeof(Tpool) == 2) {
-            // bf16 hi / lo are already staged in shared memory: coalesced 16-byte copies
-            for (int e = tid; e < 2 * R * (D / 8); e += NT) {
-              const int part = e / (R * (D / 8)), rem = e % (R * (D / 8));
-              const int j = rem / (D / 8), k8 = (rem % (D / 8)) * 8;
-              *reinterpret_cast<uint4*>(entry + part * D * D + (rbase + j) * D + k8) =
-                  *reinterpret_cast<const uint4*>(&sm.S2[part][j * RP + k8]);
-            }
-          } else {  // fp32 pool: straight from the accumulators
+      if constexpr (sizeof(Tpool) == 2) {
+        if (tid == 0) sm.pend = sm.nsnapjobs;  // copied during the next chunk's passes (or at round end)
+        __syncthreads();
+      } else {  // fp32 pool (d = 64): copied now, the open state straight from the accumulators
+        __syncthreads();
+        for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
+          const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
+          Tpool* entry = pool + (long long)p * kEntry;
+          if (srcslot < 0) {
 #pragma unroll
             for (int n = 0; n < NT8; ++n) {
               const int k = k0 + 8 * n + 2 * tg;
               put_pair(entry, D, jg0 + g, k, acc[n][0], acc[n][1]);
               put_pair(entry, D, jg0 + g + 8, k, acc[n][2], acc[n][3]);
             }
+          } else {
+            copy_state_g<D, R>(entry + (long long)rbase * D, srows(srcslot));
           }
-        } else {
-          copy_state_g<D, R>(entry + (long long)rbase * D, srows(srcslot));
         }
+        __syncthreads();
       }
+    }
+  }
+  if constexpr (sizeof(Tpool) == 2) {  // the last interval's copies, if no chunk followed
+    if (sm.pend > 0) {
+      snapshot_copies(sm.pend, tid, NT);
       __syncthreads();
     }
   }
