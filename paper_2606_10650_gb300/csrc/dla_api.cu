@@ -5,9 +5,11 @@
 // kernels of dla_scan.cu / dla_readout_*.cu / dla_decode.cu.
 #include <math.h>
 #include <algorithm>
+#include <mutex>
 #include <stdarg.h>
 #include <vector>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "dla.h"
@@ -74,7 +76,7 @@ struct FwdPlan {
   int nbuf;          // pools (1 persistent, 2 reset with several rounds)
   int pool_cap;      // pool entries per stream, per pool
   size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram, off_ointra,
-      off_pool, pool_bytes;
+      off_progress, off_pool, pool_bytes;
   int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
   size_t total;
 };
@@ -119,6 +121,8 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
   // intra-interval read-out part of one round (tensor-core read-out), fp32
   P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + BH * (size_t)R * P.interval * d * 4);
+  // scan progress per (stream, CTA) and the count of started scan CTAs (concurrent read-out)
+  P.off_progress = off;  if (with_output) off = align256(off + (2 * BH + 1) * sizeof(int32_t));
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
@@ -155,6 +159,16 @@ void finish_score_params(ScoreParams& sp) {
 }  // namespace dla
 
 namespace {
+
+// Schedule of the tensor-core forward pass (environment variable DLA_SCHEDULE,
+// read at every call): "rounds" (default) launches the scan once per round and
+// the round's read-out after it; "concurrent" launches the scan once over the
+// whole sequence and the read-out rounds beside it, each read-out CTA waiting
+// for its stream's progress.  Both compute the same results.
+bool concurrent_schedule() {
+  const char* v = getenv("DLA_SCHEDULE");
+  return v && strcmp(v, "concurrent") == 0;
+}
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
@@ -493,6 +507,66 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
   if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
   const std::vector<int> sizes = round_sizes(P);
+  if (P.persistent && tc && concurrent_schedule()) {
+    // One scan over the whole sequence (high-priority stream) and the read-out
+    // in rounds beside it (low-priority stream): each read-out CTA waits for its
+    // stream's progress, so rounds never wait for the slowest stream and the
+    // scan is launched once.  A one-CTA gate holds the read-out stream until
+    // every scan CTA has started, so a waiting read-out CTA never holds an SM
+    // the scan needs.
+    {  // kernel code loaded once per device before anything of this path runs
+      static bool loaded[kMaxDev] = {};
+      static std::mutex mu;
+      int dev = 0;
+      if ((e = cudaGetDevice(&dev)) != cudaSuccess || dev < 0 || dev >= kMaxDev) return cuda_fail(e, "device query");
+      std::lock_guard<std::mutex> g(mu);
+      if (!loaded[dev]) {
+        if ((e = dla::preload_scan_kernels()) != cudaSuccess || (e = dla::preload_readout_kernels()) != cudaSuccess)
+          return cuda_fail(e, "kernel load");
+        loaded[dev] = true;
+      }
+    }
+    int32_t* progress = (int32_t*)(ws + P.off_progress);
+    int32_t* started = progress + 2 * B * H;
+    const int ctas = dla::scan_mma_ctas_per_stream(B * H, d);
+    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1) * sizeof(int32_t), S->hi)) != cudaSuccess)
+      return cuda_fail(e, "progress reset");
+    if (P.gram_chunks) {  // K0 over the whole sequence, on every SM
+      dla::GramArgs ga;
+      ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+      ga.out = (float*)(ws + P.off_gram);
+      ga.chunk0 = 0; ga.count = P.gram_chunks;
+      e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
+      if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+    }
+    if ((e = cudaEventRecord(S->gram_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(S->lo, S->gram_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    if ((e = dla::launch_gate(started, B * H * ctas, status, S->lo)) != cudaSuccess) return cuda_fail(e, "gate launch");
+    sa.pool = ws + P.off_pool;
+    sa.t_begin = 0; sa.t_end = T;
+    sa.nsnap = P.nsnap_total; sa.snap_base = 0;
+    sa.carry_in = 0; sa.snap_at_end = 0;
+    sa.progress = progress; sa.started = started;
+    e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    ra.pool = sa.pool;
+    ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
+    int snap0 = 0;
+    for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
+      ra.t_begin = snap0 * P.interval;
+      ra.t_end = std::min(T, ra.t_begin + sizes[r] * P.interval);
+      ra.nsnap = sizes[r]; ra.snap_base = snap0;
+      e = timed(DLA_K_READOUT_INTRA, S->lo, [&] { return dla::launch_readout_intra(ra, S->lo); });
+      if (e != cudaSuccess) return cuda_fail(e, "intra read-out launch");
+      e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
+      if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+    }
+    if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaEventRecord(S->ro_done[0], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    if ((e = cudaStreamWaitEvent(st, S->ro_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    return ok();
+  }
   bool gram_rest = false;  // the scan of round 1 waits for the Gram tables of rounds 1..
   if (P.gram_chunks) {
     // K0: Gram suffix tables.  Round 0's chunks run ahead of the first scan on

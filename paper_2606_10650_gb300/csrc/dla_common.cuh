@@ -70,6 +70,32 @@ __device__ __forceinline__ float info_score_fast(float a, float beta, float gam,
   return __fdividef(nrm, y + p.eps_f);
 }
 
+// ---- flags shared with a concurrently running kernel
+__device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Read-out side: thread 0 waits until the scan CTAs of stream bh have completed
+// `need` intervals (progress[bh][0 .. ctas)), at most ~2 s (then status 5);
+// the caller's CTA barrier then orders every later read after the wait.  Data
+// the scan writes must then be read past L1 (__ldcg): another CTA on the SM may
+// hold an older copy of the line.
+__device__ __forceinline__ void wait_progress(const int32_t* progress, int ctas, int bh, int need, int32_t* status) {
+  if (!progress || threadIdx.x != 0) return;
+  const long long t0 = clock64();
+  for (int r = 0; r < ctas; ++r)
+    while (ld_acquire_gpu(progress + 2 * bh + r) < need) {
+      if (clock64() - t0 > 4000000000LL) {
+        atomicExch(status, 5);
+        return;
+      }
+    }
+}
+
 template <typename T>
 __device__ __forceinline__ float to_f32(T x);
 template <>

@@ -59,6 +59,8 @@ struct ScanArgs {
   int32_t* pstate;       // [B*H] next free pool entry, then [B*H][C] pool ids of the live entries
   const float* gram;     // Gram pre-pass output [B*H][gram_chunks][kGramBlock], or nullptr
   int gram_chunks;       // 64-token chunks of the whole sequence
+  int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
+  int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)
 };
 
@@ -98,6 +100,9 @@ struct ReadoutArgs {
   int interval;          // tokens per snapshot interval
   float* ointra;         // [B*H][ointra_T][d] fp32 intra-interval part (tensor-core path), token t - t_begin
   int ointra_T;          // tokens per stream in ointra (one round)
+  const int32_t* progress;  // [B*H][2] scan progress to wait for (the scan runs concurrently), or nullptr
+  int progress_ctas;        // scan CTAs per stream (1 or 2): entries of progress[bh] that count
+  int32_t* status;          // device status word
 };
 
 // K3: one decode step of every stream.
@@ -126,6 +131,20 @@ dla_status set_error(dla_status s, const char* fmt, ...);
 cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 // K1 for bf16 inputs with its contractions on mma.sync (dla_scan_mma.cu).
 cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s);
+// CTAs per stream of launch_scan_mma: 2 (a CTA pair) when 2*B*H CTAs fit the
+// device's SMs in one wave with d = 128, else 1.
+int scan_mma_ctas_per_stream(int BH, int d);
+// One CTA that returns once `n` scan CTAs have started (*started >= n), or after
+// ~2 s with status 5: the read-out stream runs it before its first launch, so
+// that read-out CTAs waiting for the scan never hold the SMs the scan needs.
+cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStream_t s);
+// Loads the code of the kernels of the concurrent scan / read-out path on the
+// current device (cudaFuncGetAttributes).  With lazy module loading, a kernel's
+// first launch can wait for the device's running kernels, and a read-out
+// waiting for a scan whose code is not loaded yet would wait until its time
+// limit: the forward pass calls these before its first launch.
+cudaError_t preload_scan_kernels();
+cudaError_t preload_readout_kernels();
 cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s);
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);

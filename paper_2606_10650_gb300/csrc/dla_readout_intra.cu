@@ -70,7 +70,11 @@ __global__ void __launch_bounds__(NT, 2) readout_intra_kernel(ReadoutArgs a) {
   const int C = a.C;
   const int c0 = a.t_begin + s * L;
   const int Lc = min(L, a.t_end - c0);
-  const int m0 = a.snap_m0[(long long)bh * a.snap_stride + a.snap_base + s];
+  // with a scan running concurrently: the interval must be complete; its list
+  // and trace are then read past L1 (__ldcg)
+  wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + s + 1, a.status);
+  __syncthreads();
+  const int m0 = __ldcg(a.snap_m0 + (long long)bh * a.snap_stride + a.snap_base + s);
   const long long rowbase = ((long long)b * a.T + c0) * a.H + h;
   const long long row_stride = (long long)a.H * D;
   const __nv_bfloat16* qg = reinterpret_cast<const __nv_bfloat16*>(a.q) + rowbase * D;
@@ -83,8 +87,8 @@ __global__ void __launch_bounds__(NT, 2) readout_intra_kernel(ReadoutArgs a) {
   asm volatile("cp.async.commit_group;" ::: "memory");
   if (tid < L) {
     const bool in = tid < Lc;
-    sm.bnd[tid] = in ? a.boundary[(long long)bh * a.T + c0 + tid] : (uint8_t)0;
-    sm.mlog[tid] = in ? a.merge_log[(long long)bh * a.T + c0 + tid] : -1;
+    sm.bnd[tid] = in ? __ldcg(a.boundary + (long long)bh * a.T + c0 + tid) : (uint8_t)0;
+    sm.mlog[tid] = in ? __ldcg(a.merge_log + (long long)bh * a.T + c0 + tid) : -1;
   }
   asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncthreads();
@@ -216,6 +220,11 @@ __global__ void __launch_bounds__(NT, 2) readout_intra_kernel(ReadoutArgs a) {
       if (tb < Lc) *reinterpret_cast<float2*>(col + tb * 4) = make_float2(o[n][2], o[n][3]);
     }
   }
+}
+
+cudaError_t preload_readout_intra() {
+  cudaFuncAttributes fa;
+  return cudaFuncGetAttributes(&fa, readout_intra_kernel<128>);
 }
 
 cudaError_t launch_readout_intra(const ReadoutArgs& a, cudaStream_t st) {

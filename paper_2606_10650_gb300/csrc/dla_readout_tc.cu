@@ -119,11 +119,15 @@ __global__ void __launch_bounds__(NT, 1)
   const int C = a.C;
   const int sA = 2 * pair;
   const bool hasB = (sA + 1) < a.nsnap;
+  // with a scan running concurrently: both intervals of the pair must be complete
+  wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + sA + (hasB ? 2 : 1), a.status);
+  __syncthreads();
   // interval A (side 0) and B (side 1) of the pair
   const int c0A = a.t_begin + sA * L, c0B = c0A + L;
   const int LcA = min(L, a.t_end - c0A), LcB = hasB ? min(L, a.t_end - c0B) : 0;
   const long long lrowA = (long long)bh * a.snap_stride + a.snap_base + sA, lrowB = lrowA + 1;
-  const int m0A = a.snap_m0[lrowA], m0B = hasB ? a.snap_m0[lrowB] : 0;
+  // lists and trace come from the scan: read past L1 (__ldcg)
+  const int m0A = __ldcg(a.snap_m0 + lrowA), m0B = hasB ? __ldcg(a.snap_m0 + lrowB) : 0;
   auto c0_of = [&](int side) { return side ? c0B : c0A; };
   auto Lc_of = [&](int side) { return side ? LcB : LcA; };
   volatile int* abort = &sm.abort_flag;
@@ -154,7 +158,7 @@ __global__ void __launch_bounds__(NT, 1)
   }
   for (int i = tid; i < 2 * kMaxC; i += NT) {
     const int side = i / kMaxC, x = i % kMaxC;
-    sm.ids[side][x] = (x < (side ? m0B : m0A)) ? a.snap_ids[(side ? lrowB : lrowA) * C + x] : -1;
+    sm.ids[side][x] = (x < (side ? m0B : m0A)) ? __ldcg(a.snap_ids + (side ? lrowB : lrowA) * C + x) : -1;
   }
   if (warp == 1) tmem_alloc(&sm.tmem_base, kTmemCols);
   __syncthreads();
@@ -259,8 +263,8 @@ __global__ void __launch_bounds__(NT, 1)
       const int side = etid / L, tt = etid % L;
       const bool in = tt < Lc_of(side);
       const long long tr = (long long)bh * a.T + c0_of(side) + tt;
-      sm.side[side].bnd[tt] = in ? a.boundary[tr] : (uint8_t)0;
-      sm.side[side].mlog[tt] = in ? a.merge_log[tr] : -1;
+      sm.side[side].bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
+      sm.side[side].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
     }
     // o starts from the intra-interval parts (K2a; column-quad order, so a warp
     // reads 512 contiguous bytes per load)
@@ -413,5 +417,12 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
 }
 
 size_t readout_tc_smem_bytes() { return sizeof(TcSmem) + 1024; }
+
+cudaError_t preload_readout_intra();
+cudaError_t preload_readout_kernels() {
+  cudaFuncAttributes fa;
+  cudaError_t e = cudaFuncGetAttributes(&fa, readout_tc_kernel);
+  return (e != cudaSuccess) ? e : preload_readout_intra();
+}
 
 }  // namespace dla

@@ -322,6 +322,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 
   // ---------------------------------------------------------------- round start
   if (tid == 0) {
+    if (a.started) atomicAdd(a.started, 1);  // the read-out stream's gate counts the resident scan CTAs
     int m0 = a.m[bh];
     if (m0 < 0 || m0 > C) {
       atomicExch(a.status, 6);
@@ -850,6 +851,9 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       if constexpr (sizeof(Tpool) == 2) {
         if (tid == 0) sm.pend = sm.nsnapjobs;  // copied during the next chunk's passes (or at round end)
         __syncthreads();
+        // interval snap_base + snap_idx - 1 is complete: its trace is written and its
+        // starting snapshot was copied during its first chunk (a concurrent read-out waits for this)
+        if (a.progress && tid == NT - 32) st_release_gpu(a.progress + 2 * bh + rank, a.snap_base + snap_idx);
       } else {  // fp32 pool (d = 64): copied now, the open state straight from the accumulators
         __syncthreads();
         for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
@@ -875,6 +879,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       snapshot_copies(sm.pend, tid, NT);
       __syncthreads();
     }
+  }
+  if (a.progress) {  // every interval of this launch is complete
+    __syncthreads();
+    if (tid == 0) st_release_gpu(a.progress + 2 * bh + rank, a.snap_base + a.nsnap);
   }
   // ---------------------------------------------------------------- round end
   {
@@ -1001,12 +1009,35 @@ static cudaError_t launch_scan_mma_t(const ScanArgs& a, cudaStream_t s) {
   return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
-// CTA pairs when two CTAs per stream still fit on the device in one wave.
-static bool use_pairs(const ScanArgs& a) {
+int scan_mma_ctas_per_stream(int BH, int d) {
   int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return false;
-  return 2LL * a.B * a.H <= sms;
+  if (d != 128 || cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 1;
+  return (2LL * BH <= sms) ? 2 : 1;
+}
+// CTA pairs when two CTAs per stream still fit on the device in one wave.
+static bool use_pairs(const ScanArgs& a) { return scan_mma_ctas_per_stream(a.B * a.H, 128) == 2; }
+
+__global__ void gate_kernel(const int32_t* started, int n, int32_t* status) {
+  const long long t0 = clock64();
+  while (ld_acquire_gpu(started) < n)
+    if (clock64() - t0 > 4000000000LL) {  // ~2 s
+      atomicExch(status, 5);
+      return;
+    }
+}
+cudaError_t preload_scan_kernels() {
+  cudaFuncAttributes fa;
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, gram_kernel<128>)) != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, gate_kernel);
+}
+cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStream_t s) {
+  gate_kernel<<<1, 1, 0, s>>>(started, n, status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s) {

@@ -169,3 +169,44 @@ def test_decode_steps_match_prefill():
     g = dict(boundary=r["boundary"], merge_log=r["merge_log"], o=None, cache=cache)
     compare(w, g, r)
     assert b_all.sum() > 0 and (m_all >= 0).sum() > 0
+
+
+@pytest.mark.parametrize("case", ["standard_bf16", "regime_bf16", "long_churn_bf16"])
+def test_forward_parity_concurrent_schedule(case, monkeypatch):
+    """The concurrent schedule (one scan over the whole sequence, read-out
+    waiting on per-stream progress) gives the oracle's results too."""
+    monkeypatch.setenv("DLA_SCHEDULE", "concurrent")
+    name, ov = CASES[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+    structural_checks(w, g, w.T)
+
+
+def test_concurrent_schedule_first_call_of_a_process():
+    """The first forward pass of a process under the concurrent schedule loads
+    every kernel before the read-out starts waiting for the scan (a lazily
+    loaded scan would otherwise stall behind the waiting read-out)."""
+    import os
+    import subprocess
+    import sys
+    code = (
+        "import numpy as np, torch\n"
+        "from paper_2606_10650_gb300 import dla, workloads as W\n"
+        "w = W.get('standard', B=1, H=2, T=700)\n"
+        "q, k, v, lam = W.host_batch(w, T=w.T)\n"
+        "dev = torch.device('cuda:0')\n"
+        "qt, kt, vt = (W.to_device(x, w.dtype, dev) for x in (q, k, v))\n"
+        "o = torch.empty(qt.shape, dtype=torch.float32, device=dev)\n"
+        "cache = dla.Cache(1, 2, w.C, 128, device=dev)\n"
+        "p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)\n"
+        "ws = dla.dla_forward(p, qt, kt, vt, None, o, cache, None, None)\n"
+        "torch.cuda.synchronize()\n"
+        "print('STATUS', dla.workspace_status(ws))\n")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, DLA_SCHEDULE="concurrent", PYTHONPATH=root)
+    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr[-2000:]
+    assert "STATUS 0" in out.stdout, out.stdout[-2000:]
