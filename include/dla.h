@@ -140,12 +140,12 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
  *   read them after synchronising the stream.
  *   Schedule (bf16, d = 128, workspace of at least dla_forward_workspace(...)):
  *   the environment variable DLA_SCHEDULE, read at every call, selects
- *   "rounds" (default: the scan and the read-out alternate round by round on
- *   two internal streams) or "concurrent" (the scan runs once over the whole
- *   sequence while the read-out follows it on another stream, waiting for each
- *   stream's progress; a kernel of the read-out stream waits up to ~2 s for the
- *   scan to become resident, so the device should not be saturated by other
- *   work at that moment).  Both give the same results. */
+ *   "concurrent" (default: the scan runs once over the whole sequence while
+ *   the read-out follows it on other streams, waiting for each stream's
+ *   progress; a kernel of the read-out side waits up to ~2 s for the scan to
+ *   become resident, so the device should not be saturated by other work at
+ *   that moment) or "rounds" (the scan and the read-out alternate round by
+ *   round on two internal streams).  Both give the same results. */
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,

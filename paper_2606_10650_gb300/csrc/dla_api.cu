@@ -120,7 +120,8 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
   // intra-interval read-out part of one round (tensor-core read-out), fp32
-  P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + BH * (size_t)R * P.interval * d * 4);
+  // (two buffers: in the concurrent schedule the next round's intra part overlaps this round's snapshot part)
+  P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + 2 * BH * (size_t)R * P.interval * d * 4);
   // scan progress per (stream, CTA) and the count of started scan CTAs (concurrent read-out)
   P.off_progress = off;  if (with_output) off = align256(off + (2 * BH + 1) * sizeof(int32_t));
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
@@ -161,13 +162,13 @@ void finish_score_params(ScoreParams& sp) {
 namespace {
 
 // Schedule of the tensor-core forward pass (environment variable DLA_SCHEDULE,
-// read at every call): "rounds" (default) launches the scan once per round and
-// the round's read-out after it; "concurrent" launches the scan once over the
+// read at every call): "concurrent" (default) launches the scan once over the
 // whole sequence and the read-out rounds beside it, each read-out CTA waiting
-// for its stream's progress.  Both compute the same results.
+// for its stream's progress; "rounds" launches the scan once per round and the
+// round's read-out after it.  Both compute the same results.
 bool concurrent_schedule() {
   const char* v = getenv("DLA_SCHEDULE");
-  return v && strcmp(v, "concurrent") == 0;
+  return !(v && strcmp(v, "rounds") == 0);
 }
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
@@ -209,8 +210,9 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
 // thread and device: the scan runs on a high-priority stream, the read-out on
 // a low-priority one, so the scan's few CTAs get SMs first.
 struct StreamSet {
-  cudaStream_t hi = nullptr, lo = nullptr;
+  cudaStream_t hi = nullptr, lo = nullptr, lo2 = nullptr;  // scan, snapshot read-out, intra read-out
   cudaEvent_t in = nullptr, gram_done = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
+  cudaEvent_t gate_done = nullptr, intra_done[2] = {nullptr, nullptr}, tc_done[2] = {nullptr, nullptr};
   bool ready = false;
 };
 constexpr int kMaxDev = 64;
@@ -229,6 +231,12 @@ cudaError_t stream_set(StreamSet** out) {
     if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.gram_done, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaStreamCreateWithPriority(&S.lo2, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&S.gate_done, cudaEventDisableTiming)) != cudaSuccess) return e;
+    for (int i = 0; i < 2; ++i) {
+      if ((e = cudaEventCreateWithFlags(&S.intra_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+      if ((e = cudaEventCreateWithFlags(&S.tc_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
     for (int i = 0; i < 2; ++i) {
       if ((e = cudaEventCreateWithFlags(&S.scan_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
       if ((e = cudaEventCreateWithFlags(&S.ro_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
@@ -484,6 +492,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   ra.out_bf16 = (p->out_dtype == DLA_BF16);
   ra.B = B; ra.T = T; ra.H = H; ra.C = C;
   ra.boundary = bnd; ra.merge_log = mlog;
+  ra.status = status;
   ra.interval = P.interval;
   sa.snap_chunks = P.interval / dla::kScanL;
   sa.pool_cap = P.pool_cap;
@@ -551,16 +560,28 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     ra.pool = sa.pool;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
+    // K2a of round r on lo2 into intra buffer r % 2, K2b of round r on lo after it;
+    // K2a of round r + 2 reuses the buffer once K2b of round r is done
+    if ((e = cudaEventRecord(S->gate_done, S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(S->lo2, S->gate_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    float* intra_buf[2] = {ra.ointra, ra.ointra + (size_t)B * H * ra.ointra_T * d};
     int snap0 = 0;
     for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
       ra.t_begin = snap0 * P.interval;
       ra.t_end = std::min(T, ra.t_begin + sizes[r] * P.interval);
       ra.nsnap = sizes[r]; ra.snap_base = snap0;
-      e = timed(DLA_K_READOUT_INTRA, S->lo, [&] { return dla::launch_readout_intra(ra, S->lo); });
+      ra.ointra = intra_buf[r & 1];
+      if (r >= 2 && (e = cudaStreamWaitEvent(S->lo2, S->tc_done[r & 1], 0)) != cudaSuccess)
+        return cuda_fail(e, "stream wait");
+      e = timed(DLA_K_READOUT_INTRA, S->lo2, [&] { return dla::launch_readout_intra(ra, S->lo2); });
       if (e != cudaSuccess) return cuda_fail(e, "intra read-out launch");
+      if ((e = cudaEventRecord(S->intra_done[r & 1], S->lo2)) != cudaSuccess) return cuda_fail(e, "event record");
+      if ((e = cudaStreamWaitEvent(S->lo, S->intra_done[r & 1], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+      if ((e = cudaEventRecord(S->tc_done[r & 1], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     }
+    ra.ointra = intra_buf[0];
     if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaEventRecord(S->ro_done[0], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");

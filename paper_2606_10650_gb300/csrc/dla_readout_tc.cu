@@ -22,10 +22,9 @@
 // 2..9 read TMEM, weight by lambda and accumulate both intervals' o in registers
 // (warp w reads TMEM lane quadrant w % 4; warps 2-5 own columns 0-63, warps 6-9
 // own 64-127).
-#include <cudaTypedefs.h>
-
 #include "dla_common.cuh"
 #include "dla_sm100.cuh"
+#include "dla_tmap.h"
 
 namespace dla {
 
@@ -311,7 +310,8 @@ __global__ void __launch_bounds__(NT, 1)
       const float wA = wnA, wB = wnB;
       wnA = weight(0, x + 1);
       wnB = weight(1, x + 1);
-      if (!mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status)) break;
+      // tcgen05.ld below is warp-wide: the warp takes one decision
+      if (!__all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status))) break;
       tc_fence_after();
       float dv[16];
       const uint32_t base = lane_addr + 256u * buf + 64 * ch;
@@ -361,53 +361,10 @@ __global__ void __launch_bounds__(NT, 1)
 }
 
 // ---------------------------------------------------------------- host side
-namespace {
-
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
-  return fn;
-}
-
-// [B, T, H, 128] bf16 rows of one stream: dims (k, h, t, b), box (64, 1, 128, 1).
-bool map_tokens(CUtensorMap* m, const void* base, int B, int T, int H) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
-  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2, (cuuint64_t)T * H * D * 2};
-  cuuint32_t box[4] = {64, 1, (cuuint32_t)L, 1};
-  cuuint32_t es[4] = {1, 1, 1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// Snapshot pool as rows of 128 bf16: box (64, 128).
-bool map_pool(CUtensorMap* m, const void* base, long long rows) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-  cuuint32_t box[2] = {64, (cuuint32_t)L};
-  cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-}  // namespace
-
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
   CUtensorMap mq, ms;
   const long long rows = (long long)a.B * a.H * a.pool_cap * 2 * D;
-  if (!map_tokens(&mq, a.q, a.B, a.T, a.H) || !map_pool(&ms, a.pool, rows)) return cudaErrorInvalidValue;
+  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows)) return cudaErrorInvalidValue;
   const size_t smem = sizeof(TcSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;

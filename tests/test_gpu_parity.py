@@ -172,10 +172,10 @@ def test_decode_steps_match_prefill():
 
 
 @pytest.mark.parametrize("case", ["standard_bf16", "regime_bf16", "long_churn_bf16"])
-def test_forward_parity_concurrent_schedule(case, monkeypatch):
-    """The concurrent schedule (one scan over the whole sequence, read-out
-    waiting on per-stream progress) gives the oracle's results too."""
-    monkeypatch.setenv("DLA_SCHEDULE", "concurrent")
+def test_forward_parity_rounds_schedule(case, monkeypatch):
+    """The rounds schedule (scan and read-out alternating round by round)
+    gives the oracle's results too."""
+    monkeypatch.setenv("DLA_SCHEDULE", "rounds")
     name, ov = CASES[case]
     w = W.get(name, **ov)
     q, k, v, lam = _safe(w)
@@ -206,7 +206,8 @@ def test_concurrent_schedule_first_call_of_a_process():
         "torch.cuda.synchronize()\n"
         "print('STATUS', dla.workspace_status(ws))\n")
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    env = dict(os.environ, DLA_SCHEDULE="concurrent", PYTHONPATH=root)
+    env = dict(os.environ, PYTHONPATH=root)
+    env.pop("DLA_SCHEDULE", None)  # the default schedule is the concurrent one
     out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
     assert out.returncode == 0, out.stderr[-2000:]
     assert "STATUS 0" in out.stdout, out.stdout[-2000:]
