@@ -19,9 +19,9 @@
 // Roles: warp 0 issues TMA loads (the two Q tiles, then the hi and lo parts of
 // each union state into four 32 KB half-stages), warp 1 issues tcgen05.mma (one
 // thread) into two TMEM buffers of two 128-column accumulators (A, B), warps
-// 2..9 read TMEM, weight by lambda and accumulate both intervals' o in registers
-// (warp w reads TMEM lane quadrant w % 4; warps 2-5 own columns 0-63, warps 6-9
-// own 64-127).
+// 2..17 read TMEM, weight by lambda and accumulate o in registers (one token
+// row, one interval and one 64-column half per thread; warp w reads TMEM lane
+// quadrant w % 4).
 #include "dla_common.cuh"
 #include "dla_sm100.cuh"
 #include "dla_tmap.h"
@@ -34,8 +34,8 @@ using namespace sm100;
 
 constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
-constexpr int NT = 320;  // 10 warps
-constexpr int NEPI = 8;  // epilogue warps
+constexpr int NT = 576;   // 18 warps
+constexpr int NEPI = 16;  // epilogue warps
 constexpr int NHS = 4;   // shared-memory half-stages
 constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
 constexpr int MAXU = 2 * kMaxC;  // union of two lists
@@ -251,106 +251,91 @@ __global__ void __launch_bounds__(NT, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue warps
-    const int ew = warp - 2;            // 0..7
-    const int quad = warp & 3;          // TMEM lane quadrant of this warp
-    const int ch = (warp < 6) ? 0 : 1;  // column half
-    const int t = quad * 32 + lane;     // token row of this thread (in both intervals)
+    // 16 warps: warp w reads TMEM lane quadrant w % 4; epilogue warp ew = w - 2
+    // owns interval (ew / 4) % 2 and the 64-column half ew / 8 of its rows.
+    const int ew = warp - 2;              // 0..15
+    const int quad = warp & 3;            // TMEM lane quadrant of this warp
+    const int side = (ew >> 2) & 1;       // interval A (0) or B (1)
+    const int ch = ew >> 3;               // column half
+    const int t = quad * 32 + lane;       // token row of this thread
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-    const int etid = ew * 32 + lane;    // 0..255
+    const int etid = ew * 32 + lane;      // 0..511
+    const int c0s = c0_of(side), Lcs = Lc_of(side);
 
-    {  // both intervals' boundary flags and merge indices (thread etid: interval etid / L, token etid % L)
-      const int side = etid / L, tt = etid % L;
-      const bool in = tt < Lc_of(side);
-      const long long tr = (long long)bh * a.T + c0_of(side) + tt;
-      sm.side[side].bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
-      sm.side[side].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
+    if (etid < 2 * L) {  // both intervals' boundary flags and merge indices
+      const int sd = etid / L, tt = etid % L;
+      const bool in = tt < Lc_of(sd);
+      const long long tr = (long long)bh * a.T + c0_of(sd) + tt;
+      sm.side[sd].bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
+      sm.side[sd].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
     }
-    // o starts from the intra-interval parts (K2a; column-quad order, so a warp
+    // o starts from the intra-interval part (K2a; column-quad order, so a warp
     // reads 512 contiguous bytes per load)
-    float o[2][64];
-#pragma unroll
-    for (int side = 0; side < 2; ++side) {
-      const float* src =
-          a.ointra + ((long long)bh * a.ointra_T + (c0_of(side) - a.t_begin)) * D + (16 * ch * L + t) * 4;
+    float o[64];
+    {
+      const float* src = a.ointra + ((long long)bh * a.ointra_T + (c0s - a.t_begin)) * D + (16 * ch * L + t) * 4;
 #pragma unroll
       for (int i = 0; i < 64; i += 4) {
         float4 v4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (t < Lc_of(side)) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
-        o[side][i] = v4.x; o[side][i + 1] = v4.y; o[side][i + 2] = v4.z; o[side][i + 3] = v4.w;
+        if (t < Lcs) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
+        o[i] = v4.x; o[i + 1] = v4.y; o[i + 2] = v4.z; o[i + 3] = v4.w;
       }
     }
-    asm volatile("bar.sync 1, 256;" ::: "memory");
-    if (ew == 0) build_table(sm.side[0], sm.logi, m0A, lane);
-    asm volatile("bar.sync 1, 256;" ::: "memory");  // logi is shared by the two builds
-    if (ew == 0) build_table(sm.side[1], sm.logi, m0B, lane);
-    {
-      const int side = etid / L, tt = etid % L;  // warps 2-5: interval A, 6-9: interval B
-      sm.side[side].evt[tt] = events_before(sm.side[side], tt, lane);
+    asm volatile("bar.sync 1, 512;" ::: "memory");
+    if (ew == 0) {  // both slot tables (they share logi)
+      build_table(sm.side[0], sm.logi, m0A, lane);
+      __syncwarp();
+      build_table(sm.side[1], sm.logi, m0B, lane);
     }
-    asm volatile("bar.sync 1, 256;" ::: "memory");
-    const float* lam[2];
-    const unsigned char* tabt[2];
-#pragma unroll
-    for (int side = 0; side < 2; ++side) {
-      const long long rowbase = ((long long)b * a.T + c0_of(side)) * a.H + h;
-      lam[side] = (a.lam && t < Lc_of(side)) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
-      tabt[side] = sm.side[side].tab + sm.side[side].evt[t] * kMaxC;
+    if (etid < 2 * L) {
+      const int sd = etid / L, tt = etid % L;
+      sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
     }
-    // weight of union state x for this token in interval side (0 when not in its list)
-    auto weight = [&](int side, int x) -> float {
-      if (x >= nu || t >= Lc_of(side)) return 0.f;
-      const int xi = side ? sm.uxb[x] : sm.uxa[x];
+    asm volatile("bar.sync 1, 512;" ::: "memory");
+    const long long rowbase = ((long long)b * a.T + c0s) * a.H + h;
+    const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
+    const unsigned char* tab_t = sm.side[side].tab + sm.side[side].evt[t] * kMaxC;
+    const int* ux = side ? sm.uxb : sm.uxa;
+    // weight of union state x for this token (0 when not in its interval's list)
+    auto weight = [&](int x) -> float {
+      if (x >= nu || t >= Lcs) return 0.f;
+      const int xi = ux[x];
       if (xi < 0) return 0.f;
-      return lam[side] ? lam[side][tabt[side][xi]] : 1.f;
+      return lam_t ? lam_t[tab_t[xi]] : 1.f;
     };
-    float wnA = weight(0, 0), wnB = weight(1, 0);
+    float wn = weight(0);
     for (int x = 0; x < nu; ++x) {
       const int buf = x % NBUF, kb = x / NBUF;
-      const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
-      const float wA = wnA, wB = wnB;
-      wnA = weight(0, x + 1);
-      wnB = weight(1, x + 1);
+      const bool in = (side == 0 || hasB) && ux[x] >= 0;  // warp-uniform
+      const float wx = wn;
+      wn = weight(x + 1);
       // tcgen05.ld below is warp-wide: the warp takes one decision
       if (!__all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status))) break;
       tc_fence_after();
-      float dv[16];
-      const uint32_t base = lane_addr + 256u * buf + 64 * ch;
-      if (inA) {
+      if (in) {
+        float dv[16];
+        const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
 #pragma unroll
         for (int c = 0; c < 64; c += 16) {
           tmem_ld16(base + c, dv);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) o[0][c + i] += wA * dv[i];
-        }
-      }
-      if (inB) {
-#pragma unroll
-        for (int c = 0; c < 64; c += 16) {
-          tmem_ld16(base + 128 + c, dv);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[1][c + i] += wB * dv[i];
+          for (int i = 0; i < 16; ++i) o[c + i] += wx * dv[i];
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
     }
-    if (!*abort) {
+    if (!*abort && t < Lcs) {
+      const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
+      if (a.out_bf16) {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
 #pragma unroll
-      for (int side = 0; side < 2; ++side) {
-        if (t >= Lc_of(side)) continue;
-        const long long orow = (((long long)b * a.T + c0_of(side) + t) * a.H + h) * D + 64 * ch;
-        if (a.out_bf16) {
-          __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
+        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+      } else {
+        float* out = reinterpret_cast<float*>(a.o) + orow;
 #pragma unroll
-          for (int i = 0; i < 64; i += 4)
-            store4(out + i, make_float4(o[side][i], o[side][i + 1], o[side][i + 2], o[side][i + 3]));
-        } else {
-          float* out = reinterpret_cast<float*>(a.o) + orow;
-#pragma unroll
-          for (int i = 0; i < 64; i += 4)
-            store4(out + i, make_float4(o[side][i], o[side][i + 1], o[side][i + 2], o[side][i + 3]));
-        }
+        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
       }
     }
   }
