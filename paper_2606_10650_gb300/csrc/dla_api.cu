@@ -123,7 +123,9 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // (two buffers: in the concurrent schedule the next round's intra part overlaps this round's snapshot part)
   P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + 2 * BH * (size_t)R * P.interval * d * 4);
   // scan progress per (stream, CTA) and the count of started scan CTAs (concurrent read-out)
-  P.off_progress = off;  if (with_output) off = align256(off + (2 * BH + 1) * sizeof(int32_t));
+  // and the Gram pre-pass's per-block chunk counters (a pre-pass running beside the scan)
+  P.off_progress = off;
+  if (with_output) off = align256(off + (2 * BH + 1 + BH * dla::kMaxGramBlk) * sizeof(int32_t));
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
@@ -131,12 +133,12 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
 }
 
 // Interval counts of the rounds, in order.  Rounds of at most R intervals,
-// balanced; in persistent mode followed by a taper of R/2, R/4, R/8 intervals,
-// so that the read-out left to run after the last scan is short.
-std::vector<int> round_sizes(const FwdPlan& P) {
+// balanced; with `taper` followed by rounds of R/2, R/4, R/8 intervals, so that
+// the read-out left to run after the last scan launch is short.
+std::vector<int> round_sizes(const FwdPlan& P, bool taper) {
   std::vector<int> out, tail;
   int left = P.nsnap_total;
-  if (P.persistent)
+  if (taper)
     for (int s = P.R / 2; s >= 1 && s >= P.R / 8 && left - s >= P.R; s /= 2) {
       tail.push_back(s);
       left -= s;
@@ -172,6 +174,7 @@ bool concurrent_schedule() {
 }
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
+constexpr int kMinFreeSms = 8;    // SMs the scan must leave free for the concurrent schedule
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
 
 dla_status check_params(const dla_params* p) {
@@ -515,14 +518,26 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = stream_set(&S)) != cudaSuccess) return cuda_fail(e, "internal streams");
   if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
   if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
-  const std::vector<int> sizes = round_sizes(P);
+  int free_sms = 0;  // SMs the scan leaves to the rest when all its CTAs are resident (0: they are not)
   if (P.persistent && tc && concurrent_schedule()) {
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "device query");
+    const int BH = B * H;
+    if (dla::scan_mma_resident_streams(BH, d) >= BH) free_sms = sms - BH * dla::scan_mma_ctas_per_stream(BH, d);
+  }
+  if (free_sms >= kMinFreeSms) {
     // One scan over the whole sequence (high-priority stream) and the read-out
-    // in rounds beside it (low-priority stream): each read-out CTA waits for its
+    // in rounds beside it (low-priority streams): each read-out CTA waits for its
     // stream's progress, so rounds never wait for the slowest stream and the
-    // scan is launched once.  A one-CTA gate holds the read-out stream until
-    // every scan CTA has started, so a waiting read-out CTA never holds an SM
-    // the scan needs.
+    // scan is launched once.  A one-CTA gate holds the other streams until
+    // every scan CTA has started, so that nothing launched beside the scan
+    // takes an SM the scan needs.  Then the Gram pre-pass runs on the free SMs
+    // while the scan consumes it chunk by chunk (per-block counters), and the
+    // read-out follows the pre-pass (a waiting read-out CTA must not hold an SM
+    // the pre-pass needs).  Needs every scan CTA resident at once, with SMs to
+    // spare; otherwise the rounds schedule below runs.
+    const std::vector<int> sizes = round_sizes(P, false);
     {  // kernel code loaded once per device before anything of this path runs
       static bool loaded[kMaxDev] = {};
       static std::mutex mu;
@@ -537,33 +552,41 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     }
     int32_t* progress = (int32_t*)(ws + P.off_progress);
     int32_t* started = progress + 2 * B * H;
+    int32_t* gram_ready = started + 1;
     const int ctas = dla::scan_mma_ctas_per_stream(B * H, d);
-    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1) * sizeof(int32_t), S->hi)) != cudaSuccess)
+    dla::GramArgs ga;
+    ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.out = (float*)(ws + P.off_gram);
+    ga.chunk0 = 0; ga.count = P.gram_chunks;
+    ga.ready = gram_ready;
+    dla::gram_blocks(B * H, P.gram_chunks, 2 * free_sms, &ga.nblk, &ga.per_blk);
+    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
       return cuda_fail(e, "progress reset");
-    if (P.gram_chunks) {  // K0 over the whole sequence, on every SM
-      dla::GramArgs ga;
-      ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
-      ga.out = (float*)(ws + P.off_gram);
-      ga.chunk0 = 0; ga.count = P.gram_chunks;
-      e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
-      if (e != cudaSuccess) return cuda_fail(e, "gram launch");
-    }
-    if ((e = cudaEventRecord(S->gram_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
-    if ((e = cudaStreamWaitEvent(S->lo, S->gram_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
-    if ((e = dla::launch_gate(started, B * H * ctas, status, S->lo)) != cudaSuccess) return cuda_fail(e, "gate launch");
+    if ((e = cudaEventRecord(S->gate_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(S->lo, S->gate_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     sa.pool = ws + P.off_pool;
     sa.t_begin = 0; sa.t_end = T;
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
     sa.carry_in = 0; sa.snap_at_end = 0;
     sa.progress = progress; sa.started = started;
+    if (P.gram_chunks) {
+      sa.gram_ready = gram_ready;
+      sa.gram_nblk = ga.nblk;
+      sa.gram_per_blk = ga.per_blk;
+    }
     e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    if ((e = dla::launch_gate(started, B * H * ctas, status, S->lo)) != cudaSuccess) return cuda_fail(e, "gate launch");
+    if (P.gram_chunks) {  // K0 beside the scan, on the SMs it leaves free
+      e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
+      if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+    }
+    if ((e = cudaEventRecord(S->gram_done, S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     ra.pool = sa.pool;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
     // K2a of round r on lo2 into intra buffer r % 2, K2b of round r on lo after it;
     // K2a of round r + 2 reuses the buffer once K2b of round r is done
-    if ((e = cudaEventRecord(S->gate_done, S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
-    if ((e = cudaStreamWaitEvent(S->lo2, S->gate_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    if ((e = cudaStreamWaitEvent(S->lo2, S->gram_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     float* intra_buf[2] = {ra.ointra, ra.ointra + (size_t)B * H * ra.ointra_T * d};
     int snap0 = 0;
     for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
@@ -588,6 +611,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     if ((e = cudaStreamWaitEvent(st, S->ro_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     return ok();
   }
+  const std::vector<int> sizes = round_sizes(P, P.persistent != 0);
   bool gram_rest = false;  // the scan of round 1 waits for the Gram tables of rounds 1..
   if (P.gram_chunks) {
     // K0: Gram suffix tables.  Round 0's chunks run ahead of the first scan on
@@ -595,12 +619,18 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
     ga.out = (float*)(ws + P.off_gram);
+    ga.ready = nullptr;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "device query");
     const int first = std::min(P.gram_chunks, sizes[0] * P.interval / dla::kScanL);
     ga.chunk0 = 0; ga.count = first;
+    dla::gram_blocks(B * H, ga.count, 2 * sms, &ga.nblk, &ga.per_blk);
     e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     if (first < P.gram_chunks) {
       ga.chunk0 = first; ga.count = P.gram_chunks - first;
+      dla::gram_blocks(B * H, ga.count, 2 * sms, &ga.nblk, &ga.per_blk);
       if ((e = cudaStreamWaitEvent(S->lo, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");

@@ -80,7 +80,8 @@ __device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
   asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 // Read-out side: thread 0 waits until the scan CTAs of stream bh have completed
-// `need` intervals (progress[bh][0 .. ctas)), at most ~2 s (then status 5);
+// `need` intervals (progress[bh][0 .. ctas)), at most ~2 s (then status 5)
+// and not once the status word reports a failure;
 // the caller's CTA barrier then orders every later read after the wait.  Data
 // the scan writes must then be read past L1 (__ldcg): another CTA on the SM may
 // hold an older copy of the line.
@@ -89,6 +90,7 @@ __device__ __forceinline__ void wait_progress(const int32_t* progress, int ctas,
   const long long t0 = clock64();
   for (int r = 0; r < ctas; ++r)
     while (ld_acquire_gpu(progress + 2 * bh + r) < need) {
+      if (*(volatile int32_t*)status != 0) return;  // the call has failed already
       if (clock64() - t0 > 4000000000LL) {
         atomicExch(status, 5);
         return;

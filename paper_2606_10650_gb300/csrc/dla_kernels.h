@@ -59,6 +59,11 @@ struct ScanArgs {
   int32_t* pstate;       // [B*H] next free pool entry, then [B*H][C] pool ids of the live entries
   const float* gram;     // Gram pre-pass output [B*H][gram_chunks][kGramBlock], or nullptr
   int gram_chunks;       // 64-token chunks of the whole sequence
+  // Gram pre-pass running beside the scan (nullptr: it finished before the
+  // scan started): [B*H][gram_nblk] chunks written so far by the pre-pass CTA
+  // of each block of gram_per_blk consecutive chunks, which writes them in order
+  const int32_t* gram_ready;
+  int gram_nblk, gram_per_blk;
   int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
   int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)
@@ -69,14 +74,19 @@ struct ScanArgs {
 //   gs[j][t] = sum_{j <= s < t} G_ts       (beta_t of a segment opened at j, without S)
 //   Q[j][t]  = sum_{j <= u < t} gs[j][u]   (their running sum over the segment)
 //   a_t      = G_tt
+// One CTA per (stream, block of per_blk consecutive chunks of this launch)
+// walks its block in order, loading the next chunk while it computes this one.
 struct GramArgs {
   const void* k;
   const void* v;
   int B, T, H;
   int nchunks;           // chunks of the whole sequence
   int chunk0, count;     // this launch: chunks chunk0 .. chunk0 + count - 1
+  int nblk, per_blk;     // blocks of this launch and chunks per block (nblk * per_blk >= count)
   float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64)
+  int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after each), or nullptr
 };
+constexpr int kMaxGramBlk = 64;  // blocks per stream of one Gram launch, at most
 
 // K2: read-out of one round, one CTA per (snapshot interval, stream).
 struct ReadoutArgs {
@@ -134,6 +144,13 @@ cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream
 // CTAs per stream of launch_scan_mma: 2 (a CTA pair) when 2*B*H CTAs fit the
 // device's SMs in one wave with d = 128, else 1.
 int scan_mma_ctas_per_stream(int BH, int d);
+// Streams whose launch_scan_mma CTAs (pairs or single CTAs, as
+// scan_mma_ctas_per_stream picks for BH streams) can all be resident at once.
+int scan_mma_resident_streams(int BH, int d);
+// Block count of a Gram launch over `count` chunks of BH streams whose CTAs
+// fit `slots` resident CTAs (two per SM) in one wave (at least one block per
+// stream, at most kMaxGramBlk); per_blk follows.
+void gram_blocks(int BH, int count, int slots, int* nblk, int* per_blk);
 // One CTA that returns once `n` scan CTAs have started (*started >= n), or after
 // ~2 s with status 5: the read-out stream runs it before its first launch, so
 // that read-out CTAs waiting for the scan never hold the SMs the scan needs.

@@ -11,6 +11,9 @@
 //
 // Shapes per 64-token chunk: X is 64 x d x d, the Grams 2 x 64 x 64 x d and the
 // build d x d x 64, i.e. about 6 d^2 * 64 flop, a few thousand mma per CTA.
+#include <atomic>
+#include <mutex>
+
 #include "dla_common.cuh"
 #include "dla_mma.cuh"
 #include "dla_sm100.cuh"
@@ -59,17 +62,51 @@ __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1)
   return v & (lo | hi);
 }
 
+// Gram pre-pass running beside the scan: thread 0 of the scan CTA waits until
+// the pre-pass CTA of chunk gc's block has published the chunk (its counter
+// counts the block's chunks written, in order), remembering the last count.
+struct GramFeed {
+  const int32_t* ready;  // this stream's [nblk] counters, or nullptr (the pre-pass has finished)
+  int per;               // chunks per block
+  int blk, cnt;          // last counter value read, and its block
+};
+__device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int* abort, int32_t* status) {
+  if (!f.ready) return true;
+  const int blk = gc / f.per, need = gc - blk * f.per + 1;
+  if (blk != f.blk || f.cnt < need) {
+    const long long t0 = clock64();
+    while (true) {
+      const int c = ld_acquire_gpu(f.ready + blk);
+      if (c >= need) {
+        f.blk = blk;
+        f.cnt = c;
+        break;
+      }
+      if (*abort) return false;
+      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::kWaitCycles) {
+        *abort = 1;
+        atomicCAS(status, 0, sm100::kStatusTimeout);
+        return false;
+      }
+    }
+  }
+  asm volatile("fence.proxy.async.global;" ::: "memory");  // the block is read by a bulk copy
+  return true;
+}
+
 // Next chunk's k and v rows (cp.async by every thread, zero-filled past the
-// sequence end) and its Gram block (one bulk copy by thread 0, completing on
-// `bar`).  The k, v copies are waited for with cp.async.wait_group, the Gram
+// sequence end) and its Gram block gc (one bulk copy by thread 0, completing
+// on `bar`, skipped after a failed wait for the pre-pass, which sets the abort
+// flag).  The k, v copies are waited for with cp.async.wait_group, the Gram
 // block with the mbarrier.
 template <int D>
 __device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
                                                const __nv_bfloat16* vs, int row_stride, int valid, float* dgq,
-                                               const float* gsrc, uint64_t* bar) {
+                                               const float* gsrc, uint64_t* bar, GramFeed& feed, int gc,
+                                               volatile int* abort, int32_t* status) {
   constexpr int RP = D + 8;
   constexpr int V16 = D / 8;
-  if (threadIdx.x == 0 && gsrc) {
+  if (threadIdx.x == 0 && gsrc && gram_feed_wait(feed, gc, abort, status)) {
     sm100::mbar_expect_tx(bar, (uint32_t)kGramBlock * 4u);
     sm100::bulk_g2s(dgq, gsrc, (uint32_t)kGramBlock * 4u, bar);
   }
@@ -163,6 +200,63 @@ __device__ __forceinline__ void prefix_rows(const float* src, int rs, int cs, fl
     if (lane == 0) ex = 0.f;
     dst[j * ds + 2 * lane] = ex;
     dst[j * ds + 2 * lane + 1] = ex + g0;
+  }
+}
+
+// suffix_rows / prefix_rows with the warp's L / NW rows scanned together (as
+// many independent shuffle chains; the same sums in the same order per row), for
+// the Gram pre-pass, which has the registers to spare.
+__device__ __forceinline__ void suffix_rows_ilp(float* G) {
+  constexpr int R = L / NW;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float g0[R], g1[R], r[R];
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const float* row = G + (warp + i * NW) * (L + 1);
+    g0[i] = row[2 * lane];
+    g1[i] = row[2 * lane + 1];
+    r[i] = g0[i] + g1[i];
+  }
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1)
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+      const float dn = __shfl_down_sync(0xffffffffu, r[i], o);
+      if (lane + o < 32) r[i] += dn;
+    }
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const float after = __shfl_down_sync(0xffffffffu, r[i], 1);
+    const float tail = (lane < 31) ? after : 0.f;
+    float* row = G + (warp + i * NW) * (L + 1);
+    row[2 * lane + 1] = g1[i] + tail;
+    row[2 * lane] = g0[i] + g1[i] + tail;
+  }
+}
+__device__ __forceinline__ void prefix_rows_ilp(const float* src, int rs, int cs, float* dst, int ds) {
+  constexpr int R = L / NW;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float g0[R], inc[R];
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    const int j = warp + i * NW;
+    g0[i] = src[j * rs + (2 * lane) * cs];
+    inc[i] = g0[i] + src[j * rs + (2 * lane + 1) * cs];
+  }
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1)
+#pragma unroll
+    for (int i = 0; i < R; ++i) {
+      const float up = __shfl_up_sync(0xffffffffu, inc[i], o);
+      if (lane >= o) inc[i] += up;
+    }
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    float ex = __shfl_up_sync(0xffffffffu, inc[i], 1);
+    if (lane == 0) ex = 0.f;
+    const int j = warp + i * NW;
+    dst[j * ds + 2 * lane] = ex;
+    dst[j * ds + 2 * lane + 1] = ex + g0[i];
   }
 }
 
@@ -491,9 +585,15 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const int ntok = a.t_end - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
   const long long gchunk0 = (long long)bh * a.gram_chunks + a.t_begin / L;  // Gram block of the round's first chunk
+  GramFeed feed;
+  feed.ready = a.gram_ready ? a.gram_ready + (long long)bh * a.gram_nblk : nullptr;
+  feed.per = a.gram_per_blk;
+  feed.blk = -1;
+  feed.cnt = 0;
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
-                      a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0]);
+                      a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
+                      &sm.abort_flag, a.status);
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
     const int Lc = min(L, a.t_end - t0);
@@ -503,7 +603,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const int t1 = t0 + L;
       prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
                         vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
-                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1]);
+                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
+                        a.t_begin / L + c + 1, &sm.abort_flag, a.status);
       asm volatile("cp.async.wait_group 1;" ::: "memory");
     } else {
       asm volatile("cp.async.wait_group 0;" ::: "memory");
@@ -925,52 +1026,80 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 template <int D>
 struct GramSmem {
   static constexpr int RP = D + 8;
-  __nv_bfloat16 k[L * RP];
-  __nv_bfloat16 v[L * RP];
-  float G[L * (L + 1)];
-  float Q[L * (L + 1)];
+  __nv_bfloat16 k[2][L * RP];  // [stage] the chunk's k rows
+  __nv_bfloat16 v[2][L * RP];
+  float G[L * (L + 1)];        // G[t][s], then in place gs[s][t]
+  float Q[L * (L + 1)];        // Q[j][t]
   float a[L];
 };
 
+// K0: each CTA walks the chunks of one block of one stream in order; the k, v
+// rows of the next chunk are in flight (cp.async) while it computes this one.
+// With `ready` set, the chunk count of the block is published (release) after
+// each chunk's writes, for a scan that runs concurrently and reads the block
+// through the async proxy.
 template <int D>
 __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   constexpr int RP = D + 8;
+  constexpr int V16 = D / 8;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   GramSmem<D>& sm = *reinterpret_cast<GramSmem<D>*>(smem_raw);
-  const int c = a.chunk0 + blockIdx.x, bh = blockIdx.y;
+  const int bh = blockIdx.x, blk = blockIdx.y;
   const int b = bh / a.H, h = bh % a.H;
-  const int t0 = c * L;
-  const int valid = min(L, a.T - t0);
+  const int c_begin = a.chunk0 + blk * a.per_blk;
+  const int c_end = min(a.chunk0 + a.count, c_begin + a.per_blk);
+  if (c_begin >= c_end) return;
   const int row_stride = a.H * D;
-  const __nv_bfloat16* ks =
-      reinterpret_cast<const __nv_bfloat16*>(a.k) + (((long long)b * a.T + t0) * a.H + h) * D;
-  const __nv_bfloat16* vs =
-      reinterpret_cast<const __nv_bfloat16*>(a.v) + (((long long)b * a.T + t0) * a.H + h) * D;
-  constexpr int V16 = D / 8;
-  for (int e = threadIdx.x; e < L * V16; e += NT) {
-    const int r = e / V16, cc = (e % V16) * 8;
-    uint4 kv = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-    if (r < valid) {
-      kv = *reinterpret_cast<const uint4*>(ks + (long long)r * row_stride + cc);
-      vv = *reinterpret_cast<const uint4*>(vs + (long long)r * row_stride + cc);
+  const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
+  const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
+  auto load = [&](int c, int st) {  // rows past the sequence end are zero-filled
+    const int t0 = c * L, valid = min(L, a.T - t0);
+    for (int e = threadIdx.x; e < L * V16; e += NT) {
+      const int r = e / V16, cc = (e % V16) * 8;
+      const long long off = (long long)(t0 + (r < valid ? r : 0)) * row_stride + cc;
+      const int nbytes = (r < valid) ? 16 : 0;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.k[st] + r * RP + cc)),
+                   "l"(k0 + off), "r"(nbytes) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.v[st] + r * RP + cc)),
+                   "l"(v0 + off), "r"(nbytes) : "memory");
     }
-    *reinterpret_cast<uint4*>(sm.k + r * RP + cc) = kv;
-    *reinterpret_cast<uint4*>(sm.v + r * RP + cc) = vv;
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  load(c_begin, 0);
+  for (int c = c_begin; c < c_end; ++c) {
+    const int st = (c - c_begin) & 1;
+    if (c + 1 < c_end) {
+      load(c + 1, st ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();
+    gram_tile<D>(sm.k[st], sm.v[st], sm.G, sm.a);
+    __syncthreads();
+    suffix_rows_ilp(sm.G);  // G[t][j] = gs[j][t]
+    __syncthreads();
+    prefix_rows_ilp(sm.G, 1, L + 1, sm.Q, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u]
+    __syncthreads();
+    // out: gs[j][t], Q[j][t] (four consecutive t per thread), a[t]
+    float* out = a.out + ((long long)bh * a.nchunks + c) * kGramBlock;
+    for (int e = threadIdx.x; e < L * L / 4; e += NT) {
+      const int j = e / (L / 4), t = (e % (L / 4)) * 4;
+      const float4 g4 = make_float4(sm.G[t * (L + 1) + j], sm.G[(t + 1) * (L + 1) + j], sm.G[(t + 2) * (L + 1) + j],
+                                    sm.G[(t + 3) * (L + 1) + j]);
+      const float* qr = sm.Q + j * (L + 1) + t;
+      *reinterpret_cast<float4*>(out + j * L + t) = g4;
+      *reinterpret_cast<float4*>(out + L * L + j * L + t) = make_float4(qr[0], qr[1], qr[2], qr[3]);
+    }
+    if (threadIdx.x < L / 4)
+      *reinterpret_cast<float4*>(out + 2 * L * L + 4 * threadIdx.x) = *reinterpret_cast<const float4*>(sm.a + 4 * threadIdx.x);
+    if (a.ready) asm volatile("fence.proxy.async.global;" ::: "memory");  // the scan reads the block by bulk copy
+    __syncthreads();  // the block is written; G, Q, a are reused by the next chunk
+    if (a.ready && threadIdx.x == 0) {
+      __threadfence();
+      st_release_gpu(a.ready + (long long)bh * a.nblk + blk, c - c_begin + 1);
+    }
   }
-  __syncthreads();
-  gram_tile<D>(sm.k, sm.v, sm.G, sm.a);
-  __syncthreads();
-  suffix_rows(sm.G);  // G[t][j] = gs[j][t]
-  __syncthreads();
-  prefix_rows(sm.G, 1, L + 1, sm.Q, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u]
-  __syncthreads();
-  float* out = a.out + ((long long)bh * a.nchunks + c) * kGramBlock;
-  for (int e = threadIdx.x; e < L * L; e += NT) {
-    const int t = e % L, j = e / L;
-    out[j * L + t] = sm.G[t * (L + 1) + j];
-    out[L * L + j * L + t] = sm.Q[j * (L + 1) + t];
-  }
-  if (threadIdx.x < L) out[2 * L * L + threadIdx.x] = sm.a[threadIdx.x];
 }
 
 template <int D>
@@ -979,9 +1108,19 @@ static cudaError_t launch_gram_t(const GramArgs& a, cudaStream_t s) {
   auto kern = gram_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid(a.count, a.B * a.H);
+  if (a.nblk < 1 || a.nblk > kMaxGramBlk || (long long)a.nblk * a.per_blk < a.count) return cudaErrorInvalidValue;
+  dim3 grid(a.B * a.H, a.nblk);  // streams fastest: every stream's first block is scheduled first
   kern<<<grid, NT, smem, s>>>(a);
   return cudaGetLastError();
+}
+
+void gram_blocks(int BH, int count, int slots, int* nblk, int* per_blk) {
+  int n = slots / BH;  // one wave
+  if (n > kMaxGramBlk) n = kMaxGramBlk;
+  if (n > count) n = count;
+  if (n < 1) n = 1;
+  *per_blk = (count + n - 1) / n;
+  *nblk = (count + *per_blk - 1) / *per_blk;
 }
 
 cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s) {
@@ -1019,11 +1158,72 @@ int scan_mma_ctas_per_stream(int BH, int d) {
 // CTA pairs when two CTAs per stream still fit on the device in one wave.
 static bool use_pairs(const ScanArgs& a) { return scan_mma_ctas_per_stream(a.B * a.H, 128) == 2; }
 
+static int resident_streams_query(int BH, int d) {
+  int dev = 0, sms = 0, per_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 0;
+  if (scan_mma_ctas_per_stream(BH, d) == 2) {
+    auto kern = scan_mma_kernel<128, __nv_bfloat16, 2>;
+    const size_t smem = sizeof(MmaSmem<128, 2>);
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * BH);
+    cfg.blockDim = dim3(NT);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess) return 0;
+    return clusters;
+  }
+  if (d == 128) {
+    auto kern = scan_mma_kernel<128, __nv_bfloat16, 1>;
+    const size_t smem = sizeof(MmaSmem<128, 1>);
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, smem) != cudaSuccess)
+      return 0;
+  } else {
+    auto kern = scan_mma_kernel<64, __nv_bfloat16, 1>;
+    const size_t smem = sizeof(MmaSmem<64, 1>);
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, smem) != cudaSuccess)
+      return 0;
+  }
+  return per_sm * sms;
+}
+int scan_mma_resident_streams(int BH, int d) {  // cached per device and kernel variant
+  static std::atomic<int> cache[64][3];
+  static std::atomic<bool> init{false};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  const int var = (d != 128) ? 2 : scan_mma_ctas_per_stream(BH, d) - 1;
+  if (!init.load()) {
+    std::lock_guard<std::mutex> g(mu);
+    if (!init.load()) {
+      for (auto& row : cache)
+        for (auto& c : row) c.store(-1);
+      init.store(true);
+    }
+  }
+  int v = cache[dev][var].load();
+  if (v < 0) {
+    v = resident_streams_query(BH, d);
+    cache[dev][var].store(v);
+  }
+  return v;
+}
+
 __global__ void gate_kernel(const int32_t* started, int n, int32_t* status) {
   const long long t0 = clock64();
   while (ld_acquire_gpu(started) < n)
-    if (clock64() - t0 > 4000000000LL) {  // ~2 s
-      atomicExch(status, 5);
+    if (*(volatile int32_t*)status != 0 || clock64() - t0 > 4000000000LL) {  // ~2 s
+      atomicCAS(status, 0, 5);  // a failure reported elsewhere keeps its code
       return;
     }
 }

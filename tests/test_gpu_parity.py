@@ -37,6 +37,9 @@ CASES = {
     "d128_fp32": ("tiny", dict(B=1, H=2, T=300, d=128, C=6, tau=1.4142)),
     # more streams than CTA pairs fit on the device: one scan CTA per stream
     "many_streams_bf16": ("regime", dict(B=3, H=27, T=300, C=3, tau=1.2)),
+    # more streams than SMs: the scan cannot keep every stream resident, so the
+    # forward pass takes the per-round schedule whatever DLA_SCHEDULE says
+    "streams_beyond_sms_bf16": ("regime", dict(B=4, H=40, T=200, C=3, tau=1.2)),
 }
 
 
