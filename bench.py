@@ -206,19 +206,17 @@ def bench_prefill(args, dist, pk):
     flops_total = 2.0 * d * d * (sum_m + 2 * T * BH)
     kt_tab = kernel_table(timing, args.steps)
     tc_path = (w.dtype == "bf16" and d == 128)
-    # the read-out is K2b (snapshot part) plus, on the tensor-core path, K2a (intra-interval part)
     ro_n, ro_ms = timing["readout"]
-    ri_n, ri_ms = timing.get("readout_intra", (0, 0.0))
     sc_n, sc_ms = timing["scan"]
     fp32_peak = pk_fp32(pk)
     rooflines, kernel_ms = {}, {}
     if ro_n:
-        ms_ro = ro_ms + ri_ms
+        ms_ro = ro_ms
         kernel_ms["readout"] = ms_ro
         ach = flops_readout * args.steps / (ms_ro * 1e-3) / 1e12  # flops_readout is per step
         peak = pk["bf16"] if tc_path else fp32_peak
         rooflines["readout"] = {
-            "kernel": "readout (K2a intra-interval + K2b snapshots)" if tc_path else "readout",
+            "kernel": "readout (snapshot and intra-interval parts)" if tc_path else "readout",
             "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
             "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
             "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else

@@ -141,11 +141,14 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
  *   Schedule (bf16, d = 128, workspace of at least dla_forward_workspace(...)):
  *   the environment variable DLA_SCHEDULE, read at every call, selects
  *   "concurrent" (default: the scan runs once over the whole sequence while
- *   the read-out follows it on other streams, waiting for each stream's
- *   progress; a kernel of the read-out side waits up to ~2 s for the scan to
- *   become resident, so the device should not be saturated by other work at
- *   that moment) or "rounds" (the scan and the read-out alternate round by
- *   round on two internal streams).  Both give the same results. */
+ *   the Gram pre-pass and then the read-out run beside it on another stream,
+ *   each waiting for the other side's progress; a kernel of the read-out side
+ *   waits up to ~2 s for the scan to become resident, so the device should not
+ *   be saturated by other work at that moment) or "rounds" (the scan and the
+ *   read-out alternate round by round on two internal streams).  The
+ *   concurrent schedule needs every scan CTA resident at once with SMs to
+ *   spare; calls with more streams than that take the rounds schedule.  Both
+ *   give the same results. */
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
@@ -184,16 +187,14 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
                            void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
 
 /* Instrumentation (no counterpart in the paper).  Kernel kinds of the
- * library: K1 scan, K2 read-out (for bf16, d = 128: its snapshot part K2b),
- * K3 decode, cache init, K0 Gram pre-pass, K2a intra-interval read-out part. */
+ * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass. */
 typedef enum {
   DLA_K_SCAN = 0,
   DLA_K_READOUT = 1,
   DLA_K_DECODE = 2,
   DLA_K_INIT = 3,
   DLA_K_GRAM = 4,
-  DLA_K_READOUT_INTRA = 5,
-  DLA_K_COUNT = 6
+  DLA_K_COUNT = 5
 } dla_kernel_kind;
 
 /* enable = 1: from now on, every kernel this host thread launches through the

@@ -75,7 +75,7 @@ struct FwdPlan {
   int persistent;
   int nbuf;          // pools (1 persistent, 2 reset with several rounds)
   int pool_cap;      // pool entries per stream, per pool
-  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram, off_ointra,
+  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram,
       off_progress, off_pool, pool_bytes;
   int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
   size_t total;
@@ -119,9 +119,6 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramBlock floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
-  // intra-interval read-out part of one round (tensor-core read-out), fp32
-  // (two buffers: in the concurrent schedule the next round's intra part overlaps this round's snapshot part)
-  P.off_ointra = off;    if (with_output && use_tc(in_dtype, d)) off = align256(off + 2 * BH * (size_t)R * P.interval * d * 4);
   // scan progress per (stream, CTA) and the count of started scan CTAs (concurrent read-out)
   // and the Gram pre-pass's per-block chunk counters (a pre-pass running beside the scan)
   P.off_progress = off;
@@ -213,9 +210,9 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
 // thread and device: the scan runs on a high-priority stream, the read-out on
 // a low-priority one, so the scan's few CTAs get SMs first.
 struct StreamSet {
-  cudaStream_t hi = nullptr, lo = nullptr, lo2 = nullptr;  // scan, snapshot read-out, intra read-out
+  cudaStream_t hi = nullptr, lo = nullptr;  // scan, read-out
   cudaEvent_t in = nullptr, gram_done = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
-  cudaEvent_t gate_done = nullptr, intra_done[2] = {nullptr, nullptr}, tc_done[2] = {nullptr, nullptr};
+  cudaEvent_t prep_done = nullptr;
   bool ready = false;
 };
 constexpr int kMaxDev = 64;
@@ -234,12 +231,7 @@ cudaError_t stream_set(StreamSet** out) {
     if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.gram_done, cudaEventDisableTiming)) != cudaSuccess) return e;
-    if ((e = cudaStreamCreateWithPriority(&S.lo2, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
-    if ((e = cudaEventCreateWithFlags(&S.gate_done, cudaEventDisableTiming)) != cudaSuccess) return e;
-    for (int i = 0; i < 2; ++i) {
-      if ((e = cudaEventCreateWithFlags(&S.intra_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
-      if ((e = cudaEventCreateWithFlags(&S.tc_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
-    }
+    if ((e = cudaEventCreateWithFlags(&S.prep_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     for (int i = 0; i < 2; ++i) {
       if ((e = cudaEventCreateWithFlags(&S.scan_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
       if ((e = cudaEventCreateWithFlags(&S.ro_done[i], cudaEventDisableTiming)) != cudaSuccess) return e;
@@ -508,8 +500,6 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   sa.pstate = P.persistent ? (int32_t*)(ws + P.off_pstate) : nullptr;
   sa.gram = P.gram_chunks ? (const float*)(ws + P.off_gram) : nullptr;
   sa.gram_chunks = P.gram_chunks;
-  ra.ointra = tc ? (float*)(ws + P.off_ointra) : nullptr;
-  ra.ointra_T = P.R * P.interval;
   // Round r: the scan (high-priority stream) appends to the pool, then the
   // read-out of round r (low-priority stream) runs while the scan of round
   // r + 1 proceeds.  In reset mode pool b is reused by round r + 2 only after
@@ -562,8 +552,8 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     dla::gram_blocks(B * H, P.gram_chunks, 2 * free_sms, &ga.nblk, &ga.per_blk);
     if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
       return cuda_fail(e, "progress reset");
-    if ((e = cudaEventRecord(S->gate_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
-    if ((e = cudaStreamWaitEvent(S->lo, S->gate_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    if ((e = cudaEventRecord(S->prep_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(S->lo, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     sa.pool = ws + P.off_pool;
     sa.t_begin = 0; sa.t_end = T;
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
@@ -581,30 +571,17 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     }
-    if ((e = cudaEventRecord(S->gram_done, S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     ra.pool = sa.pool;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
-    // K2a of round r on lo2 into intra buffer r % 2, K2b of round r on lo after it;
-    // K2a of round r + 2 reuses the buffer once K2b of round r is done
-    if ((e = cudaStreamWaitEvent(S->lo2, S->gram_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
-    float* intra_buf[2] = {ra.ointra, ra.ointra + (size_t)B * H * ra.ointra_T * d};
+    // the read-out rounds follow the pre-pass on the read-out stream
     int snap0 = 0;
     for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
       ra.t_begin = snap0 * P.interval;
       ra.t_end = std::min(T, ra.t_begin + sizes[r] * P.interval);
       ra.nsnap = sizes[r]; ra.snap_base = snap0;
-      ra.ointra = intra_buf[r & 1];
-      if (r >= 2 && (e = cudaStreamWaitEvent(S->lo2, S->tc_done[r & 1], 0)) != cudaSuccess)
-        return cuda_fail(e, "stream wait");
-      e = timed(DLA_K_READOUT_INTRA, S->lo2, [&] { return dla::launch_readout_intra(ra, S->lo2); });
-      if (e != cudaSuccess) return cuda_fail(e, "intra read-out launch");
-      if ((e = cudaEventRecord(S->intra_done[r & 1], S->lo2)) != cudaSuccess) return cuda_fail(e, "event record");
-      if ((e = cudaStreamWaitEvent(S->lo, S->intra_done[r & 1], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "readout launch");
-      if ((e = cudaEventRecord(S->tc_done[r & 1], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     }
-    ra.ointra = intra_buf[0];
     if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaEventRecord(S->ro_done[0], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
@@ -662,10 +639,6 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     if ((e = cudaEventRecord(S->scan_done[r % 2], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(S->lo, S->scan_done[r % 2], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
-    if (tc) {  // K2a, then K2b on the same stream (K2b starts from K2a's output)
-      e = timed(DLA_K_READOUT_INTRA, S->lo, [&] { return dla::launch_readout_intra(ra, S->lo); });
-      if (e != cudaSuccess) return cuda_fail(e, "intra read-out launch");
-    }
     e = timed(DLA_K_READOUT, S->lo, [&] {
       return tc ? dla::launch_readout_tc(ra, status, S->lo)
                 : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, S->lo);

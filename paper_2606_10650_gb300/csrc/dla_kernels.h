@@ -108,8 +108,6 @@ struct ReadoutArgs {
   int snap_base;         // global index of this round's first interval
   int nsnap;
   int interval;          // tokens per snapshot interval
-  float* ointra;         // [B*H][ointra_T][d] fp32 intra-interval part (tensor-core path), token t - t_begin
-  int ointra_T;          // tokens per stream in ointra (one round)
   const int32_t* progress;  // [B*H][2] scan progress to wait for (the scan runs concurrently), or nullptr
   int progress_ctas;        // scan CTAs per stream (1 or 2): entries of progress[bh] that count
   int32_t* status;          // device status word
@@ -166,11 +164,9 @@ cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s);
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;
-// K2 for bf16 inputs, d = 128, 128-token intervals, in two launches:
-// K2a (mma.sync) writes the intra-interval part to a.ointra; K2b (tcgen05 /
-// TMEM / TMA, snapshots stored as bf16 hi + lo) adds the snapshot part and
-// writes o.
-cudaError_t launch_readout_intra(const ReadoutArgs& a, cudaStream_t s);
+// K2 for bf16 inputs, d = 128, 128-token intervals (tcgen05 / TMEM / TMA,
+// snapshots stored as bf16 hi + lo): one CTA per pair of intervals computes the
+// snapshot part and the intra-interval part and writes o.
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t s);
 constexpr int kReadoutTcInterval = 128;
 cudaError_t launch_decode(const DecodeArgs& a, int d, bool in_bf16, cudaStream_t s);

@@ -1,12 +1,14 @@
-// dla_readout_tc.cu -- K2b on the 5th-generation tensor cores (tcgen05 + TMEM
-// + TMA): the snapshot part of the read-out of Eq. (capacity_bounded_output)
-//   o_t = o_intra[t] + sum_{x < m0} lambda_{t, L_t(x)} (S_x q_t)
-// for bf16 inputs, d = 128.  o_intra (the interval's own tokens, fp32) comes
-// from K2a.  The cache seen by token t is the snapshot taken by K1 at the start
-// of t's 128-token interval (m0 states, logical order) regrouped by the merges
-// decided inside the interval: merges only add states, so snapshot entry x
-// contributes with the lambda of its logical slot L_t(x) after the interval's
-// events up to t.
+// dla_readout_tc.cu -- K2, the read-out of Eq. (capacity_bounded_output), on
+// the 5th-generation tensor cores (tcgen05 + TMEM + TMA) for bf16 inputs,
+// d = 128:
+//   o_t = sum_{x < m0} lambda_{t, L_t(x)} (S_x q_t)                  snapshot part
+//       + sum_{s <= t in interval} lambda_{t, L_t(e(s))} (q_t . k_s) v_s   intra part
+// The cache seen by token t is the snapshot taken by K1 at the start of t's
+// 128-token interval (m0 states, logical order) regrouped by the merges decided
+// inside the interval: merges only add states, so snapshot entry x contributes
+// with the lambda of its logical slot L_t(x) after the interval's events up to
+// t.  The tokens of the interval itself belong to the entry opened by the last
+// boundary event at or before them (event 0: the snapshot's open entry).
 //
 // One CTA per (pair of consecutive intervals A, B, stream).  Consecutive
 // snapshot lists share most of their states (only entries that changed get new
@@ -15,13 +17,17 @@
 // D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128), with
 // S_x = S_hi + S_lo, the fp32 snapshot split into bf16 parts by K1 (two MMAs
 // per state and interval keep the state rounding near 2^-17 instead of 2^-9).
-// An interval's MMAs are skipped for a state that is not in its list.
+// An interval's MMAs are skipped for a state that is not in its list.  After
+// the last state, the intra part of each interval: P = Q K^T, Pt = P o W
+// (W_ts = lambda_{t, L_t(e(s))} for s <= t, else 0) written as bf16 over the Q
+// tile, V^T written into the stages the last state used, O = Pt V, added to o.
 // Roles: warp 0 issues TMA loads (the two Q tiles, then the hi and lo parts of
-// each union state into four 32 KB half-stages), warp 1 issues tcgen05.mma (one
-// thread) into two TMEM buffers of two 128-column accumulators (A, B), warps
-// 2..17 read TMEM, weight by lambda and accumulate o in registers (one token
-// row, one interval and one 64-column half per thread; warp w reads TMEM lane
-// quadrant w % 4).
+// each union state into four 32 KB stages, then the two K tiles), warp 1
+// issues tcgen05.mma (one thread) into two TMEM buffers of two 128-column
+// accumulators (A, B), warps 2..17 read TMEM, weight by lambda and accumulate o
+// in registers (one token row, one interval and one 64-column half per thread;
+// warp w reads TMEM lane quadrant w % 4).  All waits are bounded (~2 s, then
+// an abort flag and status 5).
 #include "dla_common.cuh"
 #include "dla_sm100.cuh"
 #include "dla_tmap.h"
@@ -36,40 +42,47 @@ constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
 constexpr int NT = 576;   // 18 warps
 constexpr int NEPI = 16;  // epilogue warps
-constexpr int NHS = 4;   // shared-memory half-stages
+constexpr int NHS = 4;   // shared-memory stages (32 KB: one hi or lo state part, or one K tile)
 constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
 constexpr int MAXU = 2 * kMaxC;  // union of two lists
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTile = L * 128;  // one K-major 128B-swizzled tile: 128 rows x 64 bf16
+constexpr int kRows = L + 1;         // events 0 .. L of an interval
+// Slot tables of one interval, in one region: first the snapshot entries' slots
+// tab[e][x] (row stride kMaxC), later the intra part's tab[e][i] for the entry
+// opened at event i <= e (row e at e (e + 1) / 2).
+constexpr int kSnapTab = kRows * kMaxC;
+constexpr int kIntraTab = kRows * (kRows + 1) / 2;
+constexpr int kTabBytes = kSnapTab > kIntraTab ? kSnapTab : kIntraTab;
 
-struct Side {                          // per interval of the pair
-  unsigned char tab[(L + 1) * kMaxC];  // L(x) of snapshot entry x after event e
-  int evt[L];                          // events (boundaries) at or before token t
-  int mlog[L];                         // merge indices
-  uint8_t bnd[L];                      // boundary flags
+struct Side {      // per interval of the pair
+  int evt[L];      // events (boundaries) at or before token t
+  int mlog[L];     // merge indices
+  uint8_t bnd[L];  // boundary flags
 };
 
 struct TcSmem {
-  uint8_t Q[2][2][kTile];      // [interval][k-half], A operands        64 KB
-  uint8_t hs[NHS][2][kTile];   // [half-stage][k-half]                 128 KB
+  uint8_t Q[2][2][kTile];      // [interval][k-half]: Q (A operand), then Pt           64 KB
+  uint8_t hs[NHS][2][kTile];   // [stage][k-half]: state parts, then K and V^T         128 KB
+  unsigned char tab[2][kTabBytes];
   Side side[2];
   int ids[2][kMaxC];           // pool ids of the two lists
   int uid[MAXU];               // union: pool id
   int uxa[MAXU], uxb[MAXU];    // union: index in list A / list B, or -1
-  int logi[kMaxC];
+  int logi[2][kRows];          // table-build scratch, per interval
   int nu;                      // union size
-  uint64_t bar_q, bar_done;
+  uint64_t bar_q, bar_pt, bar_done;
   uint64_t full[NHS], empty[NHS], acc_full[NBUF], acc_empty[NBUF];
   uint32_t tmem_base;
   int abort_flag;
 };
 
-// Slot table of one interval (one warp): row e holds L(x) of snapshot entry x
-// after the interval's first e boundary events.
-__device__ __forceinline__ void build_table(Side& sd, int* logi, int m0, int lane) {
+// Snapshot entries' slot table of one interval (one warp): row e holds L(x) of
+// snapshot entry x after the interval's first e boundary events.
+__device__ __forceinline__ void build_snap_table(const Side& sd, unsigned char* tab, int* logi, int m0, int lane) {
   for (int x = lane; x < m0; x += 32) {
     logi[x] = x;
-    sd.tab[x] = (unsigned char)x;
+    tab[x] = (unsigned char)x;
   }
   __syncwarp();
   unsigned long long lo64 = 0, hi64 = 0;
@@ -88,7 +101,41 @@ __device__ __forceinline__ void build_table(Side& sd, int* logi, int m0, int lan
     for (int x = lane; x < m0; x += 32) {
       int li = logi[x];
       if (j >= 0 && li > j) logi[x] = --li;
-      sd.tab[ev * kMaxC + x] = (unsigned char)li;
+      tab[ev * kMaxC + x] = (unsigned char)li;
+    }
+  }
+}
+
+// Intra part's slot table of one interval (one warp): row e (at e (e + 1) / 2)
+// holds the slot, after event e, of the entry opened at event i <= e (event 0:
+// the snapshot's open entry, slot m0 - 1).  Lane x owns the entries opened at
+// events x, x + 32, ...; a merge at index j moves every slot above j down by one.
+__device__ __forceinline__ void build_intra_table(const Side& sd, unsigned char* tab, int* logi, int m0, int lane) {
+  if (lane == 0) {
+    logi[0] = m0 - 1;  // unused when m0 = 0 (the interval then opens with a boundary)
+    tab[0] = (unsigned char)(m0 - 1);
+  }
+  unsigned long long lo64 = 0, hi64 = 0;
+#pragma unroll
+  for (int w4 = 0; w4 < 4; ++w4) {
+    const unsigned m = __ballot_sync(0xffffffffu, sd.bnd[32 * w4 + lane] != 0);
+    if (w4 < 2) lo64 |= (unsigned long long)m << (32 * w4);
+    else hi64 |= (unsigned long long)m << (32 * (w4 - 2));
+  }
+  int cnt = m0, ev = 0;
+  while (lo64 | hi64) {
+    const int tt = lo64 ? (__ffsll((long long)lo64) - 1) : (64 + __ffsll((long long)hi64) - 1);
+    if (lo64) lo64 &= lo64 - 1; else hi64 &= hi64 - 1;
+    const int j = sd.mlog[tt];
+    if (j >= 0) cnt -= 1;
+    ev += 1;
+    if ((ev & 31) == lane) logi[ev] = cnt;
+    cnt += 1;
+    unsigned char* row = tab + ev * (ev + 1) / 2;
+    for (int i = lane; i <= ev; i += 32) {
+      int li = logi[i];
+      if (j >= 0 && i < ev && li > j) logi[i] = --li;
+      row[i] = (unsigned char)li;
     }
   }
 }
@@ -107,9 +154,10 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
 
 }  // namespace
 
+// 18 warps: the sub-partitions holding five of them bound a thread to 96 registers
 __global__ void __launch_bounds__(NT, 1)
-    readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmS,
-                      int32_t* status) {
+    readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                      const __grid_constant__ CUtensorMap tmS, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -133,6 +181,7 @@ __global__ void __launch_bounds__(NT, 1)
 
   if (tid == 0) {
     mbar_init(&sm.bar_q, 1);
+    mbar_init(&sm.bar_pt, NEPI);
     mbar_init(&sm.bar_done, 1);
     for (int i = 0; i < NHS; ++i) {
       mbar_init(&sm.full[i], 1);
@@ -146,6 +195,7 @@ __global__ void __launch_bounds__(NT, 1)
     fence_mbar_init();
     // the Q tiles go out first; they depend on nothing
     prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
     prefetch_tmap(&tmS);
     mbar_expect_tx(&sm.bar_q, (hasB ? 4 : 2) * kTile);
     tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, c0A, b);
@@ -200,19 +250,30 @@ __global__ void __launch_bounds__(NT, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   const int nu = sm.nu;
+  // ring units: u < 2 nu are the hi / lo parts of union state u >> 1; units
+  // 2 nu and 2 nu + 1 the K tiles of intervals A and B.  Unit u uses stage
+  // u % NHS for the (u / NHS)-th time.
+  const int uK = 2 * nu;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int issued[NHS];  // uses of each half-stage so far
+      int issued[NHS];  // uses of each stage so far
       for (int i = 0; i < NHS; ++i) issued[i] = 0;
-      for (int u = 0; u < 2 * nu; ++u) {  // unit u: part u & 1 (hi, lo) of union state u >> 1
+      const int nunits = uK + (hasB ? 2 : 1);
+      for (int u = 0; u < nunits; ++u) {
         const int hsi = u % NHS, k = u / NHS;
         if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
-        const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
-        tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
-        tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
+        if (u < uK) {
+          const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
+          tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
+          tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
+        } else {
+          const int c0 = c0_of(u - uK);
+          tma_load_4d(sm.hs[hsi][0], &tmK, &sm.full[hsi], 0, h, c0, b);
+          tma_load_4d(sm.hs[hsi][1], &tmK, &sm.full[hsi], 64, h, c0, b);
+        }
         issued[hsi] = k + 1;
       }
       if (*abort) {  // let copies in flight land before the CTA exits
@@ -226,16 +287,26 @@ __global__ void __launch_bounds__(NT, 1)
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(L, D);
       bool ok = mbar_wait(&sm.bar_q, 0, abort, status);
-      for (int x = 0; ok && x < nu; ++x) {
-        const int buf = x % NBUF, kb = x / NBUF;
-        const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
-        if (!mbar_wait(&sm.acc_empty[buf], (uint32_t)((kb & 1) ^ 1), abort, status)) break;
+      // accumulator n (TMEM buffer n % NBUF): n < nu the union states, then P, then O
+      auto acc_acquire = [&](int n) -> bool {
+        const int buf = n % NBUF, kb = n / NBUF;
+        if (!mbar_wait(&sm.acc_empty[buf], (uint32_t)((kb & 1) ^ 1), abort, status)) return false;
         tc_fence_after();
+        return true;
+      };
+      auto unit_wait = [&](int u) -> bool {
+        if (!mbar_wait(&sm.full[u % NHS], (uint32_t)((u / NHS) & 1), abort, status)) return false;
+        tc_fence_after();
+        return true;
+      };
+      for (int x = 0; ok && x < nu; ++x) {
+        const int buf = x % NBUF;
+        const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
+        if (!(ok = acc_acquire(x))) break;
         const uint32_t dA = tmem + 256u * buf, dB = dA + 128u;
         for (int part = 0; part < 2; ++part) {
-          const int u = 2 * x + part, hsi = u % NHS, k = u / NHS;
-          if (!(ok = mbar_wait(&sm.full[hsi], (uint32_t)(k & 1), abort, status))) break;
-          tc_fence_after();
+          const int u = 2 * x + part, hsi = u % NHS;
+          if (!(ok = unit_wait(u))) break;
           for (int kk = 0; kk < 8; ++kk) {
             const uint32_t off = (uint32_t)(kk & 3) * 32;
             const uint64_t bdesc = desc_kmajor_sw128(smem_u32(sm.hs[hsi][kk >> 2]) + off);
@@ -245,6 +316,35 @@ __global__ void __launch_bounds__(NT, 1)
           mma_commit(&sm.empty[hsi]);
         }
         if (ok) mma_commit(&sm.acc_full[buf]);
+      }
+      // intra part: P = Q K^T (accumulator nu), then O = Pt V^T (accumulator nu + 1)
+      const int sKA = uK % NHS, sKB = (uK + 1) % NHS;
+      if (ok && (ok = acc_acquire(nu)) && (ok = unit_wait(uK)) && (!hasB || (ok = unit_wait(uK + 1)))) {
+        const uint32_t dA = tmem + 256u * (nu % NBUF), dB = dA + 128u;
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (uint32_t)(kk & 3) * 32;
+          mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off),
+                   desc_kmajor_sw128(smem_u32(sm.hs[sKA][kk >> 2]) + off), idesc, kk > 0);
+          if (hasB)
+            mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off),
+                     desc_kmajor_sw128(smem_u32(sm.hs[sKB][kk >> 2]) + off), idesc, kk > 0);
+        }
+        mma_commit(&sm.acc_full[nu % NBUF]);
+      }
+      // Pt (over Q), V^T (in the stages of units uK + 2, uK + 3) and o (in
+      // accumulator nu + 1) written by the epilogue
+      const int sVA = (uK + 2) % NHS, sVB = (uK + 3) % NHS;
+      if (ok && (ok = mbar_wait(&sm.bar_pt, 0, abort, status)) && (ok = acc_acquire(nu + 1))) {
+        const uint32_t dA = tmem + 256u * ((nu + 1) % NBUF), dB = dA + 128u;
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (uint32_t)(kk & 3) * 32;
+          mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off),
+                   desc_kmajor_sw128(smem_u32(sm.hs[sVA][kk >> 2]) + off), idesc, true);  // onto o
+          if (hasB)
+            mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off),
+                     desc_kmajor_sw128(smem_u32(sm.hs[sVB][kk >> 2]) + off), idesc, true);
+        }
+        mma_commit(&sm.acc_full[(nu + 1) % NBUF]);
       }
       mma_commit(&sm.bar_done);  // every MMA issued above has completed once this fires
       mbar_wait_drain(&sm.bar_done, 0);
@@ -261,6 +361,7 @@ __global__ void __launch_bounds__(NT, 1)
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
     const int etid = ew * 32 + lane;      // 0..511
     const int c0s = c0_of(side), Lcs = Lc_of(side);
+    const bool side_in = (side == 0 || hasB);  // warp-uniform
 
     if (etid < 2 * L) {  // both intervals' boundary flags and merge indices
       const int sd = etid / L, tt = etid % L;
@@ -269,24 +370,9 @@ __global__ void __launch_bounds__(NT, 1)
       sm.side[sd].bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
       sm.side[sd].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
     }
-    // o starts from the intra-interval part (K2a; column-quad order, so a warp
-    // reads 512 contiguous bytes per load)
-    float o[64];
-    {
-      const float* src = a.ointra + ((long long)bh * a.ointra_T + (c0s - a.t_begin)) * D + (16 * ch * L + t) * 4;
-#pragma unroll
-      for (int i = 0; i < 64; i += 4) {
-        float4 v4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (t < Lcs) v4 = *reinterpret_cast<const float4*>(src + (i / 4) * L * 4);
-        o[i] = v4.x; o[i + 1] = v4.y; o[i + 2] = v4.z; o[i + 3] = v4.w;
-      }
-    }
     asm volatile("bar.sync 1, 512;" ::: "memory");
-    if (ew == 0) {  // both slot tables (they share logi)
-      build_table(sm.side[0], sm.logi, m0A, lane);
-      __syncwarp();
-      build_table(sm.side[1], sm.logi, m0B, lane);
-    }
+    if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+    if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
     if (etid < 2 * L) {
       const int sd = etid / L, tt = etid % L;
       sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
@@ -294,49 +380,164 @@ __global__ void __launch_bounds__(NT, 1)
     asm volatile("bar.sync 1, 512;" ::: "memory");
     const long long rowbase = ((long long)b * a.T + c0s) * a.H + h;
     const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
-    const unsigned char* tab_t = sm.side[side].tab + sm.side[side].evt[t] * kMaxC;
+    const int evt_t = sm.side[side].evt[t];
     const int* ux = side ? sm.uxb : sm.uxa;
-    // weight of union state x for this token (0 when not in its interval's list)
-    auto weight = [&](int x) -> float {
-      if (x >= nu || t >= Lcs) return 0.f;
-      const int xi = ux[x];
-      if (xi < 0) return 0.f;
-      return lam_t ? lam_t[tab_t[xi]] : 1.f;
-    };
-    float wn = weight(0);
-    for (int x = 0; x < nu; ++x) {
-      const int buf = x % NBUF, kb = x / NBUF;
-      const bool in = (side == 0 || hasB) && ux[x] >= 0;  // warp-uniform
-      const float wx = wn;
-      wn = weight(x + 1);
-      // tcgen05.ld below is warp-wide: the warp takes one decision
-      if (!__all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status))) break;
-      tc_fence_after();
-      if (in) {
-        float dv[16];
+    bool ok = true;
+    {  // snapshot part: o in registers, then moved to TMEM (below)
+      float o[64];
+#pragma unroll
+      for (int i = 0; i < 64; ++i) o[i] = 0.f;
+      const unsigned char* tab_t = sm.tab[side] + evt_t * kMaxC;
+      // weight of union state x for this token (0 when not in its interval's list)
+      auto weight = [&](int x) -> float {
+        if (x >= nu || t >= Lcs) return 0.f;
+        const int xi = ux[x];
+        if (xi < 0) return 0.f;
+        return lam_t ? lam_t[tab_t[xi]] : 1.f;
+      };
+      float wn = weight(0);
+      for (int x = 0; x < nu; ++x) {
+        const int buf = x % NBUF, kb = x / NBUF;
+        const bool in = side_in && ux[x] >= 0;  // warp-uniform
+        const float wx = wn;
+        wn = weight(x + 1);
+        // tcgen05.ld below is warp-wide: the warp takes one decision
+        if (!(ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status)))) break;
+        tc_fence_after();
+        if (in) {
+          float dv[16];
+          const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
+#pragma unroll
+          for (int c = 0; c < 64; c += 16) {
+            tmem_ld16(base + c, dv);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) o[c + i] += wx * dv[i];
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
+      }
+      // ---- intra part.  o moves into this thread's rows of accumulator nu + 1
+      // (the last state's buffer, read by this thread already, or never used),
+      // which the O MMA accumulates onto.
+      if (ok && side_in) {
+        const uint32_t base = lane_addr + 256u * ((nu + 1) % NBUF) + 128u * side + 64 * ch;
+#pragma unroll
+        for (int c = 0; c < 64; c += 16) tmem_st16(base + c, o + c);
+        tmem_st_wait();
+      }
+    }
+    // V^T of this interval goes into the stage that unit
+    // uK + 2 + side would use: the last state's parts, whose MMAs are complete
+    // (this warp has seen the last state's accumulator), or a stage never used.
+    if (side_in) {  // element (j, s = t) of the K-major B operand [j][s]; this thread: j in its column half
+      const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(a.v) + (rowbase + (long long)t * a.H) * D + 64 * ch;
+      // row j = 64 ch + 8 i + u has j % 8 = u: its 16-byte chunk of column t is
+      // ((t % 64) / 8) ^ u (128-byte swizzle), the same for every i
+      uint8_t* vcol = sm.hs[(uK + 2 + side) % NHS][t >> 6] + 64 * ch * 128 + (t & 7) * 2;
+      const int c16 = (t & 63) >> 3;
+#pragma unroll
+      for (int i0 = 0; i0 < 8; i0 += 2) {
+        uint4 raw[2];
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+          raw[i] = (t < Lcs) ? *reinterpret_cast<const uint4*>(vrow + 8 * (i0 + i)) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const __nv_bfloat16* vv = reinterpret_cast<const __nv_bfloat16*>(&raw[i]);
+#pragma unroll
+          for (int u = 0; u < 8; ++u)
+            *reinterpret_cast<__nv_bfloat16*>(vcol + (8 * (i0 + i) + u) * 128 + ((c16 ^ u) << 4)) = vv[u];
+        }
+      }
+    }
+    asm volatile("bar.sync 1, 512;" ::: "memory");  // every warp is past the snapshot tables
+    if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+    if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    asm volatile("bar.sync 1, 512;" ::: "memory");
+    {  // P (accumulator nu) -> Pt over this interval's Q tile (its MMAs are complete)
+      const int buf = nu % NBUF, kb = nu / NBUF;
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status));
+      if (ok && side_in) {
+        tc_fence_after();
         const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
+        // the weight of column s depends on s only through evt[s], which changes
+        // at the interval's boundaries: it is looked up again only then
+        const unsigned char* trow = sm.tab[side] + evt_t * (evt_t + 1) / 2;
+        const int* evs = sm.side[side].evt;
+        int last_e = -1;
+        float last_w = 0.f;
+        uint8_t* qtile = sm.Q[side][ch];
 #pragma unroll
         for (int c = 0; c < 64; c += 16) {
-          tmem_ld16(base + c, dv);
+          float p[16];
+          tmem_ld16(base + c, p);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) o[c + i] += wx * dv[i];
+          for (int h8 = 0; h8 < 2; ++h8) {
+            uint32_t packed[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              float w2[2];
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int ss = 64 * ch + c + 8 * h8 + 2 * i + u;
+                float wt = 0.f;
+                if (ss <= t && t < Lcs) {
+                  const int e = evs[ss];
+                  if (e != last_e) {
+                    last_e = e;
+                    last_w = lam_t ? __ldg(lam_t + trow[e]) : 1.f;
+                  }
+                  wt = last_w;
+                }
+                w2[u] = p[8 * h8 + 2 * i + u] * wt;
+              }
+              const __nv_bfloat162 pr = __floats2bfloat162_rn(w2[0], w2[1]);
+              packed[i] = *reinterpret_cast<const uint32_t*>(&pr);
+            }
+            const int c8 = (c >> 3) + h8;  // 16-byte chunk of the row
+            *reinterpret_cast<uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4)) =
+                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+          }
+        }
+      }
+      fence_proxy_async();  // the generic-proxy writes (Pt, V^T) feed the tensor core (o: stores waited for above)
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&sm.acc_empty[buf]);
+        mbar_arrive(&sm.bar_pt);
+      }
+    }
+    {  // accumulator nu + 1: o + O, written out
+      const int buf = (nu + 1) % NBUF, kb = (nu + 1) / NBUF;
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status));
+      if (ok && side_in) {
+        tc_fence_after();
+        const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
+        const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
+        const bool st = !*abort && t < Lcs;
+#pragma unroll
+        for (int c = 0; c < 64; c += 16) {
+          float o[16];
+          tmem_ld16(base + c, o);  // warp-wide: every lane loads, rows past Lc store nothing
+          if (st) {
+            if (a.out_bf16) {
+              __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow + c;
+#pragma unroll
+              for (int i = 0; i < 16; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+            } else {
+              float* out = reinterpret_cast<float*>(a.o) + orow + c;
+#pragma unroll
+              for (int i = 0; i < 16; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+            }
+          }
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
-    }
-    if (!*abort && t < Lcs) {
-      const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
-      if (a.out_bf16) {
-        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
-#pragma unroll
-        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-      } else {
-        float* out = reinterpret_cast<float*>(a.o) + orow;
-#pragma unroll
-        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-      }
     }
   }
   tc_fence_before();
@@ -347,24 +548,23 @@ __global__ void __launch_bounds__(NT, 1)
 
 // ---------------------------------------------------------------- host side
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
-  CUtensorMap mq, ms;
+  CUtensorMap mq, mk, ms;
   const long long rows = (long long)a.B * a.H * a.pool_cap * 2 * D;
-  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows)) return cudaErrorInvalidValue;
+  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_tokens(&mk, a.k, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
+    return cudaErrorInvalidValue;
   const size_t smem = sizeof(TcSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid((a.nsnap + 1) / 2, a.B * a.H);  // pairs of intervals
-  readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, ms, status);
+  readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, mk, ms, status);
   return cudaGetLastError();
 }
 
 size_t readout_tc_smem_bytes() { return sizeof(TcSmem) + 1024; }
 
-cudaError_t preload_readout_intra();
 cudaError_t preload_readout_kernels() {
   cudaFuncAttributes fa;
-  cudaError_t e = cudaFuncGetAttributes(&fa, readout_tc_kernel);
-  return (e != cudaSuccess) ? e : preload_readout_intra();
+  return cudaFuncGetAttributes(&fa, readout_tc_kernel);
 }
 
 }  // namespace dla

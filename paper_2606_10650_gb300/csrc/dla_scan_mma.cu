@@ -1035,9 +1035,9 @@ struct GramSmem {
 
 // K0: each CTA walks the chunks of one block of one stream in order; the k, v
 // rows of the next chunk are in flight (cp.async) while it computes this one.
-// With `ready` set, the chunk count of the block is published (release) after
-// each chunk's writes, for a scan that runs concurrently and reads the block
-// through the async proxy.
+// With `ready` set, the count of the block's chunks written is published
+// (release) after its first chunk, every fourth and its last, for a scan that
+// runs concurrently and reads the blocks through the async proxy.
 template <int D>
 __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   constexpr int RP = D + 8;
@@ -1093,9 +1093,12 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
     }
     if (threadIdx.x < L / 4)
       *reinterpret_cast<float4*>(out + 2 * L * L + 4 * threadIdx.x) = *reinterpret_cast<const float4*>(sm.a + 4 * threadIdx.x);
-    if (a.ready) asm volatile("fence.proxy.async.global;" ::: "memory");  // the scan reads the block by bulk copy
+    // published after the first chunk, then every fourth and after the last
+    // (the scan reads the blocks by bulk copy: async proxy)
+    const bool publish = a.ready && (((c - c_begin) & 3) == 0 || c + 1 == c_end);
+    if (publish) asm volatile("fence.proxy.async.global;" ::: "memory");
     __syncthreads();  // the block is written; G, Q, a are reused by the next chunk
-    if (a.ready && threadIdx.x == 0) {
+    if (publish && threadIdx.x == 0) {
       __threadfence();
       st_release_gpu(a.ready + (long long)bh * a.nblk + blk, c - c_begin + 1);
     }
