@@ -509,7 +509,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
   if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
   int free_sms = 0;  // SMs the scan leaves to the rest when all its CTAs are resident (0: they are not)
-  if (P.persistent && tc && concurrent_schedule()) {
+  if (P.persistent && tc && concurrent_schedule() && (P.nsnap_total + 1) / 2 <= 65535) {  // one read-out launch
     int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_fail(e, "device query");
@@ -527,7 +527,6 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     // read-out follows the pre-pass (a waiting read-out CTA must not hold an SM
     // the pre-pass needs).  Needs every scan CTA resident at once, with SMs to
     // spare; otherwise the rounds schedule below runs.
-    const std::vector<int> sizes = round_sizes(P, false);
     {  // kernel code loaded once per device before anything of this path runs
       static bool loaded[kMaxDev] = {};
       static std::mutex mu;
@@ -573,15 +572,13 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     }
     ra.pool = sa.pool;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
-    // the read-out rounds follow the pre-pass on the read-out stream
-    int snap0 = 0;
-    for (int r = 0; r < (int)sizes.size(); snap0 += sizes[r], ++r) {
-      ra.t_begin = snap0 * P.interval;
-      ra.t_end = std::min(T, ra.t_begin + sizes[r] * P.interval);
-      ra.nsnap = sizes[r]; ra.snap_base = snap0;
-      e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
-      if (e != cudaSuccess) return cuda_fail(e, "readout launch");
-    }
+    // the read-out follows the pre-pass on the read-out stream: one launch over
+    // the whole sequence, its CTAs dispatched interval pair by interval pair
+    // (streams fastest), each waiting for its stream's progress
+    ra.t_begin = 0; ra.t_end = T;
+    ra.nsnap = P.nsnap_total; ra.snap_base = 0;
+    e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
+    if (e != cudaSuccess) return cuda_fail(e, "readout launch");
     if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaEventRecord(S->ro_done[0], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");

@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(NT, 1)
   extern __shared__ uint8_t smem_raw[];
   TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int pair = blockIdx.x, bh = blockIdx.y;
+  const int bh = blockIdx.x, pair = blockIdx.y;  // streams fastest: CTAs dispatched interval pair by pair
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const int sA = 2 * pair;
@@ -555,7 +555,8 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
   const size_t smem = sizeof(TcSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((a.nsnap + 1) / 2, a.B * a.H);  // pairs of intervals
+  if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
+  dim3 grid(a.B * a.H, (a.nsnap + 1) / 2);  // streams x pairs of intervals
   readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, mk, ms, status);
   return cudaGetLastError();
 }
