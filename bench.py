@@ -206,39 +206,91 @@ def bench_prefill(args, dist, pk):
     flops_total = 2.0 * d * d * (sum_m + 2 * T * BH)
     kt_tab = kernel_table(timing, args.steps)
     tc_path = (w.dtype == "bf16" and d == 128)
-    ro_n, ro_ms = timing["readout"]
-    sc_n, sc_ms = timing["scan"]
+    # Each kernel alone on the device: the same forward pass under the serial
+    # schedule (pre-pass, scan, read-out one after another), timed after the
+    # step.  Inside the step the kernels overlap and the read-out is paced by
+    # the scan, so their in-step durations are not their speeds.
+    solo, solo_steps = {}, min(args.steps, 5)
+    if tc_path:
+        os.environ["DLA_SCHEDULE"] = "serial"
+        try:
+            step()
+            torch.cuda.synchronize()
+            dla.dla_timing_read(reset=True)
+            dla.dla_timing_enable(True)
+            for _ in range(solo_steps):
+                step()
+            torch.cuda.synchronize()
+            dla.dla_timing_enable(False)
+            solo = dla.dla_timing_read(reset=True)
+        finally:
+            os.environ.pop("DLA_SCHEDULE", None)
+    t_in = {k: (n, ms) for k, (n, ms) in timing.items()}
     fp32_peak = pk_fp32(pk)
-    rooflines, kernel_ms = {}, {}
-    if ro_n:
-        ms_ro = ro_ms
-        kernel_ms["readout"] = ms_ro
-        ach = flops_readout * args.steps / (ms_ro * 1e-3) / 1e12  # flops_readout is per step
-        peak = pk["bf16"] if tc_path else fp32_peak
-        rooflines["readout"] = {
-            "kernel": "readout (snapshot and intra-interval parts)" if tc_path else "readout",
-            "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
-            "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
-            "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else
-                          "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
-            "work_per_launch": f"2*d^2*sum_t m_t / rounds = {flops_readout * args.steps / ro_n:.4g} flop",
-            "time_note": "summed CUDA-event durations of the round's read-out launches, which overlap the next scan",
-            "executed_note": ("each snapshot-state product runs as two bf16 MMAs (hi + lo split of the fp32 "
-                              "state): executed tensor flops are about 2x the algorithmic count" if tc_path else "")}
-    if sc_n:
-        kernel_ms["scan"] = sc_ms
-        flops_scan = 4.0 * d * d * T * BH  # x_t = v^T S k and the state build, 2 d^2 each per token
-        ach = flops_scan * args.steps / (sc_ms * 1e-3) / 1e12
-        peak = pk["bf16"] if tc_path else fp32_peak
-        rooflines["scan"] = {
-            "kernel": "scan", "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
-            "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
-            "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json; the scan's contractions run "
-                          "on mma.sync" if tc_path else "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
-            "work_per_launch": f"4*d^2*T*B*H / launches = {flops_scan * args.steps / sc_n:.4g} flop",
-            "note": "latency-bound: each (batch, head) stream is sequential; one CTA pair per stream"}
-    dominant = max(rooflines, key=lambda k: kernel_ms[k]) if rooflines else None
-    roof = rooflines.get(dominant)
+    rooflines, sm_ms = {}, {}
+    n_sms = 152
+    scan_sms = 2 * BH if 2 * BH <= n_sms else min(BH, n_sms)
+
+    def per_launch(table, name):
+        n, ms_ = table.get(name, (0, 0.0))
+        return (ms_ / n) if n else None
+
+    for name in ("readout", "scan", "gram"):
+        t_solo = per_launch(solo, name) if solo else None
+        t_step = per_launch(t_in, name)
+        t = t_solo if t_solo is not None else t_step
+        if t is None:
+            continue
+        n_launch = t_in.get(name, (0, 0.0))[0] / args.steps  # launches per step inside the timed region
+        timing_note = (f"CUDA events around each launch of the kernel alone on the device (serial schedule, "
+                       f"{solo_steps} forward passes after the timed steps); inside the timed step it lasts "
+                       f"{t_step:.4f} ms per launch, overlapped" if t_solo is not None else
+                       "CUDA events around each launch inside the timed steps")
+        if name == "readout":
+            work = 2.0 * d * d * sum_m / max(n_launch, 1)
+            peak = pk["bf16"] if tc_path else fp32_peak
+            ach = work / (t * 1e-3) / 1e12
+            rooflines[name] = {
+                "kernel": "readout (snapshot and intra-interval parts, K2)", "bound": "tensor" if tc_path else "alu",
+                "achieved": round(ach, 3), "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4),
+                "traffic": None, "ms_per_launch": round(t, 5),
+                "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else
+                              "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
+                "work_per_launch": f"2*d^2*sum_t m_t / launches = {work:.4g} flop", "timing": timing_note,
+                "executed_note": ("each snapshot-state product runs as two bf16 MMAs (hi + lo split of the fp32 "
+                                  "state): executed tensor flops are about 2x the algorithmic count" if tc_path else "")}
+            sm_ms[name] = t * n_launch * n_sms
+        elif name == "scan":
+            work = 4.0 * d * d * T * BH / max(n_launch, 1)  # x_t = v^T S k and the state build, 2 d^2 each per token
+            peak = pk["bf16"] if tc_path else fp32_peak
+            ach = work / (t * 1e-3) / 1e12
+            rooflines[name] = {
+                "kernel": "scan (K1)", "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
+                "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
+                "ms_per_launch": round(t, 5),
+                "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json; the scan's contractions "
+                              "run on mma.sync" if tc_path else "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
+                "work_per_launch": f"4*d^2*T*B*H / launches = {work:.4g} flop", "timing": timing_note,
+                "note": (f"latency-bound: each (batch, head) stream is sequential; {scan_sms} CTAs "
+                         f"({'pairs' if scan_sms == 2 * BH else 'one per stream'})")}
+            sm_ms[name] = t * n_launch * scan_sms
+        elif name == "gram":
+            nch = (T + 63) // 64
+            work = (2.0 * B * T * H * d * 2 + BH * nch * (2 * 64 * 64 + 64) * 4) / max(n_launch, 1)
+            ach = work / (t * 1e-3) / 1e9
+            rooflines[name] = {
+                "kernel": "Gram pre-pass (K0)", "bound": "hbm", "achieved": round(ach, 1), "peak": pk["hbm"],
+                "unit": "GB/s", "frac": round(ach / pk["hbm"], 4), "traffic": None, "ms_per_launch": round(t, 5),
+                "work_per_launch": f"k, v read (bf16) + Gram tables written (fp32) = {work:.4g} bytes",
+                "timing": timing_note}
+            sm_ms[name] = t * n_launch * n_sms
+    # dominant kernel: the largest SM-time per step (duration alone x SMs it occupies); the
+    # step is close to the summed SM-time of the kernels over the 152 SMs
+    dominant = max(sm_ms, key=lambda k: sm_ms[k]) if sm_ms else None
+    roof = dict(rooflines[dominant]) if dominant else None
+    if roof is not None:
+        roof["dominance"] = ("largest SM-time per step (ms alone x SMs occupied): " +
+                             ", ".join(f"{k} {v:.1f} SM-ms" for k, v in sm_ms.items()))
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -269,7 +321,9 @@ def bench_prefill(args, dist, pk):
         e2e = {"value": round(dist.world * tokens / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
                "h2d_bytes_per_step": hb, "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e}
     res = {"value": dist.world * tokens / (ms_max * 1e-3), "ms_per_step": ms_max, "tokens_per_step": tokens,
-           "roofline": roof, "rooflines": rooflines, "kernels": kt_tab, "tc_path": tc_path, "clocks": clk, "e2e": e2e,
+           "roofline": roof, "rooflines": rooflines, "kernels": kt_tab,
+           "kernels_alone": kernel_table(solo, solo_steps) if solo else None, "tc_path": tc_path, "clocks": clk,
+           "e2e": e2e,
            "gpu_launches": sum(n for n, _ in timing.values()),
            "algorithmic_tflops": flops_total / (ms_max * 1e-3) / 1e12, "sum_m": sum_m,
            "boundaries": int(bnd.sum().item()), "merges": int((ml >= 0).sum().item())}
@@ -491,7 +545,8 @@ def main():
                 "config": config_of(args), "peaks_source": pk["source"]}
         if pre:
             line.update(value=round(pre["value"], 1), ms_per_step=round(pre["ms_per_step"], 4),
-                        roofline=pre["roofline"], rooflines=pre["rooflines"], kernels=pre["kernels"], clocks=pre["clocks"], e2e=pre["e2e"],
+                        roofline=pre["roofline"], rooflines=pre["rooflines"], kernels=pre["kernels"],
+                        kernels_alone=pre["kernels_alone"], clocks=pre["clocks"], e2e=pre["e2e"],
                         gpu_launches=pre["gpu_launches"],
                         algorithmic_tflops=round(pre["algorithmic_tflops"], 3),
                         trace={"sum_m": pre["sum_m"], "boundaries": pre["boundaries"], "merges": pre["merges"]})

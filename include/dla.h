@@ -187,14 +187,16 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
                            void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
 
 /* Instrumentation (no counterpart in the paper).  Kernel kinds of the
- * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass. */
+ * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass, and
+ * the one-thread gate of the concurrent schedule. */
 typedef enum {
   DLA_K_SCAN = 0,
   DLA_K_READOUT = 1,
   DLA_K_DECODE = 2,
   DLA_K_INIT = 3,
   DLA_K_GRAM = 4,
-  DLA_K_COUNT = 5
+  DLA_K_GATE = 5,
+  DLA_K_COUNT = 6
 } dla_kernel_kind;
 
 /* enable = 1: from now on, every kernel this host thread launches through the

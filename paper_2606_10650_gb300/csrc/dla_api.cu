@@ -162,12 +162,18 @@ namespace {
 
 // Schedule of the tensor-core forward pass (environment variable DLA_SCHEDULE,
 // read at every call): "concurrent" (default) launches the scan once over the
-// whole sequence and the read-out rounds beside it, each read-out CTA waiting
-// for its stream's progress; "rounds" launches the scan once per round and the
-// round's read-out after it.  Both compute the same results.
-bool concurrent_schedule() {
+// whole sequence, the Gram pre-pass and the read-out beside it, each waiting
+// for the other side's progress; "rounds" launches the scan once per round and
+// the round's read-out after it; "serial" runs the pre-pass, the whole scan and
+// one read-out launch one after another, each kernel alone on the device (no
+// kernel waits for another: for timing and profiling single kernels).  All
+// compute the same results.
+enum Schedule { kConcurrent, kRounds, kSerial };
+Schedule schedule() {
   const char* v = getenv("DLA_SCHEDULE");
-  return !(v && strcmp(v, "rounds") == 0);
+  if (v && strcmp(v, "rounds") == 0) return kRounds;
+  if (v && strcmp(v, "serial") == 0) return kSerial;
+  return kConcurrent;
 }
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
@@ -508,8 +514,40 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = stream_set(&S)) != cudaSuccess) return cuda_fail(e, "internal streams");
   if ((e = cudaEventRecord(S->in, st)) != cudaSuccess) return cuda_fail(e, "event record");
   if ((e = cudaStreamWaitEvent(S->hi, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  const Schedule sched = schedule();
+  const bool one_readout = P.persistent && tc && (P.nsnap_total + 1) / 2 <= 65535;  // one read-out launch
+  if (one_readout && sched == kSerial) {
+    // pre-pass, whole scan, read-out, one after another on the scan stream
+    dla::GramArgs ga;
+    ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.out = (float*)(ws + P.off_gram);
+    ga.chunk0 = 0; ga.count = P.gram_chunks;
+    ga.ready = nullptr;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "device query");
+    dla::gram_blocks(B * H, P.gram_chunks, 2 * sms, &ga.nblk, &ga.per_blk);
+    if (P.gram_chunks) {
+      e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
+      if (e != cudaSuccess) return cuda_fail(e, "gram launch");
+    }
+    sa.pool = ws + P.off_pool;
+    sa.t_begin = 0; sa.t_end = T;
+    sa.nsnap = P.nsnap_total; sa.snap_base = 0;
+    sa.carry_in = 0; sa.snap_at_end = 0;
+    e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
+    if (e != cudaSuccess) return cuda_fail(e, "scan launch");
+    ra.pool = sa.pool;
+    ra.t_begin = 0; ra.t_end = T;
+    ra.nsnap = P.nsnap_total; ra.snap_base = 0;
+    e = timed(DLA_K_READOUT, S->hi, [&] { return dla::launch_readout_tc(ra, status, S->hi); });
+    if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+    if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
+    if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    return ok();
+  }
   int free_sms = 0;  // SMs the scan leaves to the rest when all its CTAs are resident (0: they are not)
-  if (P.persistent && tc && concurrent_schedule() && (P.nsnap_total + 1) / 2 <= 65535) {  // one read-out launch
+  if (one_readout && sched == kConcurrent) {
     int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_fail(e, "device query");
@@ -565,7 +603,8 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     }
     e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
-    if ((e = dla::launch_gate(started, B * H * ctas, status, S->lo)) != cudaSuccess) return cuda_fail(e, "gate launch");
+    e = timed(DLA_K_GATE, S->lo, [&] { return dla::launch_gate(started, B * H * ctas, status, S->lo); });
+    if (e != cudaSuccess) return cuda_fail(e, "gate launch");
     if (P.gram_chunks) {  // K0 beside the scan, on the SMs it leaves free
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");

@@ -22,7 +22,7 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
             "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc"]
-KERNELS = ["scan", "readout", "decode", "init", "gram"]
+KERNELS = ["scan", "readout", "decode", "init", "gram", "gate"]
 
 
 class DLAError(RuntimeError):

@@ -174,11 +174,13 @@ def test_decode_steps_match_prefill():
     assert b_all.sum() > 0 and (m_all >= 0).sum() > 0
 
 
+@pytest.mark.parametrize("sched", ["rounds", "serial"])
 @pytest.mark.parametrize("case", ["standard_bf16", "regime_bf16", "long_churn_bf16"])
-def test_forward_parity_rounds_schedule(case, monkeypatch):
-    """The rounds schedule (scan and read-out alternating round by round)
-    gives the oracle's results too."""
-    monkeypatch.setenv("DLA_SCHEDULE", "rounds")
+def test_forward_parity_other_schedules(case, sched, monkeypatch):
+    """The rounds schedule (scan and read-out alternating round by round) and
+    the serial one (pre-pass, scan, read-out one after another) give the
+    oracle's results too."""
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
     name, ov = CASES[case]
     w = W.get(name, **ov)
     q, k, v, lam = _safe(w)
