@@ -144,11 +144,12 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
  *   the Gram pre-pass and then the read-out run beside it on another stream,
  *   each waiting for the other side's progress; a kernel of the read-out side
  *   waits up to ~2 s for the scan to become resident, so the device should not
- *   be saturated by other work at that moment) or "rounds" (the scan and the
- *   read-out alternate round by round on two internal streams).  The
- *   concurrent schedule needs every scan CTA resident at once with SMs to
- *   spare; calls with more streams than that take the rounds schedule.  Both
- *   give the same results. */
+ *   be saturated by other work at that moment), "rounds" (the scan and the
+ *   read-out alternate round by round on two internal streams) or "serial"
+ *   (pre-pass, whole scan and read-out one after another, each kernel alone on
+ *   the device: for timing and profiling).  The concurrent schedule needs
+ *   every scan CTA resident at once with SMs to spare; calls with more streams
+ *   than that take the rounds schedule.  All give the same results. */
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
