@@ -17,12 +17,12 @@
 // D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128), with
 // S_x = S_hi + S_lo, the fp32 snapshot split into bf16 parts by K1 (two MMAs
 // per state and interval keep the state rounding near 2^-17 instead of 2^-9).
-// An interval's MMAs are skipped for a state that is not in its list.  After
-// the last state, the intra part of each interval: P = Q K^T, Pt = P o W
-// (W_ts = lambda_{t, L_t(e(s))} for s <= t, else 0) written as bf16 over the Q
-// tile, V^T written into the stages the last state used, O = Pt V, added to o.
-// Roles: warp 0 issues TMA loads (the two Q tiles, then the hi and lo parts of
-// each union state into four 32 KB stages, then the two K tiles), warp 1
+// An interval's MMAs are skipped for a state that is not in its list.  Before
+// the states, the intra part of each interval: P = Q K^T, Pt = P o W
+// (W_ts = lambda_{t, L_t(e(s))} for s <= t, else 0) written as bf16 over the K
+// tile, O = Pt V with V as loaded (an MN-major operand), which o starts from.
+// Roles: warp 0 issues TMA loads (the two Q, K and V tiles, then the
+// hi and lo parts of each union state through four 32 KB stages), warp 1
 // issues tcgen05.mma (one thread) into two TMEM buffers of two 128-column
 // accumulators (A, B), warps 2..17 read TMEM, weight by lambda and accumulate o
 // in registers (one token row, one interval and one 64-column half per thread;
@@ -42,15 +42,15 @@ constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
 constexpr int NT = 576;   // 18 warps
 constexpr int NEPI = 16;  // epilogue warps
-constexpr int NHS = 4;   // shared-memory stages (32 KB: one hi or lo state part, or one K tile)
+constexpr int NHS = 4;   // shared-memory stages (32 KB: a hi or lo state part, a K / Pt tile or a V tile)
 constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
 constexpr int MAXU = 2 * kMaxC;  // union of two lists
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTile = L * 128;  // one K-major 128B-swizzled tile: 128 rows x 64 bf16
 constexpr int kRows = L + 1;         // events 0 .. L of an interval
-// Slot tables of one interval, in one region: first the snapshot entries' slots
-// tab[e][x] (row stride kMaxC), later the intra part's tab[e][i] for the entry
-// opened at event i <= e (row e at e (e + 1) / 2).
+// Slot tables of one interval, in one region: first the intra part's tab[e][i]
+// for the entry opened at event i <= e (row e at e (e + 1) / 2), later the
+// snapshot entries' slots tab[e][x] (row stride kMaxC).
 constexpr int kSnapTab = kRows * kMaxC;
 constexpr int kIntraTab = kRows * (kRows + 1) / 2;
 constexpr int kTabBytes = kSnapTab > kIntraTab ? kSnapTab : kIntraTab;
@@ -62,8 +62,8 @@ struct Side {      // per interval of the pair
 };
 
 struct TcSmem {
-  uint8_t Q[2][2][kTile];      // [interval][k-half]: Q (A operand), then Pt           64 KB
-  uint8_t hs[NHS][2][kTile];   // [stage][k-half]: state parts, then K and V^T         128 KB
+  uint8_t Q[2][2][kTile];      // [interval][k-half]: Q, the A operand                 64 KB
+  uint8_t hs[NHS][2][kTile];   // [stage][half]: K then Pt, V, then state parts         128 KB
   unsigned char tab[2][kTabBytes];
   Side side[2];
   int ids[2][kMaxC];           // pool ids of the two lists
@@ -157,7 +157,8 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
 // 18 warps: the sub-partitions holding five of them bound a thread to 96 registers
 __global__ void __launch_bounds__(NT, 1)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                      const __grid_constant__ CUtensorMap tmS, int32_t* status) {
+                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
+                      int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -196,6 +197,7 @@ __global__ void __launch_bounds__(NT, 1)
     // the Q tiles go out first; they depend on nothing
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
     prefetch_tmap(&tmS);
     mbar_expect_tx(&sm.bar_q, (hasB ? 4 : 2) * kTile);
     tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, c0A, b);
@@ -250,30 +252,41 @@ __global__ void __launch_bounds__(NT, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   const int nu = sm.nu;
-  // ring units: u < 2 nu are the hi / lo parts of union state u >> 1; units
-  // 2 nu and 2 nu + 1 the K tiles of intervals A and B.  Unit u uses stage
-  // u % NHS for the (u / NHS)-th time.
-  const int uK = 2 * nu;
+  // Ring units: g = 0, 1 the K tiles of intervals A and B (then Pt over them),
+  // g = 2, 3 their V tiles (the MN-major B operand of O), g = 4 + u the hi / lo part
+  // u & 1 of union state u >> 1.  Unit g uses stage g % NHS for the
+  // (g / NHS)-th time.  Accumulators (TMEM buffer n % NBUF): n = 0 P = Q K^T,
+  // n = 1 O = Pt V, n = 2 + x union state x.
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int issued[NHS];  // uses of each stage so far
-      for (int i = 0; i < NHS; ++i) issued[i] = 0;
-      const int nunits = uK + (hasB ? 2 : 1);
-      for (int u = 0; u < nunits; ++u) {
-        const int hsi = u % NHS, k = u / NHS;
+      mbar_expect_tx(&sm.full[0], 2 * kTile);
+      tma_load_4d(sm.hs[0][0], &tmK, &sm.full[0], 0, h, c0A, b);
+      tma_load_4d(sm.hs[0][1], &tmK, &sm.full[0], 64, h, c0A, b);
+      mbar_expect_tx(&sm.full[2], 2 * kTile);
+      tma_load_4d(sm.hs[2][0], &tmV, &sm.full[2], 0, h, c0A, b);
+      tma_load_4d(sm.hs[2][1], &tmV, &sm.full[2], 64, h, c0A, b);
+      if (hasB) {
+        mbar_expect_tx(&sm.full[1], 2 * kTile);
+        tma_load_4d(sm.hs[1][0], &tmK, &sm.full[1], 0, h, c0B, b);
+        tma_load_4d(sm.hs[1][1], &tmK, &sm.full[1], 64, h, c0B, b);
+        mbar_expect_tx(&sm.full[3], 2 * kTile);
+        tma_load_4d(sm.hs[3][0], &tmV, &sm.full[3], 0, h, c0B, b);
+        tma_load_4d(sm.hs[3][1], &tmV, &sm.full[3], 64, h, c0B, b);
+      } else {  // first phase complete without data: the stages' later uses keep their parity
+        mbar_arrive(&sm.full[1]);
+        mbar_arrive(&sm.full[3]);
+      }
+      for (int i = 0; i < NHS; ++i) issued[i] = 1;
+      for (int u = 0; u < 2 * nu; ++u) {
+        const int g = 4 + u, hsi = g % NHS, k = g / NHS;
         if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
-        if (u < uK) {
-          const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
-          tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
-          tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
-        } else {
-          const int c0 = c0_of(u - uK);
-          tma_load_4d(sm.hs[hsi][0], &tmK, &sm.full[hsi], 0, h, c0, b);
-          tma_load_4d(sm.hs[hsi][1], &tmK, &sm.full[hsi], 64, h, c0, b);
-        }
+        const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
+        tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
+        tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
         issued[hsi] = k + 1;
       }
       if (*abort) {  // let copies in flight land before the CTA exits
@@ -286,65 +299,74 @@ __global__ void __launch_bounds__(NT, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(L, D);
-      bool ok = mbar_wait(&sm.bar_q, 0, abort, status);
-      // accumulator n (TMEM buffer n % NBUF): n < nu the union states, then P, then O
       auto acc_acquire = [&](int n) -> bool {
         const int buf = n % NBUF, kb = n / NBUF;
         if (!mbar_wait(&sm.acc_empty[buf], (uint32_t)((kb & 1) ^ 1), abort, status)) return false;
         tc_fence_after();
         return true;
       };
-      auto unit_wait = [&](int u) -> bool {
-        if (!mbar_wait(&sm.full[u % NHS], (uint32_t)((u / NHS) & 1), abort, status)) return false;
+      auto unit_wait = [&](int g) -> bool {
+        if (!mbar_wait(&sm.full[g % NHS], (uint32_t)((g / NHS) & 1), abort, status)) return false;
         tc_fence_after();
         return true;
       };
+      // Descriptors: a tile's descriptor plus (byte offset >> 4) addresses a
+      // later part of it (shared-memory addresses stay below 2^18).  K step kk
+      // of a K-major 128-row tile pair: k-half kk / 4, 32 bytes per step.
+      const uint64_t qd0 = desc_kmajor_sw128(smem_u32(sm.Q[0][0]));
+      const uint64_t qd1 = desc_kmajor_sw128(smem_u32(sm.Q[1][0]));
+      const uint64_t hd0 = desc_kmajor_sw128(smem_u32(sm.hs[0][0]));
+      constexpr uint64_t kStage = (2 * kTile) >> 4;
+      auto kstep = [](int kk) -> uint64_t { return (uint64_t)((kk >> 2) * (kTile >> 4) + (kk & 3) * 2); };
+      bool ok = mbar_wait(&sm.bar_q, 0, abort, status) && unit_wait(0) && (!hasB || unit_wait(1));
+      if (ok) {  // P = Q K^T (accumulator 0; buffer 0 is fresh)
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          mma_bf16(tmem, qd0 + kstep(kk), hd0 + kstep(kk), idesc, kk > 0);
+          if (hasB) mma_bf16(tmem + 128u, qd1 + kstep(kk), hd0 + kStage + kstep(kk), idesc, kk > 0);
+        }
+        mma_commit(&sm.acc_full[0]);
+      }
+      // O = Pt V (accumulator 1; buffer 1 is fresh): Pt over the K tiles
+      // (stages 0, 1, written by the epilogue), V in stages 2, 3 as loaded:
+      // [s][j], the MN-major B operand (K step: 16 rows of 128 bytes)
+      if (ok && (ok = mbar_wait(&sm.bar_pt, 0, abort, status)) && (ok = unit_wait(2)) && (!hasB || (ok = unit_wait(3)))) {
+        constexpr uint32_t idesc_v = idesc_bf16_f32_bmn(L, D);
+        const uint64_t vd0 = desc_mnmajor_sw128(smem_u32(sm.hs[2][0]), kTile);
+        const uint64_t vd1 = desc_mnmajor_sw128(smem_u32(sm.hs[3][0]), kTile);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          mma_bf16(tmem + 256u, hd0 + kstep(kk), vd0 + (uint64_t)(kk * (2048 >> 4)), idesc_v, kk > 0);
+          if (hasB) mma_bf16(tmem + 384u, hd0 + kStage + kstep(kk), vd1 + (uint64_t)(kk * (2048 >> 4)), idesc_v, kk > 0);
+        }
+        mma_commit(&sm.acc_full[1]);
+      }
+      for (int i = 0; i < NHS; ++i) mma_commit(&sm.empty[i]);  // every stage is free once O is done
       for (int x = 0; ok && x < nu; ++x) {
         const int buf = x % NBUF;
         const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
-        if (!(ok = acc_acquire(x))) break;
+        if (!(ok = acc_acquire(x + 2))) break;
         const uint32_t dA = tmem + 256u * buf, dB = dA + 128u;
         for (int part = 0; part < 2; ++part) {
-          const int u = 2 * x + part, hsi = u % NHS;
-          if (!(ok = unit_wait(u))) break;
-          for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t off = (uint32_t)(kk & 3) * 32;
-            const uint64_t bdesc = desc_kmajor_sw128(smem_u32(sm.hs[hsi][kk >> 2]) + off);
-            if (inA) mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off), bdesc, idesc, (part | kk) > 0);
-            if (inB) mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off), bdesc, idesc, (part | kk) > 0);
+          const int g = 4 + 2 * x + part, hsi = g % NHS;
+          if (!(ok = unit_wait(g))) break;
+          const uint64_t bd = hd0 + (uint64_t)hsi * kStage;
+          if (inA && inB) {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t acc = (part | kk) > 0;
+              mma_bf16(dA, qd0 + kstep(kk), bd + kstep(kk), idesc, acc);
+              mma_bf16(dB, qd1 + kstep(kk), bd + kstep(kk), idesc, acc);
+            }
+          } else if (inA || inB) {
+            const uint32_t dd = inA ? dA : dB;
+            const uint64_t qd = inA ? qd0 : qd1;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) mma_bf16(dd, qd + kstep(kk), bd + kstep(kk), idesc, (part | kk) > 0);
           }
           mma_commit(&sm.empty[hsi]);
         }
         if (ok) mma_commit(&sm.acc_full[buf]);
-      }
-      // intra part: P = Q K^T (accumulator nu), then O = Pt V^T (accumulator nu + 1)
-      const int sKA = uK % NHS, sKB = (uK + 1) % NHS;
-      if (ok && (ok = acc_acquire(nu)) && (ok = unit_wait(uK)) && (!hasB || (ok = unit_wait(uK + 1)))) {
-        const uint32_t dA = tmem + 256u * (nu % NBUF), dB = dA + 128u;
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (uint32_t)(kk & 3) * 32;
-          mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off),
-                   desc_kmajor_sw128(smem_u32(sm.hs[sKA][kk >> 2]) + off), idesc, kk > 0);
-          if (hasB)
-            mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off),
-                     desc_kmajor_sw128(smem_u32(sm.hs[sKB][kk >> 2]) + off), idesc, kk > 0);
-        }
-        mma_commit(&sm.acc_full[nu % NBUF]);
-      }
-      // Pt (over Q), V^T (in the stages of units uK + 2, uK + 3) and o (in
-      // accumulator nu + 1) written by the epilogue
-      const int sVA = (uK + 2) % NHS, sVB = (uK + 3) % NHS;
-      if (ok && (ok = mbar_wait(&sm.bar_pt, 0, abort, status)) && (ok = acc_acquire(nu + 1))) {
-        const uint32_t dA = tmem + 256u * ((nu + 1) % NBUF), dB = dA + 128u;
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t off = (uint32_t)(kk & 3) * 32;
-          mma_bf16(dA, desc_kmajor_sw128(smem_u32(sm.Q[0][kk >> 2]) + off),
-                   desc_kmajor_sw128(smem_u32(sm.hs[sVA][kk >> 2]) + off), idesc, true);  // onto o
-          if (hasB)
-            mma_bf16(dB, desc_kmajor_sw128(smem_u32(sm.Q[1][kk >> 2]) + off),
-                     desc_kmajor_sw128(smem_u32(sm.hs[sVB][kk >> 2]) + off), idesc, true);
-        }
-        mma_commit(&sm.acc_full[(nu + 1) % NBUF]);
       }
       mma_commit(&sm.bar_done);  // every MMA issued above has completed once this fires
       mbar_wait_drain(&sm.bar_done, 0);
@@ -362,6 +384,7 @@ __global__ void __launch_bounds__(NT, 1)
     const int etid = ew * 32 + lane;      // 0..511
     const int c0s = c0_of(side), Lcs = Lc_of(side);
     const bool side_in = (side == 0 || hasB);  // warp-uniform
+    const long long rowbase = ((long long)b * a.T + c0s) * a.H + h;
 
     if (etid < 2 * L) {  // both intervals' boundary flags and merge indices
       const int sd = etid / L, tt = etid % L;
@@ -371,22 +394,97 @@ __global__ void __launch_bounds__(NT, 1)
       sm.side[sd].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");
-    if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-    if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+    if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
     if (etid < 2 * L) {
       const int sd = etid / L, tt = etid % L;
       sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");
-    const long long rowbase = ((long long)b * a.T + c0s) * a.H + h;
     const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
     const int evt_t = sm.side[side].evt[t];
-    const int* ux = side ? sm.uxb : sm.uxa;
-    bool ok = true;
-    {  // snapshot part: o in registers, then moved to TMEM (below)
-      float o[64];
+    // an interval without boundary events (the common case) weights every
+    // column s <= t of row t by lambda of the open entry: loaded ahead of P
+    const bool no_ev = sm.side[side].evt[L - 1] == 0;  // warp-uniform
+    const float w_open = (no_ev && t < Lcs) ? (lam_t ? __ldg(lam_t + sm.tab[side][0]) : 1.f) : 0.f;
+    bool ok;
+    {  // P (accumulator 0) -> Pt over this interval's K tile (its MMAs are complete)
+      ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[0], 0, abort, status));
+      if (ok && side_in) {
+        tc_fence_after();
+        const uint32_t base = lane_addr + 128u * side + 64 * ch;
+        // the weight of column s depends on s only through evt[s], which changes
+        // at the interval's boundaries: it is looked up again only then
+        const unsigned char* trow = sm.tab[side] + evt_t * (evt_t + 1) / 2;
+        const int* evs = sm.side[side].evt;
+        int last_e = -1;
+        float last_w = 0.f;
+        uint8_t* ptile = sm.hs[side][ch];
 #pragma unroll
-      for (int i = 0; i < 64; ++i) o[i] = 0.f;
+        for (int c = 0; c < 64; c += 16) {
+          float p[16];
+          tmem_ld16(base + c, p);
+#pragma unroll
+          for (int h8 = 0; h8 < 2; ++h8) {
+            uint32_t packed[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              float w2[2];
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int ss = 64 * ch + c + 8 * h8 + 2 * i + u;
+                float wt = 0.f;
+                if (no_ev) {
+                  wt = (ss <= t) ? w_open : 0.f;
+                } else if (ss <= t && t < Lcs) {
+                  const int e = evs[ss];
+                  if (e != last_e) {
+                    last_e = e;
+                    last_w = lam_t ? __ldg(lam_t + trow[e]) : 1.f;
+                  }
+                  wt = last_w;
+                }
+                w2[u] = p[8 * h8 + 2 * i + u] * wt;
+              }
+              const __nv_bfloat162 pr = __floats2bfloat162_rn(w2[0], w2[1]);
+              packed[i] = *reinterpret_cast<const uint32_t*>(&pr);
+            }
+            const int c8 = (c >> 3) + h8;  // 16-byte chunk of the row
+            *reinterpret_cast<uint4*>(ptile + t * 128 + ((c8 ^ (t & 7)) << 4)) =
+                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+          }
+        }
+      }
+      fence_proxy_async();  // the generic-proxy writes (Pt) feed the tensor core
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&sm.acc_empty[0]);
+        mbar_arrive(&sm.bar_pt);
+      }
+    }
+    asm volatile("bar.sync 1, 512;" ::: "memory");  // every warp is past the intra tables
+    if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+    if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    asm volatile("bar.sync 1, 512;" ::: "memory");
+    float o[64];
+    {  // o starts from O (accumulator 1)
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[1], 0, abort, status));
+      if (ok && side_in) {
+        tc_fence_after();
+        const uint32_t base = lane_addr + 256u + 128u * side + 64 * ch;
+#pragma unroll
+        for (int c = 0; c < 64; c += 16) tmem_ld16(base + c, o + c);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) o[i] = 0.f;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.acc_empty[1]);
+    }
+    const int* ux = side ? sm.uxb : sm.uxa;
+    {  // snapshot part
       const unsigned char* tab_t = sm.tab[side] + evt_t * kMaxC;
       // weight of union state x for this token (0 when not in its interval's list)
       auto weight = [&](int x) -> float {
@@ -396,8 +494,8 @@ __global__ void __launch_bounds__(NT, 1)
         return lam_t ? lam_t[tab_t[xi]] : 1.f;
       };
       float wn = weight(0);
-      for (int x = 0; x < nu; ++x) {
-        const int buf = x % NBUF, kb = x / NBUF;
+      for (int x = 0; ok && x < nu; ++x) {
+        const int n = x + 2, buf = n % NBUF, kb = n / NBUF;
         const bool in = side_in && ux[x] >= 0;  // warp-uniform
         const float wx = wn;
         wn = weight(x + 1);
@@ -418,126 +516,18 @@ __global__ void __launch_bounds__(NT, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
       }
-      // ---- intra part.  o moves into this thread's rows of accumulator nu + 1
-      // (the last state's buffer, read by this thread already, or never used),
-      // which the O MMA accumulates onto.
-      if (ok && side_in) {
-        const uint32_t base = lane_addr + 256u * ((nu + 1) % NBUF) + 128u * side + 64 * ch;
-#pragma unroll
-        for (int c = 0; c < 64; c += 16) tmem_st16(base + c, o + c);
-        tmem_st_wait();
-      }
     }
-    // V^T of this interval goes into the stage that unit
-    // uK + 2 + side would use: the last state's parts, whose MMAs are complete
-    // (this warp has seen the last state's accumulator), or a stage never used.
-    if (side_in) {  // element (j, s = t) of the K-major B operand [j][s]; this thread: j in its column half
-      const __nv_bfloat16* vrow = reinterpret_cast<const __nv_bfloat16*>(a.v) + (rowbase + (long long)t * a.H) * D + 64 * ch;
-      // row j = 64 ch + 8 i + u has j % 8 = u: its 16-byte chunk of column t is
-      // ((t % 64) / 8) ^ u (128-byte swizzle), the same for every i
-      uint8_t* vcol = sm.hs[(uK + 2 + side) % NHS][t >> 6] + 64 * ch * 128 + (t & 7) * 2;
-      const int c16 = (t & 63) >> 3;
+    if (ok && !*abort && side_in && t < Lcs) {
+      const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
+      if (a.out_bf16) {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
 #pragma unroll
-      for (int i0 = 0; i0 < 8; i0 += 2) {
-        uint4 raw[2];
+        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
+      } else {
+        float* out = reinterpret_cast<float*>(a.o) + orow;
 #pragma unroll
-        for (int i = 0; i < 2; ++i)
-          raw[i] = (t < Lcs) ? *reinterpret_cast<const uint4*>(vrow + 8 * (i0 + i)) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int i = 0; i < 2; ++i) {
-          const __nv_bfloat16* vv = reinterpret_cast<const __nv_bfloat16*>(&raw[i]);
-#pragma unroll
-          for (int u = 0; u < 8; ++u)
-            *reinterpret_cast<__nv_bfloat16*>(vcol + (8 * (i0 + i) + u) * 128 + ((c16 ^ u) << 4)) = vv[u];
-        }
+        for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
       }
-    }
-    asm volatile("bar.sync 1, 512;" ::: "memory");  // every warp is past the snapshot tables
-    if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-    if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
-    asm volatile("bar.sync 1, 512;" ::: "memory");
-    {  // P (accumulator nu) -> Pt over this interval's Q tile (its MMAs are complete)
-      const int buf = nu % NBUF, kb = nu / NBUF;
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status));
-      if (ok && side_in) {
-        tc_fence_after();
-        const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
-        // the weight of column s depends on s only through evt[s], which changes
-        // at the interval's boundaries: it is looked up again only then
-        const unsigned char* trow = sm.tab[side] + evt_t * (evt_t + 1) / 2;
-        const int* evs = sm.side[side].evt;
-        int last_e = -1;
-        float last_w = 0.f;
-        uint8_t* qtile = sm.Q[side][ch];
-#pragma unroll
-        for (int c = 0; c < 64; c += 16) {
-          float p[16];
-          tmem_ld16(base + c, p);
-#pragma unroll
-          for (int h8 = 0; h8 < 2; ++h8) {
-            uint32_t packed[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              float w2[2];
-#pragma unroll
-              for (int u = 0; u < 2; ++u) {
-                const int ss = 64 * ch + c + 8 * h8 + 2 * i + u;
-                float wt = 0.f;
-                if (ss <= t && t < Lcs) {
-                  const int e = evs[ss];
-                  if (e != last_e) {
-                    last_e = e;
-                    last_w = lam_t ? __ldg(lam_t + trow[e]) : 1.f;
-                  }
-                  wt = last_w;
-                }
-                w2[u] = p[8 * h8 + 2 * i + u] * wt;
-              }
-              const __nv_bfloat162 pr = __floats2bfloat162_rn(w2[0], w2[1]);
-              packed[i] = *reinterpret_cast<const uint32_t*>(&pr);
-            }
-            const int c8 = (c >> 3) + h8;  // 16-byte chunk of the row
-            *reinterpret_cast<uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4)) =
-                make_uint4(packed[0], packed[1], packed[2], packed[3]);
-          }
-        }
-      }
-      fence_proxy_async();  // the generic-proxy writes (Pt, V^T) feed the tensor core (o: stores waited for above)
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&sm.acc_empty[buf]);
-        mbar_arrive(&sm.bar_pt);
-      }
-    }
-    {  // accumulator nu + 1: o + O, written out
-      const int buf = (nu + 1) % NBUF, kb = (nu + 1) / NBUF;
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status));
-      if (ok && side_in) {
-        tc_fence_after();
-        const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
-        const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
-        const bool st = !*abort && t < Lcs;
-#pragma unroll
-        for (int c = 0; c < 64; c += 16) {
-          float o[16];
-          tmem_ld16(base + c, o);  // warp-wide: every lane loads, rows past Lc store nothing
-          if (st) {
-            if (a.out_bf16) {
-              __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow + c;
-#pragma unroll
-              for (int i = 0; i < 16; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-            } else {
-              float* out = reinterpret_cast<float*>(a.o) + orow + c;
-#pragma unroll
-              for (int i = 0; i < 16; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
-            }
-          }
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
     }
   }
   tc_fence_before();
@@ -548,16 +538,17 @@ __global__ void __launch_bounds__(NT, 1)
 
 // ---------------------------------------------------------------- host side
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
-  CUtensorMap mq, mk, ms;
+  CUtensorMap mq, mk, mv, ms;
   const long long rows = (long long)a.B * a.H * a.pool_cap * 2 * D;
-  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_tokens(&mk, a.k, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
+  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_tokens(&mk, a.k, a.B, a.T, a.H) ||
+      !tmap_tokens(&mv, a.v, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
     return cudaErrorInvalidValue;
   const size_t smem = sizeof(TcSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
   dim3 grid(a.B * a.H, (a.nsnap + 1) / 2);  // streams x pairs of intervals
-  readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, mk, ms, status);
+  readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, mk, mv, ms, status);
   return cudaGetLastError();
 }
 

@@ -211,6 +211,20 @@ __device__ __forceinline__ uint64_t desc_kmajor_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of an MN-major operand in the 128-byte
+// swizzle mode: rows of 64 bf16 along N (or M), one row per K index, 8-row
+// groups 1024 bytes apart; n_half_bytes separates the 64-wide N blocks.  A K
+// step of 16 rows starts 2048 bytes further.
+__device__ __forceinline__ uint64_t desc_mnmajor_sw128(uint32_t saddr, uint32_t n_half_bytes) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);             // start address
+  d |= (uint64_t)((n_half_bytes >> 4) & 0x3FFFu) << 16;  // leading byte offset: next 64-wide N block
+  d |= (uint64_t)(1024 >> 4) << 32;                      // stride byte offset: next 8 K rows
+  d |= (uint64_t)1 << 46;                                // descriptor version (sm_100 family)
+  d |= (uint64_t)2 << 61;                                // SWIZZLE_128B
+  return d;
+}
+
 // Instruction descriptor of kind::f16: bf16 A and B, fp32 D, both K-major.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4)                        // D format: f32
@@ -219,6 +233,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          | ((uint32_t)(N >> 3) << 17)     // N / 8
          | ((uint32_t)(M >> 4) << 24);    // M / 16
 }
+// The same with B MN-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) { return idesc_bf16_f32(M, N) | (1u << 16); }
 
 // Byte offset of element (row r, column c) of a K-major 128B-swizzled tile
 // whose rows hold 64 bf16 (c in 0..63).
