@@ -1,4 +1,4 @@
-// dla_tmap.h -- host-side TMA tensor maps of the tensor-core read-out kernels
+// dla_tmap.h -- host-side TMA tensor maps of the tensor-core kernels
 // (cuTensorMapEncodeTiled, reached through the runtime's driver entry point).
 #pragma once
 
@@ -21,15 +21,15 @@ inline PFN_cuTensorMapEncodeTiled_v12000 tmap_encode_fn() {
   return fn;
 }
 
-// [B, T, H, 128] bf16 token rows: dims (k, h, t, b), box (64, 1, 128, 1) with the
-// 128-byte swizzle (one K-major operand tile of 128 tokens x 64 features).
-inline bool tmap_tokens(CUtensorMap* m, const void* base, int B, int T, int H) {
+// [B, T, H, D] bf16 token rows: dims (k, h, t, b), box (64, 1, box_t, 1) with the
+// 128-byte swizzle (one K-major operand tile of box_t tokens x 64 features);
+// tokens past T read as zeros.
+inline bool tmap_tokens(CUtensorMap* m, const void* base, int B, int T, int H, int box_t = 128, int D = 128) {
   auto fn = tmap_encode_fn();
   if (!fn) return false;
-  constexpr int D = 128;
   cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
   cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2, (cuuint64_t)T * H * D * 2};
-  cuuint32_t box[4] = {64, 1, 128, 1};
+  cuuint32_t box[4] = {64, 1, (cuuint32_t)box_t, 1};
   cuuint32_t es[4] = {1, 1, 1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
