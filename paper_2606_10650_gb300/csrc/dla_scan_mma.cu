@@ -165,6 +165,52 @@ __device__ __forceinline__ void gram_tile(const __nv_bfloat16* Ks, const __nv_bf
     }
 }
 
+// gram_tile computing only the 16 x 16 tiles on or below the diagonal (the
+// Gram pre-pass; the scan keeps its own copy).
+template <int D>
+__device__ __forceinline__ void gram_tile_lower(const __nv_bfloat16* Ks, const __nv_bfloat16* Vs, float* Gout, float* aout) {
+  constexpr int RP = D + 8;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> 2, tg = lane & 3, q = lane >> 3, r8 = lane & 7;
+  const int mt = warp & 3, sb = 32 * (warp >> 2);
+  // only 16 x 16 tiles with columns s <= the band's last row are needed (s < t,
+  // and the diagonal for a_t): column block sb / 16 + np against row band mt
+  const bool need0 = (sb >> 4) <= mt, need1 = (sb >> 4) + 1 <= mt;  // warp-uniform
+  float kk4[4][4], vv4[4][4];
+#pragma unroll
+  for (int n = 0; n < 4; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) kk4[n][e] = vv4[n][e] = 0.f;
+#pragma unroll 2
+  for (int kk = 0; kk < D; kk += 16) {
+    if (!need0) break;
+    uint32_t ak[4], av[4];
+    ldsm4(ak, Ks + (16 * mt + (q & 1) * 8 + r8) * RP + kk + (q >> 1) * 8);
+    ldsm4(av, Vs + (16 * mt + (q & 1) * 8 + r8) * RP + kk + (q >> 1) * 8);
+#pragma unroll
+    for (int np = 0; np < 2; ++np) {
+      if (np == 1 && !need1) continue;
+      uint32_t bk[4], bv[4];
+      ldsm4(bk, Ks + (sb + 16 * np + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8);
+      ldsm4(bv, Vs + (sb + 16 * np + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8);
+      mma16816(kk4[2 * np], ak, bk[0], bk[1]);
+      mma16816(kk4[2 * np + 1], ak, bk[2], bk[3]);
+      mma16816(vv4[2 * np], av, bv[0], bv[1]);
+      mma16816(vv4[2 * np + 1], av, bv[2], bv[3]);
+    }
+  }
+#pragma unroll
+  for (int n = 0; n < 4; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int t = 16 * mt + g + 8 * (e >> 1);
+      const int s2 = sb + 8 * n + 2 * tg + (e & 1);
+      const float gv = kk4[n][e] * vv4[n][e];
+      Gout[t * (L + 1) + s2] = (s2 < t) ? gv : 0.f;
+      if (s2 == t) aout[t] = gv;
+    }
+}
+
 // Row suffix sums in place: G[t][j] <- sum_{j <= s < t} G[t][s] (a warp per row).
 __device__ __forceinline__ void suffix_rows(float* G) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1075,7 +1121,7 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
       asm volatile("cp.async.wait_group 0;" ::: "memory");
     }
     __syncthreads();
-    gram_tile<D>(sm.k[st], sm.v[st], sm.G, sm.a);
+    gram_tile_lower<D>(sm.k[st], sm.v[st], sm.G, sm.a);
     __syncthreads();
     suffix_rows_ilp(sm.G);  // G[t][j] = gs[j][t]
     __syncthreads();
