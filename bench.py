@@ -284,6 +284,14 @@ def bench_prefill(args, dist, pk):
                 "work_per_launch": f"k, v read (bf16) + Gram tables written (fp32) = {work:.4g} bytes",
                 "timing": timing_note}
             sm_ms[name] = t * n_launch * n_sms
+    # DRAM traffic per launch from a committed ncu summary, while the kernel's source is the one
+    # captured and the workload is the one captured (else null)
+    tr = captured_traffic("readout_tc_kernel", "paper_2606_10650_gb300/csrc/dla_readout_tc.cu",
+                          "profiles/readout_dram_regime_full.md")
+    if tr and "readout" in rooflines and tc_path and (args.workload, B, T, H, d) == ("regime", 2, 16384, 16, 128):
+        rooflines["readout"]["traffic"] = tr
+        rooflines["readout"]["traffic_note"] = ("dram__bytes_read.sum + dram__bytes_write.sum of one full-size "
+                                                "launch (ncu, profiles/readout_dram_regime_full.md)")
     # dominant kernel: the largest SM-time per step (duration alone x SMs it occupies); the
     # step is close to the summed SM-time of the kernels over the 152 SMs
     dominant = max(sm_ms, key=lambda k: sm_ms[k]) if sm_ms else None
@@ -330,6 +338,26 @@ def bench_prefill(args, dist, pk):
     del qt, kt, vt, lt, o, buf, cache
     torch.cuda.empty_cache()
     return res
+
+
+def captured_traffic(kernel, source, summary):
+    """Bytes per launch recorded in a profile summary line
+    'traffic_bytes_per_launch <kernel> <bytes> <sha256 prefix of source>', if the source file
+    still has that hash; else None."""
+    import hashlib
+    root = os.path.dirname(os.path.abspath(__file__))
+    try:
+        with open(os.path.join(root, source), "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+        with open(os.path.join(root, summary)) as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) == 4 and parts[0] == "traffic_bytes_per_launch" and parts[1] == kernel:
+                    if sha.startswith(parts[3]):
+                        return int(parts[2])
+    except OSError:
+        return None
+    return None
 
 
 def pk_fp32(pk):
