@@ -599,7 +599,6 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     if (P.gram_chunks) {
       sa.gram_ready = gram_ready;
       sa.gram_nblk = ga.nblk;
-      sa.gram_per_blk = ga.per_blk;
     }
     e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");

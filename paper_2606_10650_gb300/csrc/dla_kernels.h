@@ -60,10 +60,11 @@ struct ScanArgs {
   const float* gram;     // Gram pre-pass output [B*H][gram_chunks][kGramBlock], or nullptr
   int gram_chunks;       // 64-token chunks of the whole sequence
   // Gram pre-pass running beside the scan (nullptr: it finished before the
-  // scan started): [B*H][gram_nblk] chunks written so far by the pre-pass CTA
-  // of each block of gram_per_blk consecutive chunks, which writes them in order
+  // scan started; the pre-pass then starts at chunk 0): [B*H][gram_nblk] chunks
+  // written so far by the pre-pass CTA of each block (block b: chunks b,
+  // b + gram_nblk, ..., written in that order)
   const int32_t* gram_ready;
-  int gram_nblk, gram_per_blk;
+  int gram_nblk;
   int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
   int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)
@@ -74,17 +75,17 @@ struct ScanArgs {
 //   gs[j][t] = sum_{j <= s < t} G_ts       (beta_t of a segment opened at j, without S)
 //   Q[j][t]  = sum_{j <= u < t} gs[j][u]   (their running sum over the segment)
 //   a_t      = G_tt
-// One CTA per (stream, block of per_blk consecutive chunks of this launch)
-// walks its block in order, loading the next chunk while it computes this one.
+// One CTA per (stream, block): block b of a launch takes its chunks chunk0 + b,
+// chunk0 + b + nblk, ... in order, loading the next while it computes this one.
 struct GramArgs {
   const void* k;
   const void* v;
   int B, T, H;
   int nchunks;           // chunks of the whole sequence
   int chunk0, count;     // this launch: chunks chunk0 .. chunk0 + count - 1
-  int nblk, per_blk;     // blocks of this launch and chunks per block (nblk * per_blk >= count)
+  int nblk, per_blk;     // blocks of this launch and chunks per block at most (nblk * per_blk >= count)
   float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64)
-  int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after each), or nullptr
+  int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after its first four, then every fourth), or nullptr
 };
 constexpr int kMaxGramBlk = 64;  // blocks per stream of one Gram launch, at most
 

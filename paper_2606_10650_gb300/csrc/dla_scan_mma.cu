@@ -52,6 +52,7 @@ struct MmaSmem {
   int snap_src[kMaxC][2];
   int nops, nsnapjobs;
   int pend;                         // snapshot copies waiting for the next chunk's idle warps (bf16 pool)
+  int gcnt[kMaxGramBlk];            // Gram pre-pass counters last read (thread 0)
   int m, cur, js, seg_pre, pool_next;
 };
 
@@ -63,23 +64,23 @@ __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1)
 }
 
 // Gram pre-pass running beside the scan: thread 0 of the scan CTA waits until
-// the pre-pass CTA of chunk gc's block has published the chunk (its counter
-// counts the block's chunks written, in order), remembering the last count.
+// the pre-pass CTA of chunk gc's block (block gc % nblk, which takes chunks
+// blk, blk + nblk, ... in order) has published the chunk (its counter counts
+// the block's chunks written), remembering the last count of every block.
 struct GramFeed {
   const int32_t* ready;  // this stream's [nblk] counters, or nullptr (the pre-pass has finished)
-  int per;               // chunks per block
-  int blk, cnt;          // last counter value read, and its block
+  int nblk;              // blocks of the pre-pass per stream
+  int* cnt;              // [nblk] last counter value read (shared memory, thread 0)
 };
 __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int* abort, int32_t* status) {
   if (!f.ready) return true;
-  const int blk = gc / f.per, need = gc - blk * f.per + 1;
-  if (blk != f.blk || f.cnt < need) {
+  const int blk = gc % f.nblk, need = gc / f.nblk + 1;
+  if (f.cnt[blk] < need) {
     const long long t0 = clock64();
     while (true) {
       const int c = ld_acquire_gpu(f.ready + blk);
       if (c >= need) {
-        f.blk = blk;
-        f.cnt = c;
+        f.cnt[blk] = c;
         break;
       }
       if (*abort) return false;
@@ -633,9 +634,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const long long gchunk0 = (long long)bh * a.gram_chunks + a.t_begin / L;  // Gram block of the round's first chunk
   GramFeed feed;
   feed.ready = a.gram_ready ? a.gram_ready + (long long)bh * a.gram_nblk : nullptr;
-  feed.per = a.gram_per_blk;
-  feed.blk = -1;
-  feed.cnt = 0;
+  feed.nblk = a.gram_nblk;
+  feed.cnt = sm.gcnt;
+  if (tid == 0)
+    for (int i = 0; i < kMaxGramBlk; ++i) sm.gcnt[i] = 0;
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
                       a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
@@ -1092,9 +1094,12 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   GramSmem<D>& sm = *reinterpret_cast<GramSmem<D>*>(smem_raw);
   const int bh = blockIdx.x, blk = blockIdx.y;
   const int b = bh / a.H, h = bh % a.H;
-  const int c_begin = a.chunk0 + blk * a.per_blk;
-  const int c_end = min(a.chunk0 + a.count, c_begin + a.per_blk);
-  if (c_begin >= c_end) return;
+  // this block's chunks: chunk0 + blk + i * nblk, i < n_mine (interleaved, so
+  // that the early chunks of every stream, which a concurrent scan needs first,
+  // come out together)
+  if (blk >= a.count) return;
+  const int n_mine = (a.count - blk + a.nblk - 1) / a.nblk;
+  auto chunk_of = [&](int i) { return a.chunk0 + blk + i * a.nblk; };
   const int row_stride = a.H * D;
   const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
   const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
@@ -1111,11 +1116,12 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  load(c_begin, 0);
-  for (int c = c_begin; c < c_end; ++c) {
-    const int st = (c - c_begin) & 1;
-    if (c + 1 < c_end) {
-      load(c + 1, st ^ 1);
+  load(chunk_of(0), 0);
+  for (int i = 0; i < n_mine; ++i) {
+    const int c = chunk_of(i);
+    const int st = i & 1;
+    if (i + 1 < n_mine) {
+      load(chunk_of(i + 1), st ^ 1);
       asm volatile("cp.async.wait_group 1;" ::: "memory");
     } else {
       asm volatile("cp.async.wait_group 0;" ::: "memory");
@@ -1141,12 +1147,12 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
       *reinterpret_cast<float4*>(out + 2 * L * L + 4 * threadIdx.x) = *reinterpret_cast<const float4*>(sm.a + 4 * threadIdx.x);
     // published after the first chunk, then every fourth and after the last
     // (the scan reads the blocks by bulk copy: async proxy)
-    const bool publish = a.ready && (((c - c_begin) & 3) == 0 || c + 1 == c_end);
+    const bool publish = a.ready && (i < 4 || (i & 3) == 3 || i + 1 == n_mine);
     if (publish) asm volatile("fence.proxy.async.global;" ::: "memory");
     __syncthreads();  // the block is written; G, Q, a are reused by the next chunk
     if (publish && threadIdx.x == 0) {
       __threadfence();
-      st_release_gpu(a.ready + (long long)bh * a.nblk + blk, c - c_begin + 1);
+      st_release_gpu(a.ready + (long long)bh * a.nblk + blk, i + 1);
     }
   }
 }
