@@ -642,6 +642,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
                       a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
                       &sm.abort_flag, a.status);
+  int rel_pending = 0;  // thread NT - 32: progress value not yet released
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
     const int Lc = min(L, a.t_end - t0);
@@ -751,8 +752,16 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     // ------------------------------------------------ 3b. the previous interval's snapshot copies (warps 1..)
     // They read the staged open state and closed slots, which only the state
     // updates and the publish below change, so they overlap warp 0's passes.
-    if constexpr (sizeof(Tpool) == 2)
+    // The progress word of the interval that ended with the last chunk goes out
+    // here too, where the wait of its release for this thread's earlier writes
+    // costs warp 0 nothing.
+    if constexpr (sizeof(Tpool) == 2) {
+      if (rel_pending > 0) {
+        st_release_gpu(a.progress + 2 * bh + rank, rel_pending);
+        rel_pending = 0;
+      }
       if (warp != 0 && sm.pend > 0) snapshot_copies(sm.pend, tid - 32, NT - 32);
+    }
     // ------------------------------------------------ 4. boundary passes (warp 0, tokens 2 lane, 2 lane + 1)
     // Each pass scores every undecided token as if the open segment ran to it,
     // takes the first that fires, and restarts the segment there.
@@ -1001,8 +1010,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         if (tid == 0) sm.pend = sm.nsnapjobs;  // copied during the next chunk's passes (or at round end)
         __syncthreads();
         // interval snap_base + snap_idx - 1 is complete: its trace is written and its
-        // starting snapshot was copied during its first chunk (a concurrent read-out waits for this)
-        if (a.progress && tid == NT - 32) st_release_gpu(a.progress + 2 * bh + rank, a.snap_base + snap_idx);
+        // starting snapshot was copied during its first chunk (a concurrent read-out
+        // waits for this); released at the start of the next chunk's copies, or by
+        // the final release below
+        if (a.progress && tid == NT - 32) rel_pending = a.snap_base + snap_idx;
       } else {  // fp32 pool (d = 64): copied now, the open state straight from the accumulators
         __syncthreads();
         for (int jj = 0; jj < sm.nsnapjobs; ++jj) {
