@@ -95,23 +95,23 @@ __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int
   return true;
 }
 
-// Next chunk's k and v rows (cp.async by every thread, zero-filled past the
-// sequence end) and its Gram block gc (one bulk copy by thread 0, completing
-// on `bar`, skipped after a failed wait for the pre-pass, which sets the abort
-// flag).  The k, v copies are waited for with cp.async.wait_group, the Gram
-// block with the mbarrier.
+// Next chunk's k and v rows (cp.async by threads i0, i0 + ni, ..., zero-filled
+// past the sequence end) and its Gram block gc (one bulk copy by thread i0,
+// completing on `bar`, skipped after a failed wait for the pre-pass, which sets
+// the abort flag).  The k, v copies are waited for with cp.async.wait_group by
+// the threads that issued them, the Gram block with the mbarrier.
 template <int D>
 __device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
                                                const __nv_bfloat16* vs, int row_stride, int valid, float* dgq,
                                                const float* gsrc, uint64_t* bar, GramFeed& feed, int gc,
-                                               volatile int* abort, int32_t* status) {
+                                               volatile int* abort, int32_t* status, int i0, int ni) {
   constexpr int RP = D + 8;
   constexpr int V16 = D / 8;
-  if (threadIdx.x == 0 && gsrc && gram_feed_wait(feed, gc, abort, status)) {
+  if (i0 == 0 && gsrc && gram_feed_wait(feed, gc, abort, status)) {
     sm100::mbar_expect_tx(bar, (uint32_t)kGramBlock * 4u);
     sm100::bulk_g2s(dgq, gsrc, (uint32_t)kGramBlock * 4u, bar);
   }
-  for (int e = threadIdx.x; e < L * V16; e += NT) {
+  for (int e = i0; e < L * V16; e += ni) {
     const int r = e / V16, c = (e % V16) * 8;
     const int nbytes = (r < valid) ? 16 : 0;
     const __nv_bfloat16* sk = (r < valid) ? ks + (long long)r * row_stride + c : ks;
@@ -641,23 +641,15 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
                       a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
-                      &sm.abort_flag, a.status);
+                      &sm.abort_flag, a.status, tid, NT);
   int rel_pending = 0;  // thread NT - 32: progress value not yet released
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
     const int Lc = min(L, a.t_end - t0);
     const int st = c & 1;
-    // ------------------------------------------------ 1. k, v of this chunk; prefetch the next
-    if (c + 1 < nchunks) {
-      const int t1 = t0 + L;
-      prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
-                        vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
-                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
-                        a.t_begin / L + c + 1, &sm.abort_flag, a.status);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
+    // ------------------------------------------------ 1. k, v of this chunk (issued during the
+    // previous chunk's passes, or before the loop)
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
     if (a.gram) sm100::mbar_wait(&sm.kvbar[st], (uint32_t)((c >> 1) & 1), &sm.abort_flag, a.status);
     if (tid < L) sm.mlog[tid] = -1;
     __syncthreads();
@@ -755,6 +747,15 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     // The progress word of the interval that ended with the last chunk goes out
     // here too, where the wait of its release for this thread's earlier writes
     // costs warp 0 nothing.
+    // The next chunk's k, v and Gram block are issued here as well (warps 1..;
+    // buffers st ^ 1, which the previous chunk used, are free).
+    if (warp != 0 && c + 1 < nchunks) {
+      const int t1 = t0 + L;
+      prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
+                        vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
+                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
+                        a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32);
+    }
     if constexpr (sizeof(Tpool) == 2) {
       if (rel_pending > 0) {
         st_release_gpu(a.progress + 2 * bh + rank, rel_pending);
