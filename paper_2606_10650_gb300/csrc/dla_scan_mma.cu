@@ -741,12 +741,14 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
     __syncthreads();
-    // ------------------------------------------------ 3b. the previous interval's snapshot copies (warps 1..)
-    // They read the staged open state and closed slots, which only the state
-    // updates and the publish below change, so they overlap warp 0's passes.
-    // The progress word of the interval that ended with the last chunk goes out
-    // here too, where the wait of its release for this thread's earlier writes
-    // costs warp 0 nothing.
+    // ------------------------------------------------ 3b. work beside warp 0's passes (warps 1..)
+    // First the progress word of the interval that ended with the last chunk:
+    // here the wait of its release for earlier memory operations costs warp 0
+    // nothing, and issued before the loads below it does not wait for them.
+    if (rel_pending > 0) {
+      st_release_gpu(a.progress + 2 * bh + rank, rel_pending);
+      rel_pending = 0;
+    }
     // The next chunk's k, v and Gram block are issued here as well (warps 1..;
     // buffers st ^ 1, which the previous chunk used, are free).
     if (warp != 0 && c + 1 < nchunks) {
@@ -756,13 +758,11 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
                         a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
                         a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32);
     }
-    if constexpr (sizeof(Tpool) == 2) {
-      if (rel_pending > 0) {
-        st_release_gpu(a.progress + 2 * bh + rank, rel_pending);
-        rel_pending = 0;
-      }
+    // Then the previous interval's snapshot copies: they read the staged open
+    // state and closed slots, which only the state updates and the publish below
+    // change.
+    if constexpr (sizeof(Tpool) == 2)
       if (warp != 0 && sm.pend > 0) snapshot_copies(sm.pend, tid - 32, NT - 32);
-    }
     // ------------------------------------------------ 4. boundary passes (warp 0, tokens 2 lane, 2 lane + 1)
     // Each pass scores every undecided token as if the open segment ran to it,
     // takes the first that fires, and restarts the segment there.
