@@ -526,7 +526,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_fail(e, "device query");
-    dla::gram_blocks(B * H, P.gram_chunks, 2 * sms, &ga.nblk, &ga.per_blk);
+    dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
     if (P.gram_chunks) {
       e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
@@ -586,7 +586,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     ga.out = (float*)(ws + P.off_gram);
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = gram_ready;
-    dla::gram_blocks(B * H, P.gram_chunks, 2 * free_sms, &ga.nblk, &ga.per_blk);
+    dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * free_sms, &ga.nblk, &ga.per_blk);
     if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
       return cuda_fail(e, "progress reset");
     if ((e = cudaEventRecord(S->prep_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
@@ -637,12 +637,12 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
       return cuda_fail(e, "device query");
     const int first = std::min(P.gram_chunks, sizes[0] * P.interval / dla::kScanL);
     ga.chunk0 = 0; ga.count = first;
-    dla::gram_blocks(B * H, ga.count, 2 * sms, &ga.nblk, &ga.per_blk);
+    dla::gram_blocks(B * H, ga.count, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
     e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     if (first < P.gram_chunks) {
       ga.chunk0 = first; ga.count = P.gram_chunks - first;
-      dla::gram_blocks(B * H, ga.count, 2 * sms, &ga.nblk, &ga.per_blk);
+      dla::gram_blocks(B * H, ga.count, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
       if ((e = cudaStreamWaitEvent(S->lo, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");

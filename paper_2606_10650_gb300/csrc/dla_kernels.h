@@ -88,6 +88,7 @@ struct GramArgs {
   int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after its first four, then every fourth), or nullptr
 };
 constexpr int kMaxGramBlk = 64;  // blocks per stream of one Gram launch, at most
+constexpr int kGramCtasPerSm = 3;  // resident Gram CTAs per SM (shared memory)
 
 // K2: read-out of one round, one CTA per (snapshot interval, stream).
 struct ReadoutArgs {
@@ -147,7 +148,7 @@ int scan_mma_ctas_per_stream(int BH, int d);
 // scan_mma_ctas_per_stream picks for BH streams) can all be resident at once.
 int scan_mma_resident_streams(int BH, int d);
 // Block count of a Gram launch over `count` chunks of BH streams whose CTAs
-// fit `slots` resident CTAs (two per SM) in one wave (at least one block per
+// fit `slots` resident CTAs (kGramCtasPerSm per SM) in one wave (at least one block per
 // stream, at most kMaxGramBlk); per_blk follows.
 void gram_blocks(int BH, int count, int slots, int* nblk, int* per_blk);
 // One CTA that returns once `n` scan CTAs have started (*started >= n), or after

@@ -1086,18 +1086,19 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
 template <int D>
 struct GramSmem {
   static constexpr int RP = D + 8;
-  __nv_bfloat16 k[2][L * RP];  // [stage] the chunk's k rows
-  __nv_bfloat16 v[2][L * RP];
+  __nv_bfloat16 k[L * RP];     // the chunk's k rows (then the next chunk's, once G is formed)
+  __nv_bfloat16 v[L * RP];
   float G[L * (L + 1)];        // G[t][s], then in place gs[s][t]
   float Q[L * (L + 1)];        // Q[j][t]
   float a[L];
 };
 
-// K0: each CTA walks the chunks of one block of one stream in order; the k, v
-// rows of the next chunk are in flight (cp.async) while it computes this one.
-// With `ready` set, the count of the block's chunks written is published
-// (release) after its first chunk, every fourth and its last, for a scan that
-// runs concurrently and reads the blocks through the async proxy.
+// K0: each CTA walks the chunks of one block of one stream in order, one k, v
+// buffer (three CTAs per SM): the next chunk's rows are in flight (cp.async)
+// while this chunk's tables are scanned and written.  With `ready` set, the
+// count of the block's chunks written is published (release) after each of its
+// first four chunks, every fourth and its last, for a scan that runs
+// concurrently and reads the blocks through the async proxy.
 template <int D>
 __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   constexpr int RP = D + 8;
@@ -1115,32 +1116,27 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   const int row_stride = a.H * D;
   const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
   const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
-  auto load = [&](int c, int st) {  // rows past the sequence end are zero-filled
+  auto load = [&](int c) {  // rows past the sequence end are zero-filled
     const int t0 = c * L, valid = min(L, a.T - t0);
     for (int e = threadIdx.x; e < L * V16; e += NT) {
       const int r = e / V16, cc = (e % V16) * 8;
       const long long off = (long long)(t0 + (r < valid ? r : 0)) * row_stride + cc;
       const int nbytes = (r < valid) ? 16 : 0;
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.k[st] + r * RP + cc)),
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.k + r * RP + cc)),
                    "l"(k0 + off), "r"(nbytes) : "memory");
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.v[st] + r * RP + cc)),
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.v + r * RP + cc)),
                    "l"(v0 + off), "r"(nbytes) : "memory");
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };
-  load(chunk_of(0), 0);
+  load(chunk_of(0));
   for (int i = 0; i < n_mine; ++i) {
     const int c = chunk_of(i);
-    const int st = i & 1;
-    if (i + 1 < n_mine) {
-      load(chunk_of(i + 1), st ^ 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncthreads();
-    gram_tile_lower<D>(sm.k[st], sm.v[st], sm.G, sm.a);
+    gram_tile_lower<D>(sm.k, sm.v, sm.G, sm.a);
     __syncthreads();
+    if (i + 1 < n_mine) load(chunk_of(i + 1));  // k, v are free: in flight during the scans below
     suffix_rows_ilp(sm.G);  // G[t][j] = gs[j][t]
     __syncthreads();
     prefix_rows_ilp(sm.G, 1, L + 1, sm.Q, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u]
