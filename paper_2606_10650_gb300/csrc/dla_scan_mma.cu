@@ -366,6 +366,16 @@ __device__ __forceinline__ void copy_state_split(__nv_bfloat16* dst, const float
     }
   }
 }
+// (x, y) as packed bf16 hi = bf16(x, y) and lo = bf16(x - hi, y - hi): the
+// open state's operand split, as the publish stores it.
+__device__ __forceinline__ void split_hi_lo(float x, float y, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  const float2 f = __bfloat1622float2(h);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x - f.x, y - f.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
 // dst += src over one D x D state, batched like copy_state_g.
 template <int D, int NR = D>
 __device__ __forceinline__ void add_state_g(float* dst, const float* src) {
@@ -430,8 +440,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   constexpr int WPM = NW / MT;        // warps per band
   constexpr int KC = D / WPM;         // state columns per warp
   constexpr int NT8 = KC / 8;         // n8 tiles per warp in the state build
-  constexpr int NJ8 = R / 8 / NW;     // n8 tiles per warp in the x GEMM
-  static_assert(NJ8 == 1 || NJ8 == 2, "x GEMM tiling");
+  static_assert(L == 64 && KC % 16 == 0, "x GEMM tiling");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   MmaSmem<D, CL>& sm = *reinterpret_cast<MmaSmem<D, CL>*>(smem_raw);
 
@@ -658,57 +667,67 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     const __nv_bfloat16* Vs = sm.kv[st][1];
     const int q = lane >> 3, r8 = lane & 7;
     // ------------------------------------------------ 2. x_t = v_t^T S_open k_t (this CTA's rows)
+    // Each warp adds sum_{j, k} v_t[j] S[j][k] k_t[k] over its band of the open
+    // state (rows j0 .. j0 + 15, columns k0 .. k0 + KC - 1): S straight from its
+    // accumulators (two m16n8 accumulator tiles are the m16n8k16 A fragment of
+    // those 16 columns) as bf16 hi + lo, k_t from the chunk's K tile, so that
+    // Y[j][t] = sum_k S[j][k] k_t[k] on mma.sync; then the v_t[j] weights.
     if (m_chunk > 0) {
-      float X[4][NJ8][4];
+      float Y[L / 8][4];
 #pragma unroll
-      for (int mt = 0; mt < 4; ++mt)
+      for (int n = 0; n < L / 8; ++n)
 #pragma unroll
-        for (int nj = 0; nj < NJ8; ++nj)
+        for (int e = 0; e < 4; ++e) Y[n][e] = 0.f;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) X[mt][nj][e] = 0.f;
-      const int jb = warp * 8 * NJ8;  // local rows of this warp
-      for (int kk = 0; kk < D; kk += 16) {
-        uint32_t bh_[4], bl_[4];
-        if constexpr (NJ8 == 2) {
-          ldsm4(bh_, &sm.S2[0][(jb + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8]);
-          ldsm4(bl_, &sm.S2[1][(jb + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8]);
-        } else {
-          ldsm2(bh_, &sm.S2[0][(jb + r8) * RP + kk + (q & 1) * 8]);
-          ldsm2(bl_, &sm.S2[1][(jb + r8) * RP + kk + (q & 1) * 8]);
-        }
+      for (int s8 = 0; s8 < KC / 16; ++s8) {
+        uint32_t ah[4], al[4];
+        split_hi_lo(acc[2 * s8][0], acc[2 * s8][1], ah[0], al[0]);          // row g, k 2tg, 2tg + 1
+        split_hi_lo(acc[2 * s8][2], acc[2 * s8][3], ah[1], al[1]);          // row g + 8
+        split_hi_lo(acc[2 * s8 + 1][0], acc[2 * s8 + 1][1], ah[2], al[2]);  // row g, k 2tg + 8, 2tg + 9
+        split_hi_lo(acc[2 * s8 + 1][2], acc[2 * s8 + 1][3], ah[3], al[3]);  // row g + 8
 #pragma unroll
-        for (int mt = 0; mt < 4; ++mt) {
-          uint32_t af[4];
-          ldsm4(af, Ks + (16 * mt + (q & 1) * 8 + r8) * RP + kk + (q >> 1) * 8);
-#pragma unroll
-          for (int nj = 0; nj < NJ8; ++nj) {
-            mma16816(X[mt][nj], af, bh_[2 * nj], bh_[2 * nj + 1]);
-            mma16816(X[mt][nj], af, bl_[2 * nj], bl_[2 * nj + 1]);
-          }
+        for (int np = 0; np < L / 16; ++np) {  // tokens 16 np .. 16 np + 15: two n8 tiles
+          uint32_t bf[4];
+          ldsm4(bf, Ks + (16 * np + (q >> 1) * 8 + r8) * RP + k0 + 16 * s8 + (q & 1) * 8);
+          mma16816(Y[2 * np], ah, bf[0], bf[1]);
+          mma16816(Y[2 * np], al, bf[0], bf[1]);
+          mma16816(Y[2 * np + 1], ah, bf[2], bf[3]);
+          mma16816(Y[2 * np + 1], al, bf[2], bf[3]);
         }
       }
-      // x partial over this warp's j rows: sum_j v_t[j] X[t][j]
+      // this thread's terms: tokens 8n + 2tg (+1) of rows jg0 + g and jg0 + g + 8
+      float pv[L / 4];  // [2n + e]: token 8n + 2tg + e
+      const int ja = jg0 + g, jb = ja + 8;
 #pragma unroll
-      for (int mt = 0; mt < 4; ++mt) {
-        float p0 = 0.f, p1 = 0.f;  // rows g and g + 8 of the tile
-#pragma unroll
-        for (int nj = 0; nj < NJ8; ++nj) {
-          const int j = rbase + jb + 8 * nj + 2 * tg;
-          const int ta = 16 * mt + g, tb8 = ta + 8;
-          const float2 va = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Vs + ta * RP + j));
-          const float2 vb = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Vs + tb8 * RP + j));
-          p0 += X[mt][nj][0] * va.x + X[mt][nj][1] * va.y;
-          p1 += X[mt][nj][2] * vb.x + X[mt][nj][3] * vb.y;
-        }
-        p0 += __shfl_xor_sync(0xffffffffu, p0, 1);
-        p0 += __shfl_xor_sync(0xffffffffu, p0, 2);
-        p1 += __shfl_xor_sync(0xffffffffu, p1, 1);
-        p1 += __shfl_xor_sync(0xffffffffu, p1, 2);
-        if (tg == 0) {
-          sm.red[warp][16 * mt + g] = p0;
-          sm.red[warp][16 * mt + g + 8] = p1;
-        }
+      for (int n = 0; n < L / 8; ++n) {
+        const int t = 8 * n + 2 * tg;
+        pv[2 * n] = Y[n][0] * __bfloat162float(Vs[t * RP + ja]) + Y[n][2] * __bfloat162float(Vs[t * RP + jb]);
+        pv[2 * n + 1] =
+            Y[n][1] * __bfloat162float(Vs[(t + 1) * RP + ja]) + Y[n][3] * __bfloat162float(Vs[(t + 1) * RP + jb]);
       }
+      // sum over the eight lanes of equal tg (g = 0 .. 7) by halving exchanges
+      // (lane bits 4, 3, 2 = bits 2, 1, 0 of g): afterwards lane (g, tg) holds
+      // tokens 8g + 2tg and 8g + 2tg + 1 in pv[0], pv[1]
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const bool up = (g & 4) != 0;
+        const float send = up ? pv[k] : pv[8 + k], keep = up ? pv[8 + k] : pv[k];
+        pv[k] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const bool up = (g & 2) != 0;
+        const float send = up ? pv[k] : pv[4 + k], keep = up ? pv[4 + k] : pv[k];
+        pv[k] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+      }
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const bool up = (g & 1) != 0;
+        const float send = up ? pv[k] : pv[2 + k], keep = up ? pv[2 + k] : pv[k];
+        pv[k] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+      }
+      sm.red[warp][8 * g + 2 * tg] = pv[0];
+      sm.red[warp][8 * g + 2 * tg + 1] = pv[1];
     }
     // ------------------------------------------------ 3. Gram suffix table and a_t
     // Normally prefetched from the Gram pre-pass; formed here when the call has
