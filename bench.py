@@ -299,24 +299,26 @@ def bench_prefill(args, dist, pk):
     if roof is not None:
         roof["dominance"] = ("largest SM-time per step (ms alone x SMs occupied): " +
                              ", ".join(f"{k} {v:.1f} SM-ms" for k, v in sm_ms.items()))
-    # end to end through the public API with host buffers
+    # end to end through the C ABI with host buffers: every step, dla_forward_host
+    # copies q, k, v, lambda in from page-locked host memory (piece by piece beside
+    # the scan on the concurrent schedule), runs the forward pass and copies o back
     e2e = None
     if not args.no_e2e:
         qh, kh, vh = (x.cpu().pin_memory() for x in (qt, kt, vt))
         lh = lt.cpu().pin_memory()
         oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
         n_e2e = max(2, min(args.steps, 10))
+        hnb = dla.dla_forward_host_workspace(p, B, T, H, d, d, in_code, True)
+        hbuf = torch.empty(hnb + 256, dtype=torch.uint8, device=dev)
+        hws = (hbuf, (hbuf.data_ptr() + 255) // 256 * 256, hnb)
 
         def e2e_step():
-            qt.copy_(qh, non_blocking=True)
-            kt.copy_(kh, non_blocking=True)
-            vt.copy_(vh, non_blocking=True)
-            lt.copy_(lh, non_blocking=True)
-            step()
-            oh.copy_(o, non_blocking=True)
+            dla.dla_forward_host(p, qh, kh, vh, lh, oh, cache, bnd, ml, workspace=hws, stream=stream)
 
         e2e_step()
         torch.cuda.synchronize()
+        if dla.workspace_status(hws) != 0:
+            raise RuntimeError("dla_forward_host: device status word reports a failure")
         dist.barrier()
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a0.record(stream)
@@ -327,7 +329,9 @@ def bench_prefill(args, dist, pk):
         e_ms = dist.reduce(a0.elapsed_time(a1) / n_e2e, "max")
         hb = sum(x.numel() * x.element_size() for x in (qh, kh, vh, lh))
         e2e = {"value": round(dist.world * tokens / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
-               "h2d_bytes_per_step": hb, "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e}
+               "h2d_bytes_per_step": hb, "d2h_bytes_per_step": oh.numel() * oh.element_size(), "steps": n_e2e,
+               "call": "dla_forward_host (C ABI, page-locked host buffers in and out)"}
+        del hbuf, hws
     res = {"value": dist.world * tokens / (ms_max * 1e-3), "ms_per_step": ms_max, "tokens_per_step": tokens,
            "roofline": roof, "rooflines": rooflines, "kernels": kt_tab,
            "kernels_alone": kernel_table(solo, solo_steps) if solo else None, "tc_path": tc_path, "clocks": clk,

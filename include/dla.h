@@ -178,6 +178,35 @@ dla_status dla_forward_noalloc(const dla_params* p, dla_dtype in_dtype, int B, i
                                const float* lam, void* o, const dla_cache* cache,
                                uint8_t* boundary, int32_t* merge_log, void* stream);
 
+/* Workspace bytes dla_forward_host needs for these sizes: device buffers for
+ * q, k, v, lambda and o plus dla_forward_workspace(...).  0 for bad arguments. */
+size_t dla_forward_host_workspace(const dla_params* p, int B, int T, int H, int dk, int dv,
+                                  dla_dtype in_dtype, int with_output);
+
+/* dla_forward with q, k, v, lam and o in HOST memory (same layouts and
+ * semantics; the paper has no counterpart: this is the end-to-end call of a
+ * caller whose tensors live on the host).  Page-locked host memory
+ * (cudaHostAlloc / cudaHostRegister) makes the copies asynchronous; with
+ * pageable memory they still work but do not overlap anything.
+ *   cache, boundary, merge_log: device memory, as in dla_forward.
+ *   workspace: device memory of ws_bytes >= dla_forward_host_workspace(...)
+ *   (256-byte aligned); the input and output buffers are carved from its end,
+ *   the rest is dla_forward's workspace (its status word first).
+ * On the concurrent schedule (see dla_forward) the inputs are copied in 16
+ * pieces of whole 64-token chunks on an internal stream, each piece followed
+ * by a stream memory write of the count of pieces in place; the scan waits
+ * (bounded) for the piece of every chunk it loads and forms its Gram entries
+ * itself, the read-out follows the scan, so the copies overlap the work.  On
+ * the other schedules the inputs are copied first.  o is copied back on
+ * `stream` after the read-out.  The call only enqueues work: the host buffers
+ * must stay valid, and o is filled, once `stream` has completed it.  Results
+ * equal dla_forward's on the same inputs (decisions bit-identical; the
+ * outputs to rounding of the Gram sums). */
+dla_status dla_forward_host(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
+                            int dv, const void* q, const void* k, const void* v, const float* lam,
+                            void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
+                            void* workspace, size_t ws_bytes, void* stream);
+
 /* One recurrent step (Sec. 3.1 inference rule + Algorithm 2 + read-out) for
  * every stream: token (q, k, v) [B, H, d] against the persistent cache, which
  * is updated in place.  lam [B, H, C] fp32 or NULL; o [B, H, d] (out_dtype);

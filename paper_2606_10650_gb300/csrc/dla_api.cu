@@ -3,6 +3,7 @@
 // Host logic only: argument checks, workspace layout, the round schedule of
 // the forward pass and the kernel launches.  Every compute step runs in the
 // kernels of dla_scan.cu / dla_readout_*.cu / dla_decode.cu.
+#include <cuda.h>
 #include <math.h>
 #include <algorithm>
 #include <mutex>
@@ -119,10 +120,11 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramBlock floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
-  // scan progress per (stream, CTA) and the count of started scan CTAs (concurrent read-out)
-  // and the Gram pre-pass's per-block chunk counters (a pre-pass running beside the scan)
+  // scan progress per (stream, CTA), the count of started scan CTAs (concurrent read-out),
+  // the count of input pieces streamed in by the host, and the Gram pre-pass's per-block
+  // chunk counters (a pre-pass running beside the scan)
   P.off_progress = off;
-  if (with_output) off = align256(off + (2 * BH + 1 + BH * dla::kMaxGramBlk) * sizeof(int32_t));
+  if (with_output) off = align256(off + (2 * BH + 2 + BH * dla::kMaxGramBlk) * sizeof(int32_t));
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
@@ -178,6 +180,7 @@ Schedule schedule() {
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
 constexpr int kMinFreeSms = 8;    // SMs the scan must leave free for the concurrent schedule
+constexpr int kInputPieces = 16;  // pieces of inputs streamed in from host memory (dla_forward_host)
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
 
 dla_status check_params(const dla_params* p) {
@@ -217,8 +220,9 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
 // a low-priority one, so the scan's few CTAs get SMs first.
 struct StreamSet {
   cudaStream_t hi = nullptr, lo = nullptr;  // scan, read-out
+  cudaStream_t cp = nullptr;                // host-to-device copies of streamed inputs
   cudaEvent_t in = nullptr, gram_done = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
-  cudaEvent_t prep_done = nullptr;
+  cudaEvent_t prep_done = nullptr, cp_done = nullptr;
   bool ready = false;
 };
 constexpr int kMaxDev = 64;
@@ -235,6 +239,8 @@ cudaError_t stream_set(StreamSet** out) {
     if ((e = cudaDeviceGetStreamPriorityRange(&least, &greatest)) != cudaSuccess) return e;
     if ((e = cudaStreamCreateWithPriority(&S.hi, cudaStreamNonBlocking, greatest)) != cudaSuccess) return e;
     if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
+    if ((e = cudaStreamCreateWithFlags(&S.cp, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&S.cp_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.gram_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.prep_done, cudaEventDisableTiming)) != cudaSuccess) return e;
@@ -246,6 +252,56 @@ cudaError_t stream_set(StreamSet** out) {
   }
   *out = &S;
   return cudaSuccess;
+}
+
+// ---- inputs in host memory (dla_forward_host)
+// A 32-bit write to device memory in stream order, after the stream's earlier
+// work and with a memory barrier before it (the driver's stream memory
+// operation: no kernel, so it needs no SM while kernels wait for it).
+typedef CUresult (*WriteValue32Fn)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
+WriteValue32Fn write_value_fn() {
+  static WriteValue32Fn fn = nullptr;
+  static bool tried = false;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> g(mu);
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue32", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<WriteValue32Fn>(p);
+  }
+  return fn;
+}
+
+// q, k, v, lambda in host memory and their device copies in the workspace.
+struct HostIO {
+  const void* qh;
+  const void* kh;
+  const void* vh;
+  const float* lamh;
+  void* qd;
+  void* kd;
+  void* vd;
+  float* lamd;
+  size_t elt;  // bytes per q, k, v element
+};
+// Tokens [t0, t1) of every batch row of k, v, q and lambda to the device, on stream s.
+cudaError_t h2d_tokens(const HostIO& io, int B, int T, int H, int d, int C, int t0, int t1, cudaStream_t s) {
+  cudaError_t e = cudaSuccess;
+  for (int b = 0; b < B && e == cudaSuccess; ++b) {
+    const size_t off = ((size_t)b * T + t0) * H * d * io.elt, n = (size_t)(t1 - t0) * H * d * io.elt;
+    const void* src[3] = {io.kh, io.vh, io.qh};
+    void* dst[3] = {io.kd, io.vd, io.qd};
+    for (int i = 0; i < 3 && e == cudaSuccess; ++i)
+      if (src[i]) e = cudaMemcpyAsync((char*)dst[i] + off, (const char*)src[i] + off, n, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && io.lamh) {
+      const size_t lo = ((size_t)b * T + t0) * H * C, ln = (size_t)(t1 - t0) * H * C;
+      e = cudaMemcpyAsync(io.lamd + lo, io.lamh + lo, ln * sizeof(float), cudaMemcpyHostToDevice, s);
+    }
+  }
+  return e;
 }
 
 // ---- optional per-launch CUDA-event timing (dla_timing_enable / _read)
@@ -419,9 +475,24 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
   return plan_for(1, false, p, B, T, H, dk, in_dtype, with_output != 0, true, true).total;
 }
 
-dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv, const void* q,
-                       const void* k, const void* v, const float* lam, void* o, const dla_cache* cache,
-                       uint8_t* boundary, int32_t* merge_log, void* workspace, size_t ws_bytes, void* stream) {
+// SMs the scan leaves to the rest on the concurrent schedule when all its CTAs
+// are resident (0: they are not)
+static int concurrent_free_sms(int B, int H, int d, cudaError_t* err) {
+  int dev = 0, sms = 0;
+  if ((*err = cudaGetDevice(&dev)) != cudaSuccess ||
+      (*err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+    return 0;
+  const int BH = B * H;
+  return (dla::scan_mma_resident_streams(BH, d) >= BH) ? sms - BH * dla::scan_mma_ctas_per_stream(BH, d) : 0;
+}
+
+// dla_forward; with io, q, k, v and lambda come from host memory into the
+// device buffers q, k, v, lam (workspace), streamed beside the scan on the
+// concurrent schedule, otherwise copied before anything else.
+static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
+                               const void* q, const void* k, const void* v, const float* lam, void* o,
+                               const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
+                               size_t ws_bytes, void* stream, const HostIO* io) {
   dla_status s = check_params(p);
   if (s != DLA_OK) return s;
   if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
@@ -452,6 +523,17 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   cudaStream_t st = (cudaStream_t)stream;
   char* ws = (char*)workspace;
   int32_t* status = (int32_t*)(ws + P.off_status);
+  bool stream_in = false;  // inputs from host memory streamed beside the scan
+  if (io) {
+    cudaError_t qe = cudaSuccess;
+    stream_in = with_output && use_tc(in_dtype, d) && P.persistent && (P.nsnap_total + 1) / 2 <= 65535 &&
+                schedule() == kConcurrent && concurrent_free_sms(B, H, d, &qe) >= kMinFreeSms && write_value_fn();
+    if (qe != cudaSuccess) return cuda_fail(qe, "device query");
+    if (!stream_in) {
+      const cudaError_t ce = h2d_tokens(*io, B, T, H, d, C, 0, T, st);
+      if (ce != cudaSuccess) return cuda_fail(ce, "input copy");
+    }
+  }
   uint8_t* bnd = boundary ? boundary : (uint8_t*)(ws + P.off_bnd);
   int32_t* mlog = merge_log ? merge_log : (int32_t*)(ws + P.off_mlog);
   dla_cache live;
@@ -548,11 +630,8 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   }
   int free_sms = 0;  // SMs the scan leaves to the rest when all its CTAs are resident (0: they are not)
   if (one_readout && sched == kConcurrent) {
-    int dev = 0, sms = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
-      return cuda_fail(e, "device query");
-    const int BH = B * H;
-    if (dla::scan_mma_resident_streams(BH, d) >= BH) free_sms = sms - BH * dla::scan_mma_ctas_per_stream(BH, d);
+    free_sms = concurrent_free_sms(B, H, d, &e);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
   }
   if (free_sms >= kMinFreeSms) {
     // One scan over the whole sequence (high-priority stream) and the read-out
@@ -579,7 +658,11 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     }
     int32_t* progress = (int32_t*)(ws + P.off_progress);
     int32_t* started = progress + 2 * B * H;
-    int32_t* gram_ready = started + 1;
+    int32_t* pieces = started + 1;  // input pieces streamed in so far
+    int32_t* gram_ready = started + 2;
+    // with streamed inputs the scan forms its Gram entries itself: a pre-pass
+    // waiting for the pieces would hold back the read-out behind it
+    const bool run_gram = P.gram_chunks && !stream_in;
     const int ctas = dla::scan_mma_ctas_per_stream(B * H, d);
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
@@ -587,7 +670,7 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = gram_ready;
     dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * free_sms, &ga.nblk, &ga.per_blk);
-    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 1 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
+    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 2 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
       return cuda_fail(e, "progress reset");
     if ((e = cudaEventRecord(S->prep_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(S->lo, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
@@ -596,15 +679,38 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
     sa.carry_in = 0; sa.snap_at_end = 0;
     sa.progress = progress; sa.started = started;
-    if (P.gram_chunks) {
+    if (run_gram) {
       sa.gram_ready = gram_ready;
       sa.gram_nblk = ga.nblk;
+    } else {
+      sa.gram = nullptr;
+    }
+    // Streamed inputs: pieces of pc chunks on the copy stream, each followed by
+    // the count of pieces in place (a stream memory write); the scan waits for
+    // the piece of each chunk it loads, the read-out for the scan.
+    int pc = 0, npiece = 0;
+    auto put_piece = [&](int pi) -> dla_status {
+      const int t0 = pi * pc * dla::kScanL, t1 = std::min(T, (pi + 1) * pc * dla::kScanL);
+      const cudaError_t ce = h2d_tokens(*io, B, T, H, d, C, t0, t1, S->cp);
+      if (ce != cudaSuccess) return cuda_fail(ce, "input copy");
+      if (write_value_fn()((CUstream)S->cp, (CUdeviceptr)pieces, (cuuint32_t)(pi + 1), 0) != CUDA_SUCCESS)
+        return fail(DLA_ERR_CUDA, "stream memory write failed");
+      return DLA_OK;
+    };
+    if (stream_in) {
+      const int nch = (T + dla::kScanL - 1) / dla::kScanL;
+      pc = std::max(1, (nch + kInputPieces - 1) / kInputPieces);
+      npiece = (nch + pc - 1) / pc;
+      sa.piece_ready = pieces;
+      sa.piece_chunks = pc;
+      if ((e = cudaStreamWaitEvent(S->cp, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+      if ((s = put_piece(0)) != DLA_OK) return s;
     }
     e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     e = timed(DLA_K_GATE, S->lo, [&] { return dla::launch_gate(started, B * H * ctas, status, S->lo); });
     if (e != cudaSuccess) return cuda_fail(e, "gate launch");
-    if (P.gram_chunks) {  // K0 beside the scan, on the SMs it leaves free
+    if (run_gram) {  // K0 beside the scan, on the SMs it leaves free
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     }
@@ -617,6 +723,12 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
     ra.nsnap = P.nsnap_total; ra.snap_base = 0;
     e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+    if (stream_in) {
+      for (int pi = 1; pi < npiece; ++pi)
+        if ((s = put_piece(pi)) != DLA_OK) return s;
+      if ((e = cudaEventRecord(S->cp_done, S->cp)) != cudaSuccess) return cuda_fail(e, "event record");
+      if ((e = cudaStreamWaitEvent(st, S->cp_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+    }
     if ((e = cudaEventRecord(S->scan_done[0], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaEventRecord(S->ro_done[0], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
@@ -687,6 +799,81 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
   if ((e = cudaStreamWaitEvent(st, S->scan_done[0], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
   for (int i = 0; i < 2; ++i)
     if (used[i] && (e = cudaStreamWaitEvent(st, S->ro_done[i], 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  return ok();
+}
+
+dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv, const void* q,
+                       const void* k, const void* v, const float* lam, void* o, const dla_cache* cache,
+                       uint8_t* boundary, int32_t* merge_log, void* workspace, size_t ws_bytes, void* stream) {
+  return forward_impl(p, in_dtype, B, T, H, dk, dv, q, k, v, lam, o, cache, boundary, merge_log, workspace, ws_bytes,
+                      stream, nullptr);
+}
+
+// Device buffers of dla_forward_host at the end of its workspace: q, k, v,
+// lambda, o (each 256-byte aligned); the forward pass's workspace before them.
+struct HostBuffers {
+  size_t q, k, v, lam, o, total;
+};
+static HostBuffers host_buffers(const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype, int with_output) {
+  HostBuffers hb;
+  const size_t n = (size_t)B * T * H * d, elt = (in_dtype == DLA_BF16) ? 2 : 4;
+  const size_t oelt = (p->out_dtype == DLA_BF16) ? 2 : 4;
+  size_t off = 0;
+  hb.k = off;   off = align256(off + n * elt);
+  hb.v = off;   off = align256(off + n * elt);
+  hb.q = off;   if (with_output) off = align256(off + n * elt);
+  hb.lam = off; if (with_output) off = align256(off + (size_t)B * T * H * p->capacity * sizeof(float));
+  hb.o = off;   if (with_output) off = align256(off + n * oelt);
+  hb.total = off;
+  return hb;
+}
+
+size_t dla_forward_host_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype,
+                                  int with_output) {
+  if (check_params(p) != DLA_OK || check_shape(dk, dv) != DLA_OK || B < 1 || T < 1 || H < 1) return 0;
+  return host_buffers(p, B, T, H, dk, in_dtype, with_output).total +
+         dla_forward_workspace(p, B, T, H, dk, dv, in_dtype, with_output);
+}
+
+dla_status dla_forward_host(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
+                            const void* q, const void* k, const void* v, const float* lam, void* o,
+                            const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
+                            size_t ws_bytes, void* stream) {
+  dla_status s = check_params(p);
+  if (s != DLA_OK) return s;
+  if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
+  if (B < 1 || T < 1 || H < 1) return fail(DLA_ERR_INVALID_ARG, "B, T, H must be >= 1");
+  if ((s = check_shape(dk, dv)) != DLA_OK) return s;
+  if (!k || !v) return fail(DLA_ERR_INVALID_ARG, "k and v must be non-NULL");
+  if (o && !q) return fail(DLA_ERR_INVALID_ARG, "q must be non-NULL when o is requested");
+  if (!workspace) return fail(DLA_ERR_WORKSPACE, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(DLA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const int d = dk;
+  const bool with_output = (o != nullptr);
+  const HostBuffers hb = host_buffers(p, B, T, H, d, in_dtype, with_output);
+  if (ws_bytes < hb.total) return fail(DLA_ERR_WORKSPACE, "workspace has %zu bytes, needs more than %zu", ws_bytes, hb.total);
+  const size_t fw_bytes = (ws_bytes - hb.total) & ~(size_t)255;  // the forward pass's part, before the buffers
+  char* bufs = (char*)workspace + fw_bytes;
+  HostIO io;
+  io.qh = with_output ? q : nullptr;
+  io.kh = k;
+  io.vh = v;
+  io.lamh = with_output ? lam : nullptr;
+  io.qd = bufs + hb.q;
+  io.kd = bufs + hb.k;
+  io.vd = bufs + hb.v;
+  io.lamd = (float*)(bufs + hb.lam);
+  io.elt = (in_dtype == DLA_BF16) ? 2 : 4;
+  void* od = with_output ? bufs + hb.o : nullptr;
+  s = forward_impl(p, in_dtype, B, T, H, dk, dv, with_output ? io.qd : nullptr, io.kd, io.vd,
+                   (with_output && lam) ? io.lamd : nullptr, od, cache, boundary, merge_log, workspace, fw_bytes,
+                   stream, &io);
+  if (s != DLA_OK) return s;
+  if (with_output) {
+    const size_t ob = (size_t)B * T * H * d * ((p->out_dtype == DLA_BF16) ? 2 : 4);
+    const cudaError_t e = cudaMemcpyAsync(o, od, ob, cudaMemcpyDeviceToHost, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "output copy");
+  }
   return ok();
 }
 

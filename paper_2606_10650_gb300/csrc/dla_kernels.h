@@ -65,6 +65,11 @@ struct ScanArgs {
   // b + gram_nblk, ..., written in that order)
   const int32_t* gram_ready;
   int gram_nblk;
+  // Inputs streamed in by the host (nullptr: resident before the launch): the
+  // count of pieces of piece_chunks 64-token chunks whose k, v (and q, lambda)
+  // rows have arrived, written in stream order after each piece's copies
+  const int32_t* piece_ready;
+  int piece_chunks;
   int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
   int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)

@@ -169,6 +169,9 @@ __global__ void __launch_bounds__(NT, 1)
   const bool hasB = (sA + 1) < a.nsnap;
   // with a scan running concurrently: both intervals of the pair must be complete
   wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + sA + (hasB ? 2 : 1), a.status);
+  // thread 0 issues the TMA loads: they read what the scan wrote (pool entries)
+  // and the inputs streamed in before its progress
+  if (tid == 0 && a.progress) asm volatile("fence.proxy.async.global;" ::: "memory");
   __syncthreads();
   // interval A (side 0) and B (side 1) of the pair
   const int c0A = a.t_begin + sA * L, c0B = c0A + L;
@@ -401,12 +404,13 @@ __global__ void __launch_bounds__(NT, 1)
       sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");
+    // lambda through L2 (__ldcg): inputs streamed in by the host arrive while this kernel runs
     const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
     const int evt_t = sm.side[side].evt[t];
     // an interval without boundary events (the common case) weights every
     // column s <= t of row t by lambda of the open entry: loaded ahead of P
     const bool no_ev = sm.side[side].evt[L - 1] == 0;  // warp-uniform
-    const float w_open = (no_ev && t < Lcs) ? (lam_t ? __ldg(lam_t + sm.tab[side][0]) : 1.f) : 0.f;
+    const float w_open = (no_ev && t < Lcs) ? (lam_t ? __ldcg(lam_t + sm.tab[side][0]) : 1.f) : 0.f;
     bool ok;
     {  // P (accumulator 0) -> Pt over this interval's K tile (its MMAs are complete)
       ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[0], 0, abort, status));
@@ -440,7 +444,7 @@ __global__ void __launch_bounds__(NT, 1)
                   const int e = evs[ss];
                   if (e != last_e) {
                     last_e = e;
-                    last_w = lam_t ? __ldg(lam_t + trow[e]) : 1.f;
+                    last_w = lam_t ? __ldcg(lam_t + trow[e]) : 1.f;
                   }
                   wt = last_w;
                 }
@@ -491,7 +495,7 @@ __global__ void __launch_bounds__(NT, 1)
         if (x >= nu || t >= Lcs) return 0.f;
         const int xi = ux[x];
         if (xi < 0) return 0.f;
-        return lam_t ? lam_t[tab_t[xi]] : 1.f;
+        return lam_t ? __ldcg(lam_t + tab_t[xi]) : 1.f;
       };
       float wn = weight(0);
       for (int x = 0; ok && x < nu; ++x) {

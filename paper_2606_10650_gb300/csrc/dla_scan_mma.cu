@@ -100,13 +100,28 @@ __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int
 // completing on `bar`, skipped after a failed wait for the pre-pass, which sets
 // the abort flag).  The k, v copies are waited for with cp.async.wait_group by
 // the threads that issued them, the Gram block with the mbarrier.
+// With inputs streamed in by the host (piece_ready non-null), every issuing
+// thread first waits (acquire, bounded) until the piece holding the chunk has
+// arrived: piece_need pieces, the count last read kept in piece_known.
 template <int D>
 __device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16* dv, const __nv_bfloat16* ks,
                                                const __nv_bfloat16* vs, int row_stride, int valid, float* dgq,
                                                const float* gsrc, uint64_t* bar, GramFeed& feed, int gc,
-                                               volatile int* abort, int32_t* status, int i0, int ni) {
+                                               volatile int* abort, int32_t* status, int i0, int ni,
+                                               const int32_t* piece_ready, int piece_need, int& piece_known) {
   constexpr int RP = D + 8;
   constexpr int V16 = D / 8;
+  if (piece_ready && piece_known < piece_need) {
+    const long long t0 = clock64();
+    while ((piece_known = ld_acquire_gpu(piece_ready)) < piece_need) {
+      if (*abort) break;
+      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::kWaitCycles) {
+        *abort = 1;
+        atomicCAS(status, 0, sm100::kStatusTimeout);
+        break;
+      }
+    }
+  }
   if (i0 == 0 && gsrc && gram_feed_wait(feed, gc, abort, status)) {
     sm100::mbar_expect_tx(bar, (uint32_t)kGramBlock * 4u);
     sm100::bulk_g2s(dgq, gsrc, (uint32_t)kGramBlock * 4u, bar);
@@ -645,12 +660,14 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   feed.ready = a.gram_ready ? a.gram_ready + (long long)bh * a.gram_nblk : nullptr;
   feed.nblk = a.gram_nblk;
   feed.cnt = sm.gcnt;
+  int piece_known = 0;  // streamed inputs: pieces known to have arrived (this thread)
   if (tid == 0)
     for (int i = 0; i < kMaxGramBlk; ++i) sm.gcnt[i] = 0;
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
                       a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
-                      &sm.abort_flag, a.status, tid, NT);
+                      &sm.abort_flag, a.status, tid, NT, a.piece_ready,
+                      a.piece_chunks ? a.t_begin / L / a.piece_chunks + 1 : 0, piece_known);
   int rel_pending = 0;  // thread NT - 32: progress value not yet released
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
@@ -775,7 +792,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
                         vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
                         a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
-                        a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32);
+                        a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32, a.piece_ready,
+                        a.piece_chunks ? (a.t_begin / L + c + 1) / a.piece_chunks + 1 : 0, piece_known);
     }
     // Then the previous interval's snapshot copies: they read the staged open
     // state and closed slots, which only the state updates and the publish below

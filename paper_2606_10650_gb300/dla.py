@@ -21,7 +21,8 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
-            "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc"]
+            "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc",
+            "dla_forward_host_workspace", "dla_forward_host"]
 KERNELS = ["scan", "readout", "decode", "init", "gram", "gate"]
 
 
@@ -72,6 +73,9 @@ def lib():
         L.dla_status_string.argtypes = [ci]
         L.dla_version.restype = ci
         L.dla_forward_noalloc.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp]
+        L.dla_forward_host_workspace.restype = sz
+        L.dla_forward_host_workspace.argtypes = [P, ci, ci, ci, ci, ci, ci, ci]
+        L.dla_forward_host.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp, sz, vp]
         L.dla_timing_enable.argtypes = [ci]
         L.dla_timing_read.argtypes = [ctypes.POINTER(ci), ctypes.POINTER(ctypes.c_double), ci]
         _LIB = L
@@ -132,6 +136,10 @@ def dla_cache_bytes(B, H, C, dk, dv):
 
 def dla_forward_workspace(params, B, T, H, dk, dv, in_dtype, with_output=True):
     return lib().dla_forward_workspace(ctypes.byref(params), B, T, H, dk, dv, in_dtype, int(bool(with_output)))
+
+
+def dla_forward_host_workspace(params, B, T, H, dk, dv, in_dtype, with_output=True):
+    return lib().dla_forward_host_workspace(ctypes.byref(params), B, T, H, dk, dv, in_dtype, int(bool(with_output)))
 
 
 def dla_forward_min_workspace(params, B, T, H, dk, dv, in_dtype, with_output=True):
@@ -239,6 +247,31 @@ def dla_forward_noalloc(params, q, k, v, lam=None, o=None, cache=None, boundary=
                                    _ptr(lam), _ptr(o), ctypes.byref(cache.c) if cache is not None else None,
                                    _ptr(boundary), _ptr(merge_log), _stream(stream))
     _check(st)
+
+
+def dla_forward_host(params, q, k, v, lam=None, o=None, cache=None, boundary=None, merge_log=None,
+                     workspace=None, device=None, stream=None):
+    """Raw call of dla_forward_host: q, k, v, lam, o are contiguous CPU tensors
+    (page-locked for asynchronous copies), same shapes and dtypes as for
+    dla_forward; cache, boundary, merge_log are device tensors or None;
+    workspace: (tensor, base_ptr, nbytes) on `device` or None (allocated here).
+    Only enqueues: o is filled once the stream has run the call."""
+    B, T, H, d = k.shape
+    dt = _dtype_code(k)
+    for t in (q, k, v, lam, o):
+        if t is not None and (not t.is_contiguous() or t.is_cuda):
+            raise ValueError("q, k, v, lam, o must be contiguous host tensors")
+    if workspace is None:
+        dev = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
+        nb = dla_forward_host_workspace(params, B, T, H, d, d, dt, o is not None)
+        buf, base = _aligned_workspace(nb, dev)
+        workspace = (buf, base, nb)
+    _, base, nb = workspace
+    st = lib().dla_forward_host(ctypes.byref(params), dt, B, T, H, d, d, _ptr(q), _ptr(k), _ptr(v), _ptr(lam),
+                                _ptr(o), ctypes.byref(cache.c) if cache is not None else None, _ptr(boundary),
+                                _ptr(merge_log), ctypes.c_void_p(base), nb, _stream(stream))
+    _check(st)
+    return workspace
 
 
 def workspace_status(workspace):

@@ -78,3 +78,20 @@ def test_cache_carve_layout(L):
     assert c.states == 1 << 30 and c.C == 4
     assert all(getattr(c, f) % 256 == 0 for f in ("states", "slot", "n", "ibar", "m"))
     assert L.dla_cache_carve(_fake(1 << 30), nb - 1, 2, 3, 4, 64, 64, ctypes.byref(c)) == 3
+
+
+def test_host_buffer_entry_point_errors_and_workspace(L):
+    p = dla.make_params(0.6, 32)
+    fw = L.dla_forward_workspace(ctypes.byref(p), 2, 16384, 16, 128, 128, 0, 1)
+    hw = L.dla_forward_host_workspace(ctypes.byref(p), 2, 16384, 16, 128, 128, 0, 1)
+    io = 4 * 2 * 16384 * 16 * 128 * 2 + 2 * 16384 * 16 * 32 * 4  # q, k, v (bf16), o (fp32), lambda
+    assert hw >= fw + io
+    assert L.dla_forward_host_workspace(ctypes.byref(p), 0, 16, 1, 128, 128, 0, 1) == 0
+
+    def fh(k=True, ws=True, ws_bytes=1 << 40):
+        return L.dla_forward_host(ctypes.byref(p), 0, 1, 64, 2, 128, 128, _fake(), _fake() if k else None, _fake(),
+                                  None, _fake(), None, None, None, _fake(1 << 24) if ws else None, ws_bytes, None)
+    assert fh(k=False) == 1
+    assert fh(ws=False) == 3
+    assert fh(ws_bytes=1024) == 3
+    assert b"workspace" in L.dla_last_error()

@@ -216,3 +216,32 @@ def test_concurrent_schedule_first_call_of_a_process():
     out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
     assert out.returncode == 0, out.stderr[-2000:]
     assert "STATUS 0" in out.stdout, out.stdout[-2000:]
+
+
+@pytest.mark.parametrize("sched", ["concurrent", "rounds"])
+@pytest.mark.parametrize("case", ["regime_bf16", "standard_bf16", "d128_fp32"])
+def test_forward_host_buffers(case, sched, monkeypatch):
+    """dla_forward_host: q, k, v, lambda and o in page-locked host memory.  On
+    the concurrent schedule (bf16, d = 128) the inputs stream in piece by piece
+    beside the scan, which forms its Gram entries itself; elsewhere they are
+    copied first.  The oracle's results either way."""
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
+    name, ov = CASES[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    qt, kt, vt, lt = upload(w, q, k, v, lam)
+    qh, kh, vh, lh = (x.cpu().pin_memory() for x in (qt, kt, vt, lt))
+    B, T, H, d = kh.shape
+    dev = torch.device("cuda:0")
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    oh = torch.full((B, T, H, d), float("nan"), dtype=torch.float32).pin_memory()
+    bnd = torch.full((B, H, T), 7, dtype=torch.uint8, device=dev)
+    ml = torch.full((B, H, T), -7, dtype=torch.int32, device=dev)
+    ws = dla.dla_forward_host(p, qh, kh, vh, lh, oh, cache, bnd, ml, device=dev)
+    torch.cuda.synchronize()
+    assert dla.workspace_status(ws) == 0, "device status word reports a failure"
+    g = dict(o=oh.double().numpy(), boundary=bnd.cpu().numpy(), merge_log=ml.cpu().numpy(), cache=cache)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+    structural_checks(w, g, w.T)
