@@ -68,6 +68,9 @@ int readout_interval(dla_dtype in_dtype, int d) {
 // sequence, so rounds continue it and a scan never waits for a read-out.
 // Reset mode (small workspaces): each round restarts a pool of its own, two
 // pools alternate, and a round copies the live states into its pool first.
+constexpr int kInputPieces = 16;  // pieces of inputs streamed in from host memory (dla_forward_host)
+constexpr int kOutPieces = 16;    // pieces of the output copied back while the read-out runs
+
 struct FwdPlan {
   int interval;      // tokens per snapshot interval
   int nsnap_total;   // intervals over the whole sequence
@@ -124,7 +127,7 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // the count of input pieces streamed in by the host, and the Gram pre-pass's per-block
   // chunk counters (a pre-pass running beside the scan)
   P.off_progress = off;
-  if (with_output) off = align256(off + (2 * BH + 2 + BH * dla::kMaxGramBlk) * sizeof(int32_t));
+  if (with_output) off = align256(off + (2 * BH + 2 + kOutPieces + BH * dla::kMaxGramBlk) * sizeof(int32_t));
   P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
@@ -180,7 +183,6 @@ Schedule schedule() {
 
 constexpr int kTargetRounds = 8;  // rounds the read-out overlaps with the scan
 constexpr int kMinFreeSms = 8;    // SMs the scan must leave free for the concurrent schedule
-constexpr int kInputPieces = 16;  // pieces of inputs streamed in from host memory (dla_forward_host)
 constexpr size_t kPreferredWorkspace = (size_t)16 << 30;  // 16 GiB of read-out staging
 
 dla_status check_params(const dla_params* p) {
@@ -221,8 +223,9 @@ dla_status cuda_fail(cudaError_t e, const char* what) {
 struct StreamSet {
   cudaStream_t hi = nullptr, lo = nullptr;  // scan, read-out
   cudaStream_t cp = nullptr;                // host-to-device copies of streamed inputs
+  cudaStream_t cpo = nullptr;               // device-to-host copies of the streamed output
   cudaEvent_t in = nullptr, gram_done = nullptr, scan_done[2] = {nullptr, nullptr}, ro_done[2] = {nullptr, nullptr};
-  cudaEvent_t prep_done = nullptr, cp_done = nullptr;
+  cudaEvent_t prep_done = nullptr, cp_done = nullptr, cpo_done = nullptr;
   bool ready = false;
 };
 constexpr int kMaxDev = 64;
@@ -240,7 +243,9 @@ cudaError_t stream_set(StreamSet** out) {
     if ((e = cudaStreamCreateWithPriority(&S.hi, cudaStreamNonBlocking, greatest)) != cudaSuccess) return e;
     if ((e = cudaStreamCreateWithPriority(&S.lo, cudaStreamNonBlocking, least)) != cudaSuccess) return e;
     if ((e = cudaStreamCreateWithFlags(&S.cp, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    if ((e = cudaStreamCreateWithFlags(&S.cpo, cudaStreamNonBlocking)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.cp_done, cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&S.cpo_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.in, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.gram_done, cudaEventDisableTiming)) != cudaSuccess) return e;
     if ((e = cudaEventCreateWithFlags(&S.prep_done, cudaEventDisableTiming)) != cudaSuccess) return e;
@@ -275,7 +280,28 @@ WriteValue32Fn write_value_fn() {
   return fn;
 }
 
-// q, k, v, lambda in host memory and their device copies in the workspace.
+// A stream wait until a 32-bit word of device memory is >= a value (the
+// driver's stream memory operation: the stream, not an SM, waits).
+typedef CUresult (*WaitValue32Fn)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
+WaitValue32Fn wait_value_fn() {
+  static WaitValue32Fn fn = nullptr;
+  static bool tried = false;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> g(mu);
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuStreamWaitValue32", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<WaitValue32Fn>(p);
+  }
+  return fn;
+}
+
+// q, k, v, lambda in host memory and their device copies in the workspace;
+// o in host memory (copied back by the forward pass when it streams, else by
+// the caller).
 struct HostIO {
   const void* qh;
   const void* kh;
@@ -286,6 +312,9 @@ struct HostIO {
   void* vd;
   float* lamd;
   size_t elt;  // bytes per q, k, v element
+  void* oh;    // host output, or nullptr
+  size_t oelt; // bytes per o element
+  bool o_streamed = false;  // set by the forward pass: o was copied back piece by piece
 };
 // Tokens [t0, t1) of every batch row of k, v, q and lambda to the device, on stream s.
 cudaError_t h2d_tokens(const HostIO& io, int B, int T, int H, int d, int C, int t0, int t1, cudaStream_t s) {
@@ -492,7 +521,7 @@ static int concurrent_free_sms(int B, int H, int d, cudaError_t* err) {
 static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
                                const void* q, const void* k, const void* v, const float* lam, void* o,
                                const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
-                               size_t ws_bytes, void* stream, const HostIO* io) {
+                               size_t ws_bytes, void* stream, HostIO* io) {
   dla_status s = check_params(p);
   if (s != DLA_OK) return s;
   if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
@@ -659,7 +688,8 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
     int32_t* progress = (int32_t*)(ws + P.off_progress);
     int32_t* started = progress + 2 * B * H;
     int32_t* pieces = started + 1;  // input pieces streamed in so far
-    int32_t* gram_ready = started + 2;
+    int32_t* out_done = started + 2;  // [kOutPieces] read-out CTAs done per output piece
+    int32_t* gram_ready = out_done + kOutPieces;
     // with streamed inputs the scan forms its Gram entries itself: a pre-pass
     // waiting for the pieces would hold back the read-out behind it
     const bool run_gram = P.gram_chunks && !stream_in;
@@ -670,7 +700,8 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = gram_ready;
     dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * free_sms, &ga.nblk, &ga.per_blk);
-    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 2 + B * H * ga.nblk) * sizeof(int32_t), S->hi)) != cudaSuccess)
+    if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 2 + kOutPieces + B * H * ga.nblk) * sizeof(int32_t), S->hi)) !=
+        cudaSuccess)
       return cuda_fail(e, "progress reset");
     if ((e = cudaEventRecord(S->prep_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(S->lo, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
@@ -721,8 +752,39 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
     // (streams fastest), each waiting for its stream's progress
     ra.t_begin = 0; ra.t_end = T;
     ra.nsnap = P.nsnap_total; ra.snap_base = 0;
+    // Streamed output: pieces of opp interval pairs, each copied back once its
+    // read-out CTAs are done (a stream wait on their count: the copy stream
+    // waits, no SM does)
+    const bool stream_out = stream_in && io->oh && wait_value_fn();
+    const int npairs = (P.nsnap_total + 1) / 2;
+    const int opp = std::max(1, (npairs + kOutPieces - 1) / kOutPieces), nop = (npairs + opp - 1) / opp;
+    if (stream_out) {
+      ra.out_done = out_done;
+      ra.out_piece_pairs = opp;
+    }
+    ra.lam_l2 = stream_in ? 1 : 0;
     e = timed(DLA_K_READOUT, S->lo, [&] { return dla::launch_readout_tc(ra, status, S->lo); });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
+    if (stream_out) {
+      if ((e = cudaStreamWaitEvent(S->cpo, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+      const int tp = 2 * P.interval;  // tokens per interval pair
+      for (int op = 0; op < nop; ++op) {
+        const int p0 = op * opp, p1 = std::min(npairs, p0 + opp);
+        if (wait_value_fn()((CUstream)S->cpo, (CUdeviceptr)(out_done + op), (cuuint32_t)(B * H * (p1 - p0)), 0) !=
+            CUDA_SUCCESS)
+          return fail(DLA_ERR_CUDA, "stream memory wait failed");
+        const int t0 = p0 * tp, t1 = std::min(T, p1 * tp);
+        for (int b = 0; b < B; ++b) {
+          const size_t off = ((size_t)b * T + t0) * H * d * io->oelt, n = (size_t)(t1 - t0) * H * d * io->oelt;
+          if ((e = cudaMemcpyAsync((char*)io->oh + off, (const char*)o + off, n, cudaMemcpyDeviceToHost, S->cpo)) !=
+              cudaSuccess)
+            return cuda_fail(e, "output copy");
+        }
+      }
+      if ((e = cudaEventRecord(S->cpo_done, S->cpo)) != cudaSuccess) return cuda_fail(e, "event record");
+      if ((e = cudaStreamWaitEvent(st, S->cpo_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+      io->o_streamed = true;
+    }
     if (stream_in) {
       for (int pi = 1; pi < npiece; ++pi)
         if ((s = put_piece(pi)) != DLA_OK) return s;
@@ -864,12 +926,14 @@ dla_status dla_forward_host(const dla_params* p, dla_dtype in_dtype, int B, int 
   io.vd = bufs + hb.v;
   io.lamd = (float*)(bufs + hb.lam);
   io.elt = (in_dtype == DLA_BF16) ? 2 : 4;
+  io.oh = with_output ? o : nullptr;
+  io.oelt = (p->out_dtype == DLA_BF16) ? 2 : 4;
   void* od = with_output ? bufs + hb.o : nullptr;
   s = forward_impl(p, in_dtype, B, T, H, dk, dv, with_output ? io.qd : nullptr, io.kd, io.vd,
                    (with_output && lam) ? io.lamd : nullptr, od, cache, boundary, merge_log, workspace, fw_bytes,
                    stream, &io);
   if (s != DLA_OK) return s;
-  if (with_output) {
+  if (with_output && !io.o_streamed) {
     const size_t ob = (size_t)B * T * H * d * ((p->out_dtype == DLA_BF16) ? 2 : 4);
     const cudaError_t e = cudaMemcpyAsync(o, od, ob, cudaMemcpyDeviceToHost, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "output copy");

@@ -117,6 +117,12 @@ struct ReadoutArgs {
   int interval;          // tokens per snapshot interval
   const int32_t* progress;  // [B*H][2] scan progress to wait for (the scan runs concurrently), or nullptr
   int progress_ctas;        // scan CTAs per stream (1 or 2): entries of progress[bh] that count
+  // Output copied back piece by piece while the read-out runs (tensor-core
+  // read-out), or nullptr: every CTA adds 1 to out_done[pair / out_piece_pairs]
+  // once its rows of o are stored (after a device-scope fence)
+  int32_t* out_done;
+  int out_piece_pairs;
+  int lam_l2;  // 1: lambda arrives while the kernel runs (streamed inputs): read it through L2
   int32_t* status;          // device status word
 };
 

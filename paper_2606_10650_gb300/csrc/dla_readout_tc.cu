@@ -154,7 +154,11 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
 
 }  // namespace
 
-// 18 warps: the sub-partitions holding five of them bound a thread to 96 registers
+// 18 warps: the sub-partitions holding five of them bound a thread to 96 registers.
+// kStream: inputs streamed in by the host while the kernel runs (lambda read
+// through L2) and the output copied back piece by piece (per-piece CTA counts);
+// a separate instance, so the common one keeps its code unchanged.
+template <bool kStream>
 __global__ void __launch_bounds__(NT, 1)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
@@ -404,13 +408,18 @@ __global__ void __launch_bounds__(NT, 1)
       sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");
-    // lambda through L2 (__ldcg): inputs streamed in by the host arrive while this kernel runs
     const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
+    // lambda is read-only while the kernel runs (the read-only path), except when
+    // the host streams it in beside the work (then through L2)
+    auto lam_at = [&](int i) -> float {
+      if constexpr (kStream) return __ldcg(lam_t + i);
+      else return __ldg(lam_t + i);
+    };
     const int evt_t = sm.side[side].evt[t];
     // an interval without boundary events (the common case) weights every
     // column s <= t of row t by lambda of the open entry: loaded ahead of P
     const bool no_ev = sm.side[side].evt[L - 1] == 0;  // warp-uniform
-    const float w_open = (no_ev && t < Lcs) ? (lam_t ? __ldcg(lam_t + sm.tab[side][0]) : 1.f) : 0.f;
+    const float w_open = (no_ev && t < Lcs) ? (lam_t ? lam_at(sm.tab[side][0]) : 1.f) : 0.f;
     bool ok;
     {  // P (accumulator 0) -> Pt over this interval's K tile (its MMAs are complete)
       ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[0], 0, abort, status));
@@ -444,7 +453,7 @@ __global__ void __launch_bounds__(NT, 1)
                   const int e = evs[ss];
                   if (e != last_e) {
                     last_e = e;
-                    last_w = lam_t ? __ldcg(lam_t + trow[e]) : 1.f;
+                    last_w = lam_t ? lam_at(trow[e]) : 1.f;
                   }
                   wt = last_w;
                 }
@@ -495,7 +504,7 @@ __global__ void __launch_bounds__(NT, 1)
         if (x >= nu || t >= Lcs) return 0.f;
         const int xi = ux[x];
         if (xi < 0) return 0.f;
-        return lam_t ? __ldcg(lam_t + tab_t[xi]) : 1.f;
+        return lam_t ? lam_at(tab_t[xi]) : 1.f;
       };
       float wn = weight(0);
       for (int x = 0; ok && x < nu; ++x) {
@@ -538,6 +547,14 @@ __global__ void __launch_bounds__(NT, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  // every CTA reaches this point, also after a failed wait: the host's copy of
+  // the output piece waits for the count of its CTAs
+  if constexpr (kStream) {
+    if (a.out_done && tid == 0) {
+      __threadfence();
+      atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
+    }
+  }
 }
 
 // ---------------------------------------------------------------- host side
@@ -548,11 +565,13 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
       !tmap_tokens(&mv, a.v, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
     return cudaErrorInvalidValue;
   const size_t smem = sizeof(TcSmem) + 1024;
-  cudaError_t e = cudaFuncSetAttribute(readout_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const bool stream = a.lam_l2 || a.out_done;
+  auto kern = stream ? readout_tc_kernel<true> : readout_tc_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
   dim3 grid(a.B * a.H, (a.nsnap + 1) / 2);  // streams x pairs of intervals
-  readout_tc_kernel<<<grid, NT, smem, st>>>(a, mq, mk, mv, ms, status);
+  kern<<<grid, NT, smem, st>>>(a, mq, mk, mv, ms, status);
   return cudaGetLastError();
 }
 
@@ -560,7 +579,9 @@ size_t readout_tc_smem_bytes() { return sizeof(TcSmem) + 1024; }
 
 cudaError_t preload_readout_kernels() {
   cudaFuncAttributes fa;
-  return cudaFuncGetAttributes(&fa, readout_tc_kernel);
+  cudaError_t e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false>);
+  if (e != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, readout_tc_kernel<true>);
 }
 
 }  // namespace dla
