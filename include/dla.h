@@ -18,7 +18,8 @@
  *
  * Conventions
  *   - Every pointer argument is DEVICE memory owned by the caller, except the
- *     dla_params / dla_cache structs themselves, which are read on the host.
+ *     dla_params / dla_cache structs themselves, which are read on the host,
+ *     and the q, k, v, lam, o of dla_forward_host, which are host memory.
  *     The library never allocates device memory and frees nothing.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  All device
  *     work is enqueued asynchronously on it; argument errors are returned
@@ -196,9 +197,10 @@ size_t dla_forward_host_workspace(const dla_params* p, int B, int T, int H, int 
  * pieces of whole 64-token chunks on an internal stream, each piece followed
  * by a stream memory write of the count of pieces in place; the scan waits
  * (bounded) for the piece of every chunk it loads and forms its Gram entries
- * itself, the read-out follows the scan, so the copies overlap the work.  On
- * the other schedules the inputs are copied first.  o is copied back on
- * `stream` after the read-out.  The call only enqueues work: the host buffers
+ * itself, the read-out follows the scan, and o goes back in 16 pieces on
+ * another internal stream, each after a stream wait for the count of its
+ * read-out CTAs, so the copies overlap the work.  On the other schedules the
+ * inputs are copied first and o after the read-out.  The call only enqueues work: the host buffers
  * must stay valid, and o is filled, once `stream` has completed it.  Results
  * equal dla_forward's on the same inputs (decisions bit-identical; the
  * outputs to rounding of the Gram sums). */
