@@ -245,3 +245,19 @@ def test_forward_host_buffers(case, sched, monkeypatch):
     r = run_oracle(w, q, k, v, lam)
     compare(w, g, r)
     structural_checks(w, g, w.T)
+
+
+def test_dla_i_without_capacity_bound():
+    """DLA(I) (Table 5: dynamic merging without the capacity bound) on the GPU:
+    with C = 64 above each stream's number of segments nothing merges, and the
+    oracle without a capacity bound (C = T + 1) gives the same decisions and
+    outputs."""
+    w = W.get("regime", B=1, H=2, T=1500, C=64)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    assert (g["merge_log"] == -1).all() and g["boundary"].sum() > 4
+    lam_o = np.zeros(lam.shape[:3] + (w.T + 1,))
+    lam_o[..., :w.C] = lam
+    r = oracle.forward(q, k, v, lam_o, tau=w.tau, C=w.T + 1, eps=w.eps, rms_eps=w.rms_eps)
+    compare(w, g, r, check_cache=False)
+    structural_checks(w, g, w.T)

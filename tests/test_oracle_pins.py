@@ -181,6 +181,38 @@ def test_tau_zero_per_token_states_closed_form():
     np.testing.assert_allclose(ex["ibar"], it, rtol=0, atol=0)
 
 
+def test_uncapped_dla_i_segment_sums():
+    """DLA(I) (Table 5: dynamic merging without the capacity bound): with C above
+    the number of segments nothing merges, every segment keeps its own state
+    S_i = sum of v_s k_s^T over its tokens, and o_t = sum_i lambda_{t,i} S_i q_t
+    over the segments begun at or before t, the open one holding the tokens up
+    to t.  Recomputed here from the boundary trace alone."""
+    rng = np.random.default_rng(23)
+    T, d = 60, 4
+    q, k, v = _rand_stream(rng, T, d)
+    probe = oracle.Stream(2, d, d, tau=1e300)
+    _, _, _, it = probe.run(q, k, v)
+    tau = float(np.quantile(it[1:], 0.8))
+    C = T + 1
+    lam = rng.uniform(0.5, 1.5, size=(T, C))
+    st = oracle.Stream(C, d, d, tau=tau)
+    o, bnd, ml, _ = st.run(q, k, v, lam)
+    assert (ml == -1).all() and 3 < int(bnd.sum()) < T
+    starts = [int(s_) for s_ in np.flatnonzero(bnd)]
+    ends = starts[1:] + [T]
+    O = np.zeros((T, d))
+    for t in range(T):
+        for i, (s0, s1) in enumerate(zip(starts, ends)):
+            if s0 > t:
+                break
+            S = sum(np.outer(v[s_], k[s_]) for s_ in range(s0, min(s1, t + 1)))
+            O[t] += lam[t, i] * (S @ q[t])
+    np.testing.assert_allclose(o, O, rtol=1e-12, atol=1e-12)
+    ex = st.export()
+    assert ex["m"] == len(starts)
+    assert ex["n"][:len(starts)].tolist() == [e - s_ for s_, e in zip(starts, ends)]
+
+
 # ------------------------------------------------------------------ brute force on tiny inputs
 
 @pytest.mark.parametrize("C", [2, 3, 4])
