@@ -71,7 +71,14 @@ typedef enum { DLA_BF16 = 0, DLA_F32 = 1 } dla_dtype;
  *   score_mode 0: Algorithm 1's score, token state s_t against the last state.
  *   score_mode 1: Eq. (importance_score) read literally: N(S + s_t) against N(S).
  *   from_cache  0: dla_forward starts from an empty cache (prefill);
- *               1: it continues from the contents of `cache` (chunked prefill). */
+ *               1: it continues from the contents of `cache` (chunked prefill).
+ *   seq_lens    NULL: every batch row holds T tokens.  Else device int32 [B],
+ *               4-byte aligned (ragged batches in the padded layout): row b
+ *               holds its first seq_lens[b] tokens (clamped to [0, T]); the
+ *               tokens after them are padding: not processed, boundary 0 and
+ *               merge_log -1 there, their o rows not written, and the row's
+ *               cache is the one after its own tokens.  The forward calls read
+ *               it; dla_decode_step ignores it. */
 typedef struct {
   double tau;
   double eps;
@@ -80,6 +87,7 @@ typedef struct {
   int score_mode;
   dla_dtype out_dtype;
   int from_cache;
+  const int32_t* seq_lens;
 } dla_params;
 
 /* The state cache M of Algorithm 2 for B x H streams (device memory, caller

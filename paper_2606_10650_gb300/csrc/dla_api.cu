@@ -389,6 +389,7 @@ void dla_default_params(dla_params* p) {
   p->score_mode = 0;
   p->out_dtype = DLA_F32;
   p->from_cache = 0;
+  p->seq_lens = nullptr;
 }
 
 int dla_version(void) { return DLA_VERSION; }
@@ -536,6 +537,7 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
   if (!aligned(k, vec) || !aligned(v, vec) || (q && !aligned(q, vec)) || (o && !aligned(o, vec)))
     return fail(DLA_ERR_INVALID_ARG, "q, k, v, o must be 16-byte aligned");
   if (lam && !aligned(lam, 4)) return fail(DLA_ERR_INVALID_ARG, "lambda must be 4-byte aligned");
+  if (p->seq_lens && !aligned(p->seq_lens, 4)) return fail(DLA_ERR_INVALID_ARG, "seq_lens must be 4-byte aligned");
   if (cache) {
     if ((s = check_cache(cache, B, H, C, d)) != DLA_OK) return s;
   } else if (p->from_cache) {
@@ -588,6 +590,7 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
   sa.states = live.states; sa.slot = live.slot; sa.n = live.n; sa.ibar = live.ibar; sa.m = live.m;
   sa.boundary = bnd; sa.merge_log = mlog;
   sa.status = status;
+  sa.seq_lens = p->seq_lens;
   const bool in_bf16 = (in_dtype == DLA_BF16);
   const bool tc = use_tc(in_dtype, d);
   const bool pool_bf16 = tc;
@@ -605,6 +608,7 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
   ra.B = B; ra.T = T; ra.H = H; ra.C = C;
   ra.boundary = bnd; ra.merge_log = mlog;
   ra.status = status;
+  ra.seq_lens = p->seq_lens;
   ra.interval = P.interval;
   sa.snap_chunks = P.interval / dla::kScanL;
   sa.pool_cap = P.pool_cap;

@@ -85,6 +85,21 @@ __device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
 // the caller's CTA barrier then orders every later read after the wait.  Data
 // the scan writes must then be read past L1 (__ldcg): another CTA on the SM may
 // hold an older copy of the line.
+// This stream's end of the round [t_begin, t_end): the call's t_end, or, with
+// per-row lengths, row b's length clamped to [t_begin, t_end] (tokens past it
+// are padding).
+__device__ __forceinline__ int row_t_end(const int32_t* seq_lens, int b, int t_begin, int t_end) {
+  if (!seq_lens) return t_end;
+  return max(t_begin, min(t_end, __ldg(seq_lens + b)));
+}
+// Decision trace of padding tokens [t0, t1) of one stream: no boundary, no merge.
+__device__ __forceinline__ void fill_padding_trace(uint8_t* bnd, int32_t* mlog, int t0, int t1, int i0, int ni) {
+  for (int t = t0 + i0; t < t1; t += ni) {
+    bnd[t] = 0;
+    mlog[t] = -1;
+  }
+}
+
 __device__ __forceinline__ void wait_progress(const int32_t* progress, int ctas, int bh, int need, int32_t* status) {
   if (!progress || threadIdx.x != 0) return;
   const long long t0 = clock64();

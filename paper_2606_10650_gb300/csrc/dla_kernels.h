@@ -70,6 +70,7 @@ struct ScanArgs {
   // rows have arrived, written in stream order after each piece's copies
   const int32_t* piece_ready;
   int piece_chunks;
+  const int32_t* seq_lens;  // [B] tokens of each row (padding after them), or nullptr: T each
   int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
   int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)
@@ -122,6 +123,7 @@ struct ReadoutArgs {
   // once its rows of o are stored (after a device-scope fence)
   int32_t* out_done;
   int out_piece_pairs;
+  const int32_t* seq_lens;  // [B] tokens of each row (padding after them), or nullptr: T each
   int lam_l2;  // 1: lambda arrives while the kernel runs (streamed inputs): read it through L2
   int32_t* status;          // device status word
 };

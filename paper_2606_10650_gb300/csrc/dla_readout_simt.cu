@@ -65,7 +65,8 @@ __global__ void __launch_bounds__(NT, 1) readout_simt_kernel(ReadoutArgs a) {
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const int c0 = a.t_begin + s * L;
-  const int Lc = min(L, a.t_end - c0);
+  const int Lc = min(L, row_t_end(a.seq_lens, b, a.t_begin, a.t_end) - c0);
+  if (Lc <= 0) return;  // the interval lies past this row's length: padding, o not written
   const int row_stride = a.H * D;
   const long long tok0 = ((long long)b * a.T + c0) * a.H + h;  // row index of token c0
   const int m0 = a.snap_m0[(long long)bh * a.snap_stride + a.snap_base + s];

@@ -156,9 +156,10 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
 
 // 18 warps: the sub-partitions holding five of them bound a thread to 96 registers.
 // kStream: inputs streamed in by the host while the kernel runs (lambda read
-// through L2) and the output copied back piece by piece (per-piece CTA counts);
-// a separate instance, so the common one keeps its code unchanged.
-template <bool kStream>
+// through L2) and the output copied back piece by piece (per-piece CTA counts).
+// kRagged: per-row lengths (padding after them).  Separate instances, so the
+// common one keeps its code unchanged.
+template <bool kStream, bool kRagged>
 __global__ void __launch_bounds__(NT, 1)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
@@ -170,7 +171,17 @@ __global__ void __launch_bounds__(NT, 1)
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const int sA = 2 * pair;
-  const bool hasB = (sA + 1) < a.nsnap;
+  // this row's end (padding after it)
+  const int t_end = kRagged ? row_t_end(a.seq_lens, b, a.t_begin, a.t_end) : a.t_end;
+  if constexpr (kRagged) {
+    if (a.t_begin + sA * L >= t_end) {  // the pair lies past the row's length: o not written
+      if constexpr (kStream) {
+        if (a.out_done && tid == 0) atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
+      }
+      return;
+    }
+  }
+  const bool hasB = (sA + 1) < a.nsnap && (!kRagged || a.t_begin + (sA + 1) * L < t_end);
   // with a scan running concurrently: both intervals of the pair must be complete
   wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + sA + (hasB ? 2 : 1), a.status);
   // thread 0 issues the TMA loads: they read what the scan wrote (pool entries)
@@ -179,7 +190,7 @@ __global__ void __launch_bounds__(NT, 1)
   __syncthreads();
   // interval A (side 0) and B (side 1) of the pair
   const int c0A = a.t_begin + sA * L, c0B = c0A + L;
-  const int LcA = min(L, a.t_end - c0A), LcB = hasB ? min(L, a.t_end - c0B) : 0;
+  const int LcA = min(L, t_end - c0A), LcB = hasB ? min(L, t_end - c0B) : 0;
   const long long lrowA = (long long)bh * a.snap_stride + a.snap_base + sA, lrowB = lrowA + 1;
   // lists and trace come from the scan: read past L1 (__ldcg)
   const int m0A = __ldcg(a.snap_m0 + lrowA), m0B = hasB ? __ldcg(a.snap_m0 + lrowB) : 0;
@@ -565,8 +576,9 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
       !tmap_tokens(&mv, a.v, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
     return cudaErrorInvalidValue;
   const size_t smem = sizeof(TcSmem) + 1024;
-  const bool stream = a.lam_l2 || a.out_done;
-  auto kern = stream ? readout_tc_kernel<true> : readout_tc_kernel<false>;
+  const bool stream = a.lam_l2 || a.out_done, ragged = a.seq_lens != nullptr;
+  auto kern = stream ? (ragged ? readout_tc_kernel<true, true> : readout_tc_kernel<true, false>)
+                     : (ragged ? readout_tc_kernel<false, true> : readout_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
@@ -579,9 +591,11 @@ size_t readout_tc_smem_bytes() { return sizeof(TcSmem) + 1024; }
 
 cudaError_t preload_readout_kernels() {
   cudaFuncAttributes fa;
-  cudaError_t e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false>);
-  if (e != cudaSuccess) return e;
-  return cudaFuncGetAttributes(&fa, readout_tc_kernel<true>);
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false, false>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<true, false>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false, true>)) != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, readout_tc_kernel<true, true>);
 }
 
 }  // namespace dla

@@ -192,9 +192,10 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   }
   __syncthreads();
 
-  const int ntok = a.t_end - a.t_begin;
+  const int t_end = row_t_end(a.seq_lens, b, a.t_begin, a.t_end);  // this row's end of the round
+  const int ntok = t_end - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
-  if constexpr (sizeof(Tin) == 2) {
+  if (sizeof(Tin) == 2 && ntok > 0) {  // a row that ended before this round has no chunk to load
     prefetch_kv<D>(sm.raw[0][0], sm.raw[0][1], reinterpret_cast<const __nv_bfloat16*>(kbase) +
                                                    (long long)a.t_begin * row_stride,
                    reinterpret_cast<const __nv_bfloat16*>(vbase) + (long long)a.t_begin * row_stride, row_stride,
@@ -202,7 +203,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   }
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
-    const int Lc = min(L, a.t_end - t0);
+    const int Lc = min(L, t_end - t0);
     // ------------------------------------------------ 1. stage k, v
     if constexpr (sizeof(Tin) == 2) {
       // bf16: this chunk was prefetched during the previous one; start the next
@@ -211,7 +212,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
         prefetch_kv<D>(sm.raw[(c + 1) & 1][0], sm.raw[(c + 1) & 1][1],
                        reinterpret_cast<const __nv_bfloat16*>(kbase) + (long long)t1 * row_stride,
                        reinterpret_cast<const __nv_bfloat16*>(vbase) + (long long)t1 * row_stride, row_stride,
-                       min(L, a.t_end - t1));
+                       min(L, t_end - t1));
         asm volatile("cp.async.wait_group 1;" ::: "memory");
       } else {
         asm volatile("cp.async.wait_group 0;" ::: "memory");
@@ -576,6 +577,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
     }
   }
   // ---------------------------------------------------------------- round end
+  fill_padding_trace(bnd_out, mlog_out, t_end, a.t_end, tid, NT);
   {
     const int m = sm.m;
     if (m > 0) {

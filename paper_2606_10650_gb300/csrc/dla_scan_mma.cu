@@ -447,7 +447,9 @@ __device__ __forceinline__ void entry_next(const T (&f)[2], T (&nx)[2]) {
 // parts meet through distributed shared memory once per chunk; both CTAs then
 // take the same decisions from the same sums (x = part of rank 0 + part of
 // rank 1 in both), and rank 0 writes the trace, the lists and the metadata.
-template <int D, typename Tpool, int CL>
+// kRagged: per-row lengths (padding after them); a separate instance, so the
+// common one keeps its code.
+template <int D, typename Tpool, int CL, bool kRagged = false>
 __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   constexpr int RP = D + 8;
   constexpr int R = D / CL;           // state rows of this CTA
@@ -653,7 +655,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   publish_state(0);
   __syncthreads();
 
-  const int ntok = a.t_end - a.t_begin;
+  // this row's end of the round (the call's t_end unless per-row lengths are given)
+  const int t_end_r = kRagged ? row_t_end(a.seq_lens, b, a.t_begin, a.t_end) : 0;
+#define DLA_T_END (kRagged ? t_end_r : a.t_end)
+  const int ntok = DLA_T_END - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
   const long long gchunk0 = (long long)bh * a.gram_chunks + a.t_begin / L;  // Gram block of the round's first chunk
   GramFeed feed;
@@ -663,6 +668,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   int piece_known = 0;  // streamed inputs: pieces known to have arrived (this thread)
   if (tid == 0)
     for (int i = 0; i < kMaxGramBlk; ++i) sm.gcnt[i] = 0;
+  if (!kRagged || ntok > 0)  // a row that ended before this round has no chunk to load
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
                       a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
@@ -671,7 +677,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   int rel_pending = 0;  // thread NT - 32: progress value not yet released
   for (int c = 0; c < nchunks; ++c) {
     const int t0 = a.t_begin + c * L;
-    const int Lc = min(L, a.t_end - t0);
+    const int Lc = min(L, DLA_T_END - t0);
     const int st = c & 1;
     // ------------------------------------------------ 1. k, v of this chunk (issued during the
     // previous chunk's passes, or before the loop)
@@ -790,7 +796,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     if (warp != 0 && c + 1 < nchunks) {
       const int t1 = t0 + L;
       prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
-                        vbase + (long long)t1 * row_stride, row_stride, min(L, a.t_end - t1), sm.gq[st ^ 1],
+                        vbase + (long long)t1 * row_stride, row_stride, min(L, DLA_T_END - t1), sm.gq[st ^ 1],
                         a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
                         a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32, a.piece_ready,
                         a.piece_chunks ? (a.t_begin / L + c + 1) / a.piece_chunks + 1 : 0, piece_known);
@@ -1083,6 +1089,9 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     if (tid == 0) st_release_gpu(a.progress + 2 * bh + rank, a.snap_base + a.nsnap);
   }
   // ---------------------------------------------------------------- round end
+  if constexpr (kRagged)
+    if (lead) fill_padding_trace(bnd_out, mlog_out, t_end_r, a.t_end, tid, NT);
+#undef DLA_T_END
   {
     const int m = sm.m;
     if (m > 0) {
@@ -1227,10 +1236,10 @@ cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s) {
   return d == 128 ? launch_gram_t<128>(a, s) : launch_gram_t<64>(a, s);
 }
 
-template <int D, typename Tpool, int CL>
-static cudaError_t launch_scan_mma_t(const ScanArgs& a, cudaStream_t s) {
+template <int D, typename Tpool, int CL, bool kRagged>
+static cudaError_t launch_scan_mma_r(const ScanArgs& a, cudaStream_t s) {
   const size_t smem = sizeof(MmaSmem<D, CL>);
-  auto kern = scan_mma_kernel<D, Tpool, CL>;
+  auto kern = scan_mma_kernel<D, Tpool, CL, kRagged>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -1246,6 +1255,10 @@ static cudaError_t launch_scan_mma_t(const ScanArgs& a, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = CL > 1 ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, a);
+}
+template <int D, typename Tpool, int CL>
+static cudaError_t launch_scan_mma_t(const ScanArgs& a, cudaStream_t s) {
+  return a.seq_lens ? launch_scan_mma_r<D, Tpool, CL, true>(a, s) : launch_scan_mma_r<D, Tpool, CL, false>(a, s);
 }
 
 int scan_mma_ctas_per_stream(int BH, int d) {
@@ -1332,6 +1345,8 @@ cudaError_t preload_scan_kernels() {
   cudaError_t e;
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2, true>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1, true>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_kernel<128>)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, gate_kernel);
 }

@@ -35,7 +35,7 @@ class DLAError(RuntimeError):
 class dla_params(ctypes.Structure):
     _fields_ = [("tau", ctypes.c_double), ("eps", ctypes.c_double), ("rms_eps", ctypes.c_double),
                 ("capacity", ctypes.c_int), ("score_mode", ctypes.c_int), ("out_dtype", ctypes.c_int),
-                ("from_cache", ctypes.c_int)]
+                ("from_cache", ctypes.c_int), ("seq_lens", ctypes.c_void_p)]
 
 
 class dla_cache(ctypes.Structure):
@@ -105,9 +105,12 @@ def _dtype_code(t):
     raise TypeError(f"unsupported input dtype {t.dtype} (bf16 or fp32)")
 
 
-def make_params(tau, capacity, eps=1e-6, rms_eps=1e-6, score_mode=0, out_dtype=DLA_F32, from_cache=0):
+def make_params(tau, capacity, eps=1e-6, rms_eps=1e-6, score_mode=0, out_dtype=DLA_F32, from_cache=0,
+                seq_lens=None):
+    """seq_lens: None, or an int32 CUDA tensor [B] of per-row lengths (ragged
+    batches in the padded layout; it must outlive the calls that use the params)."""
     return dla_params(float(tau), float(eps), float(rms_eps), int(capacity), int(score_mode), int(out_dtype),
-                      int(from_cache))
+                      int(from_cache), None if seq_lens is None else seq_lens.data_ptr())
 
 
 def dla_default_params():

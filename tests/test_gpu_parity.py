@@ -261,3 +261,60 @@ def test_dla_i_without_capacity_bound():
     r = oracle.forward(q, k, v, lam_o, tau=w.tau, C=w.T + 1, eps=w.eps, rms_eps=w.rms_eps)
     compare(w, g, r, check_cache=False)
     structural_checks(w, g, w.T)
+
+
+RAGGED = {
+    # name: (workload, overrides, per-row lengths)
+    "regime_bf16": ("regime", dict(B=3, H=2, T=1300), [1300, 517, 1]),
+    "standard_bf16": ("standard", dict(B=3, H=2, T=700), [0, 700, 333]),
+    "d64_bf16": ("standard", dict(B=2, H=2, T=700, d=64, C=8, tau=1.4215), [257, 700]),
+    "d128_fp32": ("tiny", dict(B=2, H=2, T=300, d=128, C=6, tau=1.4142), [300, 129]),
+}
+
+
+@pytest.mark.parametrize("sched", ["concurrent", "rounds"])
+@pytest.mark.parametrize("case", list(RAGGED))
+def test_ragged_rows(case, sched, monkeypatch):
+    """Ragged batches in the padded layout (dla_params.seq_lens): row b runs
+    over its first seq_lens[b] tokens exactly as a call on those tokens alone
+    (the oracle per row); padding tokens get boundary 0 and merge_log -1, and
+    their output rows are not written."""
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
+    name, ov, lens = RAGGED[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    dev = torch.device("cuda:0")
+    qt, kt, vt, lt = upload(w, q, k, v, lam)
+    B, T, H, d = kt.shape
+    sl = torch.tensor(lens, dtype=torch.int32, device=dev)
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps, seq_lens=sl)
+    o = torch.full((B, T, H, d), float("nan"), dtype=torch.float32, device=dev)
+    bnd = torch.full((B, H, T), 7, dtype=torch.uint8, device=dev)
+    ml = torch.full((B, H, T), -7, dtype=torch.int32, device=dev)
+    ws = dla.dla_forward(p, qt, kt, vt, lt, o, cache, bnd, ml)
+    torch.cuda.synchronize()
+    assert dla.workspace_status(ws) == 0, "device status word reports a failure"
+    g = dict(o=o.double().cpu().numpy(), boundary=bnd.cpu().numpy(), merge_log=ml.cpu().numpy(), cache=cache)
+    r = dict(o=np.full((B, T, H, d), np.nan), boundary=np.zeros((B, H, T), np.uint8),
+             merge_log=np.full((B, H, T), -1, np.int32), caches={})
+    live = []
+    for b, n in enumerate(lens):
+        if n == 0:
+            continue
+        rb = oracle.forward(q[b:b + 1, :n], k[b:b + 1, :n], v[b:b + 1, :n], lam[b:b + 1, :n], tau=w.tau, C=w.C,
+                            eps=w.eps, rms_eps=w.rms_eps)
+        r["o"][b, :n] = rb["o"][0]
+        r["boundary"][b, :, :n] = rb["boundary"][0]
+        r["merge_log"][b, :, :n] = rb["merge_log"][0]
+        for h in range(H):
+            r["caches"][(b, h)] = rb["caches"][(0, h)]
+            live.append((b, h))
+    compare(w, g, r, streams=live)
+    ex = cache.export()
+    for b, n in enumerate(lens):
+        assert np.isnan(g["o"][b, n:]).all(), f"row {b}: padding output written"
+        np.testing.assert_array_equal(g["boundary"][b, :, n:], 0)
+        np.testing.assert_array_equal(g["merge_log"][b, :, n:], -1)
+        if n == 0:
+            assert (ex["m"][b] == 0).all()
