@@ -95,3 +95,14 @@ def test_host_buffer_entry_point_errors_and_workspace(L):
     assert fh(ws=False) == 3
     assert fh(ws_bytes=1024) == 3
     assert b"workspace" in L.dla_last_error()
+
+
+def test_params_layout_and_seq_lens_checks(L):
+    p = dla.dla_params()
+    p.seq_lens = 12345
+    L.dla_default_params(ctypes.byref(p))
+    assert p.tau == 0.6 and p.capacity == 30 and p.from_cache == 0 and not p.seq_lens
+    q = dla.make_params(0.6, 8)
+    q.seq_lens = (1 << 20) + 2  # not 4-byte aligned
+    assert _fwd(L, q) == 1
+    assert b"seq_lens" in L.dla_last_error()
