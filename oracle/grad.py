@@ -1,0 +1,88 @@
+"""fp64 oracle of the gradients of the read-out with hard decisions.
+
+TEST INFRASTRUCTURE ONLY (like the rest of ``oracle/``): plain numpy in fp64,
+shares no code with the CUDA library.
+
+With the boundary and merge decisions of a forward pass held fixed (they are
+piecewise constant in k and v, so their derivative is zero almost everywhere),
+the read-out of Eq. (capacity_bounded_output) is a weighted causal linear
+attention.  Every state is a sum of token states (Sec. 2 recurrent form; a
+merge of Algorithm 2 sums two adjacent states), so
+
+    o_t = sum_i lambda_{t,i} S_i q_t = sum_{s <= t} lambda_{t, slot_t(s)} (k_s . q_t) v_s,
+
+where slot_t(s) is the logical slot (0 = oldest) of the state holding token s
+after token t.  With W[t, s] = lambda_{t, slot_t(s)} for s <= t (0 above the
+diagonal), o = ((Q K^T) * W) V, and for a loss with dL/do = G:
+
+    dQ = ((G V^T) * W) K          dK = ((G V^T) * W)^T Q
+    dV = ((Q K^T) * W)^T G        dlambda_{t,i} = sum_{s <= t, slot_t(s) = i} (q_t . k_s)(g_t . v_s)
+
+The slots come from replaying Algorithm 2's decisions (the boundary flags and
+merge indices the forward pass reports) on token ranges: every state holds a
+contiguous range of tokens, a boundary appends a new range, a merge at index j
+joins ranges j and j + 1.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def token_slots(boundary, merge_log):
+    """slot[t, s]: logical slot of the state holding token s after token t
+    (s <= t), -1 for s > t.  boundary [T] (b_t, the first token of an empty
+    cache counted as a boundary), merge_log [T] (i* of the merge at token t, or
+    -1), as the forward pass reports them (Algorithm 2 replayed on token ranges)."""
+    boundary = np.asarray(boundary)
+    merge_log = np.asarray(merge_log)
+    T = boundary.shape[0]
+    firsts = []  # first token of each state, chronological (states are contiguous ranges)
+    slot = np.full((T, T), -1, dtype=np.int64)
+    for t in range(T):
+        if boundary[t] or not firsts:
+            j = int(merge_log[t])
+            if j >= 0:  # states j and j + 1 become one: the later range joins the earlier
+                del firsts[j + 1]
+            firsts.append(t)
+        # token s belongs to the last state whose first token is <= s
+        slot[t, : t + 1] = np.searchsorted(np.asarray(firsts), np.arange(t + 1), side="right") - 1
+    return slot
+
+
+def weights(boundary, merge_log, lam):
+    """W[t, s] = lambda_{t, slot_t(s)} for s <= t, else 0 (lam [T, C]; None = ones)."""
+    slot = token_slots(boundary, merge_log)
+    T = slot.shape[0]
+    W = np.zeros((T, T))
+    for t in range(T):
+        sl = slot[t, : t + 1]
+        W[t, : t + 1] = 1.0 if lam is None else np.asarray(lam, dtype=np.float64)[t, sl]
+    return W
+
+
+def readout_dense(q, k, v, W):
+    """o = ((Q K^T) * W) V: the read-out as a weighted causal linear attention."""
+    q, k, v = (np.asarray(x, dtype=np.float64) for x in (q, k, v))
+    return ((q @ k.T) * W) @ v
+
+
+def readout_grads(q, k, v, lam, boundary, merge_log, g):
+    """Gradients of L = sum_t g_t . o_t with the decisions held fixed.
+    Returns dict(dq, dk, dv, dlam); dlam is None when lam is None."""
+    q, k, v, g = (np.asarray(x, dtype=np.float64) for x in (q, k, v, g))
+    slot = token_slots(boundary, merge_log)
+    W = weights(boundary, merge_log, lam)
+    A = q @ k.T            # (q_t . k_s)
+    Bg = g @ v.T           # (g_t . v_s)
+    dq = (Bg * W) @ k
+    dk = (Bg * W).T @ q
+    dv = (A * W).T @ g
+    dlam = None
+    if lam is not None:
+        lam = np.asarray(lam, dtype=np.float64)
+        dlam = np.zeros_like(lam)
+        P = A * Bg
+        T = q.shape[0]
+        for t in range(T):
+            np.add.at(dlam[t], slot[t, : t + 1], P[t, : t + 1])
+    return dict(dq=dq, dk=dk, dv=dv, dlam=dlam)
