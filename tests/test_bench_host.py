@@ -46,3 +46,22 @@ def test_reference_arm_prints_one_json_line():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["value"] > 0 and d["e2e"]["h2d_bytes_per_step"] == 0
     assert d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_captured_traffic_follows_the_source_hash(tmp_path, monkeypatch):
+    """The roofline's DRAM traffic comes from a profile summary line only while
+    the kernel source still has the hash recorded beside it."""
+    import hashlib
+    import bench
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    src = tmp_path / "kernel.cu"
+    src.write_text("// kernel source\n")
+    sha = hashlib.sha256(src.read_bytes()).hexdigest()
+    summ = tmp_path / "summary.md"
+    summ.write_text(f"text\ntraffic_bytes_per_launch my_kernel 123456 {sha[:16]}\n")
+    rel = lambda p: os.path.relpath(str(p), root)
+    assert bench.captured_traffic("my_kernel", rel(src), rel(summ)) == 123456
+    assert bench.captured_traffic("other_kernel", rel(src), rel(summ)) is None
+    src.write_text("// kernel source, changed\n")
+    assert bench.captured_traffic("my_kernel", rel(src), rel(summ)) is None
+    assert bench.captured_traffic("my_kernel", rel(tmp_path / "missing.cu"), rel(summ)) is None
