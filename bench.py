@@ -286,12 +286,11 @@ def bench_prefill(args, dist, pk):
             sm_ms[name] = t * n_launch * n_sms
     # DRAM traffic per launch from a committed ncu summary, while the kernel's source is the one
     # captured and the workload is the one captured (else null)
-    tr = captured_traffic("readout_tc_kernel", "paper_2606_10650_gb300/csrc/dla_readout_tc.cu",
-                          "profiles/readout_dram_regime_full.md")
-    if tr and "readout" in rooflines and tc_path and (args.workload, B, T, H, d) == ("regime", 2, 16384, 16, 128):
-        rooflines["readout"]["traffic"] = tr
+    tr = captured_traffic("readout_tc_kernel", f"{args.workload} B{B} H{H} T{T} d{d}")
+    if tr and "readout" in rooflines and tc_path:
+        rooflines["readout"]["traffic"] = tr["bytes_per_launch"]
         rooflines["readout"]["traffic_note"] = ("dram__bytes_read.sum + dram__bytes_write.sum of one full-size "
-                                                "launch (ncu, profiles/readout_dram_regime_full.md)")
+                                                f"launch (ncu, {tr['summary']})")
     # dominant kernel: the largest SM-time per step (duration alone x SMs it occupies); the
     # step is close to the summed SM-time of the kernels over the 152 SMs
     dominant = max(sm_ms, key=lambda k: sm_ms[k]) if sm_ms else None
@@ -344,24 +343,23 @@ def bench_prefill(args, dist, pk):
     return res
 
 
-def captured_traffic(kernel, source, summary):
-    """Bytes per launch recorded in a profile summary line
-    'traffic_bytes_per_launch <kernel> <bytes> <sha256 prefix of source>', if the source file
-    still has that hash; else None."""
+def captured_traffic(kernel, workload, table=None):
+    """The DRAM traffic record of `kernel` in `table` (default
+    profiles/traffic.json: bytes per launch from one ncu capture), if it was
+    taken on `workload` and the kernel's source file (relative to the
+    repository root) still has the recorded hash; else None."""
     import hashlib
     root = os.path.dirname(os.path.abspath(__file__))
     try:
-        with open(os.path.join(root, source), "rb") as f:
+        with open(table or os.path.join(root, "profiles", "traffic.json")) as f:
+            rec = json.load(f).get(kernel)
+        if not rec or rec.get("workload") != workload:
+            return None
+        with open(os.path.join(root, rec["source"]), "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()
-        with open(os.path.join(root, summary)) as f:
-            for line in f:
-                parts = line.split()
-                if len(parts) == 4 and parts[0] == "traffic_bytes_per_launch" and parts[1] == kernel:
-                    if sha.startswith(parts[3]):
-                        return int(parts[2])
-    except OSError:
+        return rec if sha.startswith(rec["sha256_prefix"]) else None
+    except (OSError, ValueError, KeyError):
         return None
-    return None
 
 
 def pk_fp32(pk):

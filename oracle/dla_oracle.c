@@ -29,7 +29,7 @@
  *   read-out             o_t = sum_i lambda_{t,i} S_i q_t over the cache after
  *                        token t                                Eq. (capacity_bounded_output)
  *
- * Readings where the paper is silent or inconsistent (listed in the design doc):
+ * Readings taken where the paper is silent or inconsistent:
  *   first token opens state 0 with I_0 = 0; the boundary token's score goes to
  *   the state it opens; the capacity counts the open state; the argmin takes
  *   the lowest index on exact ties; lambda NULL means all ones; the state a

@@ -1,7 +1,7 @@
 """Helpers of the GPU parity tests: run the CUDA path through the C ABI and the
 fp64 oracle on the same seeded inputs and compare them.
 
-Bar (stated in the design doc): boundary flags, merge indices, live-state counts,
+Bar: boundary flags, merge indices, live-state counts,
 token counts and logical slot order bit-exact; outputs and states within
 max-abs 2e-2 for bf16 inputs and 1e-4 for fp32 inputs; summed scores Ibar
 within a relative error well below the tie margin of the input generator.

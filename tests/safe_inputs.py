@@ -13,7 +13,11 @@ oracle and
       token and replays from a checkpoint (G3).
 
 Redraws come from generators keyed by (seed, b, h, t, attempt), so the result
-is reproducible.  The margins are the ones stated in the design doc.
+is reproducible.  THR_MARGIN is 1e-3 relative.  TIE_MARGIN is 1e-5 relative:
+a 1e-3 tie margin admits almost no streams (the pair densities of a full cache
+of i.i.d. tokens crowd into a band about 1e-3 wide), while the device's summed
+scores differ from the oracle's by at most ~2.5e-8 relative, so 1e-5 keeps a
+safety factor of 400.
 """
 from __future__ import annotations
 

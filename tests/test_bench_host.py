@@ -48,20 +48,31 @@ def test_reference_arm_prints_one_json_line():
     assert d["cpu_baseline"]["kind"] == "oracle"
 
 
-def test_captured_traffic_follows_the_source_hash(tmp_path, monkeypatch):
-    """The roofline's DRAM traffic comes from a profile summary line only while
-    the kernel source still has the hash recorded beside it."""
+def test_captured_traffic_follows_the_source_hash(tmp_path):
+    """The roofline's DRAM traffic comes from the traffic table only while the
+    kernel source still has the hash recorded beside it and the workload is the
+    one captured."""
     import hashlib
     import bench
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     src = tmp_path / "kernel.cu"
     src.write_text("// kernel source\n")
     sha = hashlib.sha256(src.read_bytes()).hexdigest()
-    summ = tmp_path / "summary.md"
-    summ.write_text(f"text\ntraffic_bytes_per_launch my_kernel 123456 {sha[:16]}\n")
-    rel = lambda p: os.path.relpath(str(p), root)
-    assert bench.captured_traffic("my_kernel", rel(src), rel(summ)) == 123456
-    assert bench.captured_traffic("other_kernel", rel(src), rel(summ)) is None
+    table = tmp_path / "traffic.json"
+    rec = {"source": os.path.relpath(str(src), ROOT), "sha256_prefix": sha[:16], "workload": "w B1",
+           "bytes_per_launch": 123456, "summary": "s.md"}
+    table.write_text(json.dumps({"my_kernel": rec}))
+    assert bench.captured_traffic("my_kernel", "w B1", str(table))["bytes_per_launch"] == 123456
+    assert bench.captured_traffic("other_kernel", "w B1", str(table)) is None
+    assert bench.captured_traffic("my_kernel", "w B2", str(table)) is None
     src.write_text("// kernel source, changed\n")
-    assert bench.captured_traffic("my_kernel", rel(src), rel(summ)) is None
-    assert bench.captured_traffic("my_kernel", rel(tmp_path / "missing.cu"), rel(summ)) is None
+    assert bench.captured_traffic("my_kernel", "w B1", str(table)) is None
+
+
+def test_committed_traffic_table_is_well_formed():
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        t = json.load(f)
+    for k, rec in t.items():
+        if k.startswith("_"):
+            continue
+        assert set(rec) >= {"source", "sha256_prefix", "workload", "bytes_per_launch", "summary"}
+        assert os.path.exists(os.path.join(ROOT, rec["source"])) and os.path.exists(os.path.join(ROOT, rec["summary"]))

@@ -69,6 +69,24 @@ def test_hand_example_mode1():
     assert b == 0 and j == -1
 
 
+def test_hand_example_mode1_at_a_merge():
+    """Eq. importance_score read literally, at a token that opens a boundary on a
+    full cache (Algorithm 2 merge), values derived by hand."""
+    g = json.load(open(os.path.join(GOLD, "hand_example.json")))
+    h = g["mode1_merge"]
+    st = oracle.Stream(h["C"], 2, 2, tau=h["tau"], eps=0.0, rms_eps=0.0, score_mode=1)
+    K = np.array(g["tokens_k"], float)
+    V = np.array(g["tokens_v"], float)
+    for t in range(3):
+        I, b, j = st.step(K[t], V[t])
+        assert I == pytest.approx(h["I"][t], abs=1e-15)
+        assert b == h["boundary"][t] and j == h["merge"][t]
+    ex = st.export()
+    np.testing.assert_array_equal(ex["states"], np.array(h["after_t2_states"], float))
+    np.testing.assert_array_equal(ex["n"], h["after_t2_n"])
+    np.testing.assert_allclose(ex["ibar"], h["after_t2_ibar"], rtol=0, atol=1e-15)
+
+
 # ------------------------------------------------------------------ closed forms of the score
 
 def _rms(x2, D, e):
@@ -215,9 +233,10 @@ def test_uncapped_dla_i_segment_sums():
 
 # ------------------------------------------------------------------ brute force on tiny inputs
 
+@pytest.mark.parametrize("mode", [0, 1])
 @pytest.mark.parametrize("C", [2, 3, 4])
 @pytest.mark.parametrize("seed", [0, 1, 2])
-def test_merge_brute_force(C, seed):
+def test_merge_brute_force(C, seed, mode):
     """Algorithm 2 step by step: before every token recompute from the exported
     cache what must happen (merge iff boundary and |M| = C; i* = argmin of the
     adjacent pair densities, lowest index on ties; S, n, Ibar summed; rest
@@ -225,8 +244,8 @@ def test_merge_brute_force(C, seed):
     rng = np.random.default_rng(100 + seed)
     T, d = 64, 3
     q, k, v = _rand_stream(rng, T, d)
-    tau = _median_tau(q, k, v, d)
-    st = oracle.Stream(C, d, d, tau=tau)
+    tau = _median_tau(q, k, v, d) if mode == 0 else 0.25
+    st = oracle.Stream(C, d, d, tau=tau, score_mode=mode)
     merges = 0
     for t in range(T):
         pre = st.export()
@@ -271,6 +290,47 @@ def test_merge_lowest_index_on_exact_tie():
         st.step(np.array([1.0, 0.0]), np.array([0.0, 1.0]))
     I, b, j = st.step(np.array([1.0, 0.0]), np.array([0.0, 1.0]))
     assert b == 1 and j == 0
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("C", [3, 4, 5])
+def test_probe_runner_up_gap_and_rollback_brute_force(C, mode):
+    """orc_probe's merge diagnostics, which the decision-safe input generator
+    relies on: at every token that merges, recompute from the exported cache
+    all C - 1 adjacent pair densities (Algorithm 2's definition), order them by
+    (density, index) and check the best pair, the runner-up density, the
+    relative gap (runner-up - best) / |best| and the first token of the newest
+    state among the two pairs (from the states' token counts, not from the
+    oracle's own token ranges).  The probe must leave the stream unchanged and
+    announce the decision the next step takes, with |I - tau| / tau as margin."""
+    rng = np.random.default_rng(300 + 7 * C + mode)
+    T, d = 96, 3
+    q, k, v = _rand_stream(rng, T, d)
+    tau = _median_tau(q, k, v, d) if mode == 0 else 0.25
+    st = oracle.Stream(C, d, d, tau=tau, score_mode=mode)
+    checked = 0
+    for t in range(T):
+        pre = st.export()
+        r = st.probe(k[t], v[t])
+        assert st.export()["m"] == pre["m"] and st.t == t
+        I, b, j = st.step(k[t], v[t])
+        assert (r["boundary"], r["merge"]) == (b, j)
+        assert r["I"] == I
+        if t > 0:
+            assert r["thr_margin"] == pytest.approx(abs(I - tau) / tau, rel=1e-12)
+        if j < 0:
+            assert r["rollback_to"] == -1 and math.isinf(r["tie_gap"])
+            continue
+        n, ib = pre["n"].astype(np.int64), pre["ibar"]
+        dens = [((ib[i] + ib[i + 1]) / (n[i] + n[i + 1]), i) for i in range(C - 1)]
+        order = sorted(dens)
+        (bd, bi), (sd, si) = order[0], order[1]
+        assert j == bi and r["best"] == bd and r["runner_up"] == sd
+        assert r["tie_gap"] == pytest.approx((sd - bd) / abs(bd), rel=1e-12, abs=1e-300)
+        newest = max(bi, si) + 1
+        assert r["rollback_to"] == int(n[:newest].sum())
+        checked += 1
+    assert checked >= 5
 
 
 # ------------------------------------------------------------------ invariants
