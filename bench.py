@@ -144,21 +144,28 @@ def kernel_table(timing, steps):
 
 # ---------------------------------------------------------------- prefill
 
-def bench_prefill(args, dist, pk):
+def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headline=True):
+    """One workload's prefill: warm-up, `steps` timed dla_forward calls (the
+    default concurrent schedule), the call's device status checked, the kernels
+    timed alone (serial schedule) and the timed run's decision trace checked
+    against the serial run's.  With `headline`, also the end-to-end figure
+    through dla_forward_host."""
     import numpy as np
     import torch
 
     from paper_2606_10650_gb300 import dla
     from paper_2606_10650_gb300 import workloads as W
 
+    workload = workload or args.workload
+    steps = args.steps if steps is None else steps
+    warmup = args.warmup if warmup is None else warmup
     dev = torch.device("cuda", dist.local)
     torch.cuda.set_device(dev)
-    w = W.get(args.workload)
-    if args.T:
-        w = W.get(args.workload, T=args.T)
-    q, k, v, lam = W.host_batch(w, T=w.T)
+    w = W.get(workload, **({"T": args.T} if (args.T and headline) else {}))
+    q, k, v, lam = W.host_batch_parallel(w, T=w.T)
     qt, kt, vt = (W.to_device(x, w.dtype, dev) for x in (q, k, v))
-    lt = torch.from_numpy(lam.astype(np.float32)).to(dev)
+    lt = torch.from_numpy(lam).to(dev)
+    del q, k, v, lam
     B, T, H, d = kt.shape
     p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
     in_code = dla.DLA_BF16 if w.dtype == "bf16" else dla.DLA_F32
@@ -176,41 +183,52 @@ def bench_prefill(args, dist, pk):
     def step():
         dla.dla_forward(p, qt, kt, vt, lt, o, cache, bnd, ml, workspace=ws, stream=stream)
 
-    for _ in range(args.warmup):
+    def check_status(what):
+        st = dla.dla_sync_status(stream)
+        if st != 0 or dla.workspace_status(ws) != 0:
+            raise RuntimeError(f"{workload}: device status {st} after {what} (a bounded wait gave up or a "
+                               "device check failed): the timing would not be valid")
+
+    for _ in range(warmup):
         step()
     torch.cuda.synchronize()
+    check_status("the warm-up steps")
     dla.dla_timing_read(reset=True)
-    clocks = Clocks(dist.local)
-    clocks.start()
+    clocks = Clocks(dist.local) if headline else None
+    if clocks:
+        clocks.start()
     dist.barrier()
     torch.cuda.synchronize()
     dla.dla_timing_enable(True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
+    for _ in range(steps):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
     dla.dla_timing_enable(False)
     dist.barrier()
-    clk = clocks.stop()
-    ms = e0.elapsed_time(e1) / args.steps
+    clk = clocks.stop() if clocks else None
+    ms = e0.elapsed_time(e1) / steps
     timing = dla.dla_timing_read(reset=True)
+    check_status("the timed steps")
     ms_max = dist.reduce(ms, "max")
     tokens = B * T
+    # the timed run's decisions, checked below against a serial-schedule run
+    timed_trace = (bnd.clone(), ml.clone(), cache.view("m").clone(), cache.view("n").clone())
     # algorithmic work from the decision trace: m_t = live states after token t
     m_t = torch.cumsum(bnd.to(torch.int64), 2) - torch.cumsum((ml >= 0).to(torch.int64), 2)
     sum_m = int(m_t.sum().item())
+    del m_t
     BH = B * H
-    flops_readout = 2.0 * d * d * sum_m
     flops_total = 2.0 * d * d * (sum_m + 2 * T * BH)
-    kt_tab = kernel_table(timing, args.steps)
+    kt_tab = kernel_table(timing, steps)
     tc_path = (w.dtype == "bf16" and d == 128)
     # Each kernel alone on the device: the same forward pass under the serial
     # schedule (pre-pass, scan, read-out one after another), timed after the
     # step.  Inside the step the kernels overlap and the read-out is paced by
     # the scan, so their in-step durations are not their speeds.
-    solo, solo_steps = {}, min(args.steps, 5)
+    solo, solo_steps, validated = {}, min(steps, 5), None
     if tc_path:
         os.environ["DLA_SCHEDULE"] = "serial"
         try:
@@ -223,17 +241,25 @@ def bench_prefill(args, dist, pk):
             torch.cuda.synchronize()
             dla.dla_timing_enable(False)
             solo = dla.dla_timing_read(reset=True)
+            check_status("the serial-schedule steps")
         finally:
             os.environ.pop("DLA_SCHEDULE", None)
-    t_in = {k: (n, ms) for k, (n, ms) in timing.items()}
+        same = [torch.equal(a_, b_) for a_, b_ in zip(timed_trace, (bnd, ml, cache.view("m"), cache.view("n")))]
+        if not all(same):
+            raise RuntimeError(f"{workload}: the timed run's decisions differ from the serial schedule's "
+                               f"(boundary, merge_log, m, n equal: {same})")
+        validated = ("device status 0 after the warm-up, timed and serial steps; the timed run's boundary flags, "
+                     "merge indices and final live / token counts equal a serial-schedule run on the same inputs")
+    del timed_trace
+    t_in = {k_: (n_, ms_) for k_, (n_, ms_) in timing.items()}
     fp32_peak = pk_fp32(pk)
     rooflines, sm_ms = {}, {}
     n_sms = 152
     scan_sms = 2 * BH if 2 * BH <= n_sms else min(BH, n_sms)
 
     def per_launch(table, name):
-        n, ms_ = table.get(name, (0, 0.0))
-        return (ms_ / n) if n else None
+        n_, ms_ = table.get(name, (0, 0.0))
+        return (ms_ / n_) if n_ else None
 
     for name in ("readout", "scan", "gram"):
         t_solo = per_launch(solo, name) if solo else None
@@ -241,7 +267,7 @@ def bench_prefill(args, dist, pk):
         t = t_solo if t_solo is not None else t_step
         if t is None:
             continue
-        n_launch = t_in.get(name, (0, 0.0))[0] / args.steps  # launches per step inside the timed region
+        n_launch = t_in.get(name, (0, 0.0))[0] / steps  # launches per step inside the timed region
         timing_note = (f"CUDA events around each launch of the kernel alone on the device (serial schedule, "
                        f"{solo_steps} forward passes after the timed steps); inside the timed step it lasts "
                        f"{t_step:.4f} ms per launch, overlapped" if t_solo is not None else
@@ -268,8 +294,8 @@ def bench_prefill(args, dist, pk):
                 "kernel": "scan (K1)", "bound": "tensor" if tc_path else "alu", "achieved": round(ach, 3),
                 "peak": round(peak, 2), "unit": "TFLOP/s", "frac": round(ach / peak, 4), "traffic": None,
                 "ms_per_launch": round(t, 5),
-                "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json; the scan's contractions "
-                              "run on mma.sync" if tc_path else "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
+                "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else
+                              "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
                 "work_per_launch": f"4*d^2*T*B*H / launches = {work:.4g} flop", "timing": timing_note,
                 "note": (f"latency-bound: each (batch, head) stream is sequential; {scan_sms} CTAs "
                          f"({'pairs' if scan_sms == 2 * BH else 'one per stream'})")}
@@ -284,29 +310,29 @@ def bench_prefill(args, dist, pk):
                 "work_per_launch": f"k, v read (bf16) + Gram tables written (fp32) = {work:.4g} bytes",
                 "timing": timing_note}
             sm_ms[name] = t * n_launch * n_sms
-    # DRAM traffic per launch from a committed ncu summary, while the kernel's source is the one
+    # DRAM traffic per launch from profiles/traffic.json, while the kernel's source is the one
     # captured and the workload is the one captured (else null)
-    tr = captured_traffic("readout_tc_kernel", f"{args.workload} B{B} H{H} T{T} d{d}")
+    tr = captured_traffic("readout_tc_kernel", f"{workload} B{B} H{H} T{T} d{d}")
     if tr and "readout" in rooflines and tc_path:
         rooflines["readout"]["traffic"] = tr["bytes_per_launch"]
         rooflines["readout"]["traffic_note"] = ("dram__bytes_read.sum + dram__bytes_write.sum of one full-size "
                                                 f"launch (ncu, {tr['summary']})")
     # dominant kernel: the largest SM-time per step (duration alone x SMs it occupies); the
     # step is close to the summed SM-time of the kernels over the 152 SMs
-    dominant = max(sm_ms, key=lambda k: sm_ms[k]) if sm_ms else None
+    dominant = max(sm_ms, key=lambda k_: sm_ms[k_]) if sm_ms else None
     roof = dict(rooflines[dominant]) if dominant else None
     if roof is not None:
         roof["dominance"] = ("largest SM-time per step (ms alone x SMs occupied): " +
-                             ", ".join(f"{k} {v:.1f} SM-ms" for k, v in sm_ms.items()))
+                             ", ".join(f"{k_} {v_:.1f} SM-ms" for k_, v_ in sm_ms.items()))
     # end to end through the C ABI with host buffers: every step, dla_forward_host
     # copies q, k, v, lambda in from page-locked host memory (piece by piece beside
     # the scan on the concurrent schedule), runs the forward pass and copies o back
     e2e = None
-    if not args.no_e2e:
+    if headline and not args.no_e2e:
         qh, kh, vh = (x.cpu().pin_memory() for x in (qt, kt, vt))
         lh = lt.cpu().pin_memory()
         oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
-        n_e2e = max(2, min(args.steps, 10))
+        n_e2e = max(2, min(steps, 10))
         hnb = dla.dla_forward_host_workspace(p, B, T, H, d, d, in_code, True)
         hbuf = torch.empty(hnb + 256, dtype=torch.uint8, device=dev)
         hws = (hbuf, (hbuf.data_ptr() + 255) // 256 * 256, hnb)
@@ -316,8 +342,8 @@ def bench_prefill(args, dist, pk):
 
         e2e_step()
         torch.cuda.synchronize()
-        if dla.workspace_status(hws) != 0:
-            raise RuntimeError("dla_forward_host: device status word reports a failure")
+        if dla.dla_sync_status(stream) != 0 or dla.workspace_status(hws) != 0:
+            raise RuntimeError("dla_forward_host: device status reports a failure")
         dist.barrier()
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a0.record(stream)
@@ -325,6 +351,8 @@ def bench_prefill(args, dist, pk):
             e2e_step()
         a1.record(stream)
         torch.cuda.synchronize()
+        if dla.dla_sync_status(stream) != 0:
+            raise RuntimeError("dla_forward_host: device status reports a failure in the timed steps")
         e_ms = dist.reduce(a0.elapsed_time(a1) / n_e2e, "max")
         hb = sum(x.numel() * x.element_size() for x in (qh, kh, vh, lh))
         e2e = {"value": round(dist.world * tokens / (e_ms * 1e-3), 1), "unit": "tokens/s", "ms_per_step": round(e_ms, 4),
@@ -334,10 +362,11 @@ def bench_prefill(args, dist, pk):
     res = {"value": dist.world * tokens / (ms_max * 1e-3), "ms_per_step": ms_max, "tokens_per_step": tokens,
            "roofline": roof, "rooflines": rooflines, "kernels": kt_tab,
            "kernels_alone": kernel_table(solo, solo_steps) if solo else None, "tc_path": tc_path, "clocks": clk,
-           "e2e": e2e,
-           "gpu_launches": sum(n for n, _ in timing.values()),
+           "e2e": e2e, "validated": validated, "steps": steps,
+           "gpu_launches": sum(n_ for n_, _ in timing.values()),
            "algorithmic_tflops": flops_total / (ms_max * 1e-3) / 1e12, "sum_m": sum_m,
-           "boundaries": int(bnd.sum().item()), "merges": int((ml >= 0).sum().item())}
+           "boundaries": int(bnd.sum().item()), "merges": int((ml >= 0).sum().item()),
+           "workload": f"{w.name}: B={w.B} H={w.H} T={w.T} d={w.d} C={w.C} {w.dtype} inputs, fp32 states"}
     del qt, kt, vt, lt, o, buf, cache
     torch.cuda.empty_cache()
     return res
@@ -424,6 +453,8 @@ def bench_decode(args, dist, pk):
     dist.barrier()
     ms = dist.reduce(e0.elapsed_time(e1) / args.steps, "max")
     timing = dla.dla_timing_read(reset=True)
+    if dla.dla_sync_status(stream) != 0:
+        raise RuntimeError("decode: device status reports a failure in the timed steps")
     dn, dms = timing["decode"]
     achieved = bytes_per_step / (dms / dn * 1e-3) / 1e9
     roof = {"kernel": "decode", "bound": "hbm", "achieved": round(achieved, 1), "peak": pk["hbm"], "unit": "GB/s",
@@ -551,6 +582,7 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the standard and long prefill lines")
     ap.add_argument("--decode-batch", type=int, default=0)
     ap.add_argument("--ws-gb", type=float, default=0.0, help="cap the prefill workspace (GiB)")
     ap.add_argument("--cpu-tokens", type=int, default=8192)
@@ -566,6 +598,17 @@ def main():
     __graft_entry__.build()
     pk = peaks()
     pre = None if args.no_prefill else bench_prefill(args, dist, pk)
+    others = {}
+    if not (args.no_prefill or args.no_configs):
+        for name in ("standard", "long"):  # the other prefill workloads, fewer steps
+            r = bench_prefill(args, dist, pk, workload=name, steps=min(args.steps, 10), warmup=max(args.warmup, 3),
+                              headline=False)
+            others[name] = {k_: r[k_] for k_ in ("workload", "value", "ms_per_step", "steps", "roofline",
+                                                 "kernels_alone", "validated", "gpu_launches", "algorithmic_tflops",
+                                                 "boundaries", "merges", "sum_m")}
+            others[name]["value"] = round(others[name]["value"], 1)
+            others[name]["unit"] = "tokens/s"
+            others[name]["algorithmic_frac_of_peak"] = round(r["algorithmic_tflops"] / pk["bf16"], 4)
     dec = None if args.no_decode else bench_decode(args, dist, pk)
     cpu = cpu_baseline(args) if (dist.rank == 0 and dist.world == 1 and not args.no_cpu) else None
     if dist.rank == 0:
@@ -579,7 +622,11 @@ def main():
                         kernels_alone=pre["kernels_alone"], clocks=pre["clocks"], e2e=pre["e2e"],
                         gpu_launches=pre["gpu_launches"],
                         algorithmic_tflops=round(pre["algorithmic_tflops"], 3),
+                        algorithmic_frac_of_peak=round(pre["algorithmic_tflops"] / pk["bf16"], 4),
+                        validated=pre["validated"],
                         trace={"sum_m": pre["sum_m"], "boundaries": pre["boundaries"], "merges": pre["merges"]})
+        if others:
+            line["other_prefill_workloads"] = others
         if dec:
             line["decode"] = dec
         line["cpu_baseline"] = cpu

@@ -25,6 +25,22 @@
  *     work is enqueued asynchronously on it; argument errors are returned
  *     synchronously before anything is enqueued.  A launch failure returns
  *     DLA_ERR_CUDA.  No C++ exception crosses this interface.
+ *   - Failures found on the device -- a bounded wait of a kernel that gave up
+ *     (DLA_ERR_TIMEOUT) or an inconsistent cache or snapshot list
+ *     (DLA_ERR_DEVICE_CHECK) -- cannot be returned by the call that enqueued
+ *     the work.  Each call folds its device status into a status word of its
+ *     stream (the first failure since the last read sticks), and
+ *     dla_sync_status(stream) waits for the stream and returns that status.
+ *     dla_forward also leaves its own call's status in its workspace.  After a
+ *     device failure the call's outputs and cache are undefined; the library
+ *     stays usable (every wait is bounded, no kernel traps).  Two environment
+ *     variables, read at every call and unset in normal use, exist for tests
+ *     of this path: DLA_DEBUG_WAIT_MS=x makes every bounded wait give up after
+ *     about x ms instead of about 2 s, and DLA_DEBUG_WITHHOLD_PIECES=1 makes
+ *     dla_forward_host report only its first input piece as arrived.
+ *   - The first call on each device from each host thread creates that
+ *     thread's internal streams and events and looks up the device address
+ *     of the library's status words; make it before any stream capture.
  *   - Layouts are row-major and contiguous:
  *       q, k, v   [B, T, H, d]   (bf16 or fp32, see dla_dtype)
  *       lambda    [B, T, H, C]   fp32, logical cache slot i = 0 is the oldest
@@ -51,7 +67,7 @@
 extern "C" {
 #endif
 
-#define DLA_VERSION 1
+#define DLA_VERSION 2
 
 typedef enum {
   DLA_OK = 0,
@@ -134,6 +150,17 @@ size_t dla_forward_workspace(const dla_params* p, int B, int T, int H, int dk, i
 size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int dk, int dv,
                                  dla_dtype in_dtype, int with_output);
 
+/* Waits for `stream` (a cudaStream_t) to complete its work, then returns the
+ * device status of the library's calls enqueued on it since the previous
+ * dla_sync_status on that stream, and clears it: DLA_OK, DLA_ERR_TIMEOUT (a
+ * bounded device wait gave up) or DLA_ERR_DEVICE_CHECK (a kernel found an
+ * inconsistent cache, snapshot list or pool); DLA_ERR_CUDA if the stream
+ * could not be synchronised.  Each status word belongs to a (device, stream)
+ * pair; a device keeps 255 of them for its first 255 streams and one shared
+ * word for every later stream.  A stream handle that is destroyed and reused
+ * inherits an unread status. */
+dla_status dla_sync_status(void* stream);
+
 /* Prefill / training-shaped forward over T tokens of B x H streams
  * (Algorithm 1 + Algorithm 2 + Eq. capacity_bounded_output).
  *   q, k, v, lam, o, boundary, merge_log: layouts above; o, lam, boundary and
@@ -146,7 +173,7 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
  *   Its first 4 bytes receive the device status of the call once the work has
  *   run (int32: 0 ok, DLA_ERR_TIMEOUT when a bounded wait of a kernel gave up,
  *   DLA_ERR_DEVICE_CHECK when a kernel found an inconsistent cache or pool);
- *   read them after synchronising the stream.
+ *   the same status goes to the stream's status word (dla_sync_status).
  *   Schedule (bf16, d = 128, workspace of at least dla_forward_workspace(...)):
  *   the environment variable DLA_SCHEDULE, read at every call, selects
  *   "concurrent" (default: the scan runs once over the whole sequence while
@@ -174,14 +201,18 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
  * 64 MiB compiled into the library, which every GPU that loads the library
  * holds until the process exits.  It allocates nothing.
  *   - The first call on each device (with that device current) looks up the
- *     array's device address with cudaGetSymbolAddress; make that first call
- *     before any stream capture.
+ *     array's device address with cudaGetSymbolAddress, and the first call
+ *     from each host thread creates that thread's internal streams and events
+ *     (as for dla_forward); make those first calls before any stream capture.
  *   - A call whose workspace need exceeds 64 MiB returns DLA_ERR_WORKSPACE with
  *     a message naming the limit; pass your own `cache` (and boundary /
  *     merge_log arrays) to keep the need small, or use dla_forward.
  *   - Every call shares the one array and rewrites the parts it reads; calls
  *     that overlap on the GPU (different streams, or different host threads,
- *     on the same device) race on it and must be serialised by the caller. */
+ *     on the same device) race on it and must be serialised by the caller.
+ *   - The call's device status (a bounded wait that gave up, a failed device
+ *     check) goes to its stream's status word: read it with
+ *     dla_sync_status(stream). */
 dla_status dla_forward_noalloc(const dla_params* p, dla_dtype in_dtype, int B, int T, int H,
                                int dk, int dv, const void* q, const void* k, const void* v,
                                const float* lam, void* o, const dla_cache* cache,
@@ -221,14 +252,17 @@ dla_status dla_forward_host(const dla_params* p, dla_dtype in_dtype, int B, int 
  * every stream: token (q, k, v) [B, H, d] against the persistent cache, which
  * is updated in place.  lam [B, H, C] fp32 or NULL; o [B, H, d] (out_dtype);
  * boundary [B, H] uint8 or NULL; merge_idx [B, H] int32 (i* or -1) or NULL.
- * p->capacity must equal cache->C. */
+ * p->capacity must equal cache->C.  A cache whose live count or slot map is
+ * out of range is clamped and reported as DLA_ERR_DEVICE_CHECK through the
+ * stream's status word (dla_sync_status). */
 dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtype in_dtype,
                            const void* q, const void* k, const void* v, const float* lam,
                            void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
 
 /* Instrumentation (no counterpart in the paper).  Kernel kinds of the
- * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass, and
- * the one-thread gate of the concurrent schedule. */
+ * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass, the
+ * one-thread gate of the concurrent schedule, and the one-thread kernel that
+ * folds a forward call's status into its stream's status word. */
 typedef enum {
   DLA_K_SCAN = 0,
   DLA_K_READOUT = 1,
@@ -236,7 +270,8 @@ typedef enum {
   DLA_K_INIT = 3,
   DLA_K_GRAM = 4,
   DLA_K_GATE = 5,
-  DLA_K_COUNT = 6
+  DLA_K_STATUS = 6,
+  DLA_K_COUNT = 7
 } dla_kernel_kind;
 
 /* enable = 1: from now on, every kernel this host thread launches through the

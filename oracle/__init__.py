@@ -124,10 +124,11 @@ class Stream:
     def probe(self, k, v) -> dict:
         """The decision ``step`` would take, with its margins; no state change."""
         k, v = _f64(k), _f64(v)
-        out = np.zeros(8)
+        out = np.zeros(9)
         lib().orc_probe(self._h, _p(k), _p(v), _p(out))
         return dict(I=out[0], boundary=int(out[1]), merge=int(out[2]), best=out[3],
-                    runner_up=out[4], thr_margin=out[5], tie_gap=out[6], rollback_to=int(out[7]))
+                    runner_up=out[4], thr_margin=out[5], tie_gap=out[6], rollback_to=int(out[7]),
+                    rollback_last=int(out[8]))
 
     def readout(self, q, lam=None) -> np.ndarray:
         """o = sum_i lambda_i S_i q over the current cache (Eq. capacity_bounded_output)."""

@@ -234,14 +234,15 @@ int orc_step(orc_stream *st, const double *k, const double *v, double *I_out,
  * density, out[4] runner-up density (or +inf), out[5] relative threshold
  * margin |I - tau| / tau (inf for the first token), out[6] relative gap
  * (runner-up - best) / |best| (inf when no merge happens), out[7] first token
- * of the newest state among the best and runner-up pairs (-1 when no merge).
+ * of the newest state among the best and runner-up pairs (-1 when no merge),
+ * out[8] the last token of that state (-1 when no merge).  out must hold 9.
  */
 int orc_probe(orc_stream *st, const double *k, const double *v, double *out) {
   double *s = st->s_tok;
   token_state(st, k, v, s);
-  for (int e = 0; e < 8; ++e) out[e] = 0.0;
+  for (int e = 0; e < 9; ++e) out[e] = 0.0;
   out[2] = -1.0; out[4] = INFINITY; out[5] = INFINITY; out[6] = INFINITY;
-  out[7] = -1.0;
+  out[7] = -1.0; out[8] = -1.0;
   if (st->m == 0) { out[1] = 1.0; return 0; }
   double I = score_token(st, s);
   int b = (I >= st->tau) ? 1 : 0;
@@ -257,6 +258,7 @@ int orc_probe(orc_stream *st, const double *k, const double *v, double *out) {
       out[6] = (sd - bd) / scale;
       int newest = (j > sec ? j : sec) + 1;
       out[7] = (double)st->first[newest];
+      out[8] = (double)st->last[newest];
     }
   }
   return 0;

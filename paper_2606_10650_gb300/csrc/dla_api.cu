@@ -259,6 +259,76 @@ cudaError_t stream_set(StreamSet** out) {
   return cudaSuccess;
 }
 
+// ---- device status of each stream (dla_sync_status)
+// One word per (device, stream) in a static device array of the library
+// (nothing is allocated): every call folds its device status into its
+// stream's word (the first failure sticks) and dla_sync_status reads and
+// clears it.  Streams are given words in the order they are first used; past
+// kStatusWords - 1 streams on a device, the rest share the last word.
+constexpr int kStatusWords = 256;
+static __device__ int32_t g_status_board[kStatusWords];
+
+struct StatusBoard {
+  std::mutex mu;
+  int32_t* base = nullptr;  // device address of g_status_board on this device
+  std::vector<std::pair<cudaStream_t, int>> words;
+};
+StatusBoard g_board[64];
+
+// The first failure of a call (its workspace status word) into its stream's word.
+__global__ void status_fold_kernel(const int32_t* call_status, int32_t* word) {
+  const int v = *(volatile const int32_t*)call_status;
+  if (v != 0) atomicCAS(word, 0, v);
+}
+
+// Device address of the status word of `s` on the current device.
+cudaError_t status_word(cudaStream_t s, int32_t** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  StatusBoard& B = g_board[dev];
+  std::lock_guard<std::mutex> g(B.mu);
+  if (!B.base) {
+    // the module holding the board and the fold kernel is loaded here, before
+    // any kernel of the call that might wait on another is enqueued
+    cudaFuncAttributes fa;
+    if ((e = cudaFuncGetAttributes(&fa, status_fold_kernel)) != cudaSuccess) return e;
+    void* a = nullptr;
+    if ((e = cudaGetSymbolAddress(&a, g_status_board)) != cudaSuccess) return e;
+    B.base = (int32_t*)a;
+  }
+  int w = -1;
+  for (const auto& p : B.words)
+    if (p.first == s) w = p.second;
+  if (w < 0) {
+    w = (int)B.words.size() < kStatusWords - 1 ? (int)B.words.size() : kStatusWords - 1;
+    B.words.emplace_back(s, w);
+  }
+  *out = B.base + w;
+  return cudaSuccess;
+}
+
+// Debugging knobs of the failure-detection tests (environment variables read at
+// every call; unset in normal use):
+//   DLA_DEBUG_WAIT_MS=x       bounded device waits give up after about x ms
+//                             instead of about 2 s;
+//   DLA_DEBUG_WITHHOLD_PIECES=1  dla_forward_host copies every input piece but
+//                             reports only the first as arrived, so a scan
+//                             waiting for a later piece gives up (status 5).
+int debug_wait_units() {  // the wait limit in units of 1024 SM clocks (0: default)
+  const char* v = getenv("DLA_DEBUG_WAIT_MS");
+  if (!v) return 0;
+  const double ms = atof(v);
+  if (!(ms > 0.0)) return 0;
+  const double units = ms * 2.07e6 / 1024.0;  // SM clocks at 2.07 GHz
+  return units < 1.0 ? 1 : (units > 2e9 ? 2000000000 : (int)units);
+}
+bool debug_withhold_pieces() {
+  const char* v = getenv("DLA_DEBUG_WITHHOLD_PIECES");
+  return v && strcmp(v, "1") == 0;
+}
+
 // ---- inputs in host memory (dla_forward_host)
 // A 32-bit write to device memory in stream order, after the stream's earlier
 // work and with a memory barrier before it (the driver's stream memory
@@ -424,6 +494,27 @@ dla_status dla_timing_read(int* launches, double* ms, int reset) {
   return ok();
 }
 
+dla_status dla_sync_status(void* stream) {
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  int32_t* word = nullptr;
+  if ((e = status_word(s, &word)) != cudaSuccess) return cuda_fail(e, "status word");
+  int32_t v = 0;
+  if ((e = cudaMemcpyAsync(&v, word, sizeof(v), cudaMemcpyDeviceToHost, s)) != cudaSuccess ||
+      (e = cudaMemsetAsync(word, 0, sizeof(int32_t), s)) != cudaSuccess || (e = cudaStreamSynchronize(s)) != cudaSuccess)
+    return cuda_fail(e, "status read");
+  switch (v) {
+    case 0: return ok();
+    case DLA_ERR_TIMEOUT:
+      return fail(DLA_ERR_TIMEOUT, "a bounded device wait gave up in a call on this stream (its outputs are undefined)");
+    case DLA_ERR_DEVICE_CHECK:
+      return fail(DLA_ERR_DEVICE_CHECK, "a device-side consistency check failed in a call on this stream");
+    default:
+      return fail(DLA_ERR_DEVICE_CHECK, "unexpected device status %d on this stream", v);
+  }
+}
+
 const char* dla_last_error(void) { return g_err; }
 
 const char* dla_status_string(dla_status s) {
@@ -519,10 +610,33 @@ static int concurrent_free_sms(int B, int H, int d, cudaError_t* err) {
 // dla_forward; with io, q, k, v and lambda come from host memory into the
 // device buffers q, k, v, lam (workspace), streamed beside the scan on the
 // concurrent schedule, otherwise copied before anything else.
+static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
+                                 const void* q, const void* k, const void* v, const float* lam, void* o,
+                                 const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
+                                 size_t ws_bytes, void* stream, HostIO* io, int32_t** word);
+
+// forward_launch, then the call's device status folded into its stream's status
+// word once every kernel of the call has run (the stream waits for them).
 static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
                                const void* q, const void* k, const void* v, const float* lam, void* o,
                                const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
                                size_t ws_bytes, void* stream, HostIO* io) {
+  int32_t* word = nullptr;
+  dla_status s = forward_launch(p, in_dtype, B, T, H, dk, dv, q, k, v, lam, o, cache, boundary, merge_log, workspace,
+                                ws_bytes, stream, io, &word);
+  if (s != DLA_OK) return s;
+  cudaError_t e = timed(DLA_K_STATUS, (cudaStream_t)stream, [&] {
+    status_fold_kernel<<<1, 1, 0, (cudaStream_t)stream>>>((const int32_t*)workspace, word);
+    return cudaGetLastError();
+  });
+  if (e != cudaSuccess) return cuda_fail(e, "status fold launch");
+  return ok();
+}
+
+static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
+                                 const void* q, const void* k, const void* v, const float* lam, void* o,
+                                 const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
+                                 size_t ws_bytes, void* stream, HostIO* io, int32_t** word) {
   dla_status s = check_params(p);
   if (s != DLA_OK) return s;
   if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
@@ -573,8 +687,17 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
   } else {
     dla_cache_carve(ws + P.off_cache, cache_layout(B, H, C, d, d).total, B, H, C, d, d, &live);
   }
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);
+  // the stream's status word (looked up before anything is enqueued), the call's
+  // status word and, after it, the wait limit of its kernels (0: default)
+  cudaError_t e = status_word(st, word);
+  if (e != cudaSuccess) return cuda_fail(e, "status word");
+  e = cudaMemsetAsync(status, 0, 2 * sizeof(int32_t), st);
   if (e != cudaSuccess) return cuda_fail(e, "status reset");
+  if (const int wu = debug_wait_units()) {
+    if (!write_value_fn() ||
+        write_value_fn()((CUstream)st, (CUdeviceptr)(status + 1), (cuuint32_t)wu, 0) != CUDA_SUCCESS)
+      return fail(DLA_ERR_CUDA, "stream memory write of the debug wait limit failed");
+  }
   if (!p->from_cache) {
     e = timed(DLA_K_INIT, st, [&] { return dla::launch_init_cache(live.slot, live.n, live.ibar, live.m, B * H, C, st); });
     if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
@@ -724,10 +847,12 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
     // the count of pieces in place (a stream memory write); the scan waits for
     // the piece of each chunk it loads, the read-out for the scan.
     int pc = 0, npiece = 0;
+    const bool withhold = stream_in && debug_withhold_pieces();
     auto put_piece = [&](int pi) -> dla_status {
       const int t0 = pi * pc * dla::kScanL, t1 = std::min(T, (pi + 1) * pc * dla::kScanL);
       const cudaError_t ce = h2d_tokens(*io, B, T, H, d, C, t0, t1, S->cp);
       if (ce != cudaSuccess) return cuda_fail(ce, "input copy");
+      if (pi > 0 && withhold) return DLA_OK;  // debugging: later pieces never reported
       if (write_value_fn()((CUstream)S->cp, (CUdeviceptr)pieces, (cuuint32_t)(pi + 1), 0) != CUDA_SUCCESS)
         return fail(DLA_ERR_CUDA, "stream memory write failed");
       return DLA_OK;
@@ -965,7 +1090,9 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
   dla::finish_score_params(da.sp);
   da.states = cache->states; da.slot = cache->slot; da.n = cache->n; da.ibar = cache->ibar; da.m = cache->m;
   da.boundary = boundary; da.merge_idx = merge_idx;
-  cudaError_t e = timed(DLA_K_DECODE, (cudaStream_t)stream,
+  cudaError_t e = status_word((cudaStream_t)stream, &da.status);
+  if (e != cudaSuccess) return cuda_fail(e, "status word");
+  e = timed(DLA_K_DECODE, (cudaStream_t)stream,
                         [&] { return dla::launch_decode(da, cache->dk, in_dtype == DLA_BF16, (cudaStream_t)stream); });
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   return ok();

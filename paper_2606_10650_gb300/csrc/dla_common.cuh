@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include "dla_kernels.h"
+#include "dla_sm100.cuh"
 
 namespace dla {
 
@@ -79,12 +80,6 @@ __device__ __forceinline__ int ld_acquire_gpu(const int32_t* p) {
 __device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
   asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
-// Read-out side: thread 0 waits until the scan CTAs of stream bh have completed
-// `need` intervals (progress[bh][0 .. ctas)), at most ~2 s (then status 5)
-// and not once the status word reports a failure;
-// the caller's CTA barrier then orders every later read after the wait.  Data
-// the scan writes must then be read past L1 (__ldcg): another CTA on the SM may
-// hold an older copy of the line.
 // This stream's end of the round [t_begin, t_end): the call's t_end, or, with
 // per-row lengths, row b's length clamped to [t_begin, t_end] (tokens past it
 // are padding).
@@ -100,14 +95,20 @@ __device__ __forceinline__ void fill_padding_trace(uint8_t* bnd, int32_t* mlog, 
   }
 }
 
+// Read-out side: thread 0 waits until the scan CTAs of stream bh have completed
+// `need` intervals (progress[bh][0 .. ctas)), at most the wait limit (then
+// status 5) and not once the status word reports a failure; the caller's CTA
+// barrier then orders every later read after the wait.  Data the scan writes
+// must then be read past L1 (__ldcg): another CTA on the SM may hold an older
+// copy of the line.
 __device__ __forceinline__ void wait_progress(const int32_t* progress, int ctas, int bh, int need, int32_t* status) {
   if (!progress || threadIdx.x != 0) return;
-  const long long t0 = clock64();
+  const long long t0 = clock64(), lim = sm100::wait_limit(status);
   for (int r = 0; r < ctas; ++r)
     while (ld_acquire_gpu(progress + 2 * bh + r) < need) {
       if (*(volatile int32_t*)status != 0) return;  // the call has failed already
-      if (clock64() - t0 > 4000000000LL) {
-        atomicExch(status, 5);
+      if (clock64() - t0 > lim) {
+        atomicCAS(status, 0, sm100::kStatusTimeout);
         return;
       }
     }

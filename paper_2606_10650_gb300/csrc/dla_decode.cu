@@ -52,9 +52,16 @@ __global__ void __launch_bounds__(NT, 2) decode_kernel(DecodeArgs a) {
   const int col = 4 * li;
   float* states = a.states + (long long)bh * C * D * D;
 
-  if (tid == 0) sm.m = min(max(a.m[bh], 0), C);  // a corrupted cache cannot index out of bounds
+  // a corrupted cache is reported (device check) and clamped, so that it
+  // cannot index out of bounds
+  if (tid == 0) {
+    const int m0 = a.m[bh];
+    if ((m0 < 0 || m0 > C) && a.status) atomicCAS(a.status, 0, 6);
+    sm.m = min(max(m0, 0), C);
+  }
   for (int i = tid; i < C; i += NT) {
     const int sl = a.slot[(long long)bh * C + i];
+    if ((sl < 0 || sl >= C) && a.status) atomicCAS(a.status, 0, 6);
     sm.slot[i] = (sl >= 0 && sl < C) ? sl : i;
     sm.n[i] = a.n[(long long)bh * C + i];
     sm.ibar[i] = a.ibar[(long long)bh * C + i];

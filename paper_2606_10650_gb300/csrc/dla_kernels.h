@@ -145,6 +145,7 @@ struct DecodeArgs {
   int32_t* m;
   uint8_t* boundary;     // [B, H] or nullptr
   int32_t* merge_idx;    // [B, H] or nullptr
+  int32_t* status;       // device status word of the call's stream (6 when the cache is inconsistent)
 };
 
 // Records a formatted message as the calling thread's dla_last_error() and

@@ -75,6 +75,7 @@ struct TcSmem {
   uint64_t full[NHS], empty[NHS], acc_full[NBUF], acc_empty[NBUF];
   uint32_t tmem_base;
   int abort_flag;
+  int skip;                    // the call has failed before this CTA's work: do none of it
 };
 
 // Snapshot entries' slot table of one interval (one warp): row e holds L(x) of
@@ -184,16 +185,35 @@ __global__ void __launch_bounds__(NT, 1)
   const bool hasB = (sA + 1) < a.nsnap && (!kRagged || a.t_begin + (sA + 1) * L < t_end);
   // with a scan running concurrently: both intervals of the pair must be complete
   wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + sA + (hasB ? 2 : 1), a.status);
-  // thread 0 issues the TMA loads: they read what the scan wrote (pool entries)
-  // and the inputs streamed in before its progress
-  if (tid == 0 && a.progress) asm volatile("fence.proxy.async.global;" ::: "memory");
+  if (tid == 0) {
+    // thread 0 issues the TMA loads: they read what the scan wrote (pool entries)
+    // and the inputs streamed in before its progress
+    if (a.progress) asm volatile("fence.proxy.async.global;" ::: "memory");
+    // A failed call (a bounded wait that gave up, here or in another kernel, or a
+    // device check): the scan may not have written this pair's lists, so the
+    // CTA does none of the work and leaves o unwritten.
+    sm.skip = (*(volatile int32_t*)a.status != 0);
+  }
   __syncthreads();
+  if (sm.skip) {
+    if constexpr (kStream) {
+      if (a.out_done && tid == 0) atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
+    }
+    return;
+  }
   // interval A (side 0) and B (side 1) of the pair
   const int c0A = a.t_begin + sA * L, c0B = c0A + L;
   const int LcA = min(L, t_end - c0A), LcB = hasB ? min(L, t_end - c0B) : 0;
   const long long lrowA = (long long)bh * a.snap_stride + a.snap_base + sA, lrowB = lrowA + 1;
   // lists and trace come from the scan: read past L1 (__ldcg)
-  const int m0A = __ldcg(a.snap_m0 + lrowA), m0B = hasB ? __ldcg(a.snap_m0 + lrowB) : 0;
+  // live entries of the two lists, checked against the capacity (a violation is
+  // a device-check failure and is clamped, so that nothing indexes out of bounds)
+  int m0A = __ldcg(a.snap_m0 + lrowA), m0B = hasB ? __ldcg(a.snap_m0 + lrowB) : 0;
+  if (m0A < 0 || m0A > C || m0B < 0 || m0B > C) {
+    if (tid == 0) atomicCAS(a.status, 0, 6);
+    m0A = min(max(m0A, 0), C);
+    m0B = min(max(m0B, 0), C);
+  }
   auto c0_of = [&](int side) { return side ? c0B : c0A; };
   auto Lc_of = [&](int side) { return side ? LcB : LcA; };
   volatile int* abort = &sm.abort_flag;
@@ -227,7 +247,12 @@ __global__ void __launch_bounds__(NT, 1)
   }
   for (int i = tid; i < 2 * kMaxC; i += NT) {
     const int side = i / kMaxC, x = i % kMaxC;
-    sm.ids[side][x] = (x < (side ? m0B : m0A)) ? __ldcg(a.snap_ids + (side ? lrowB : lrowA) * C + x) : -1;
+    int id = (x < (side ? m0B : m0A)) ? __ldcg(a.snap_ids + (side ? lrowB : lrowA) * C + x) : -1;
+    if (x < (side ? m0B : m0A) && (id < 0 || id >= a.pool_cap)) {  // a pool id outside the pool
+      atomicCAS(a.status, 0, 6);
+      id = 0;
+    }
+    sm.ids[side][x] = id;
   }
   if (warp == 1) tmem_alloc(&sm.tmem_base, kTmemCols);
   __syncthreads();

@@ -145,7 +145,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   if (tid == 0) {
     int m0 = a.m[bh];
     if (m0 < 0 || m0 > C) {  // corrupted cache: flag it and start empty
-      atomicExch(a.status, 2);
+      atomicExch(a.status, 6);
       m0 = 0;
     }
     sm.m = m0;
@@ -155,7 +155,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   for (int i = tid; i < C; i += NT) {
     int sl = a.slot[(long long)bh * C + i];
     if (sl < 0 || sl >= C) {
-      atomicExch(a.status, 2);
+      atomicExch(a.status, 6);
       sl = i;
     }
     sm.slot[i] = sl;
@@ -551,7 +551,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
           if (sm.dirty[i] || sm.pid[i] < 0) {
             int p = sm.pool_next++;
             if (p >= a.pool_cap) {  // cannot happen with a correctly sized workspace
-              atomicExch(a.status, 1);
+              atomicExch(a.status, 6);
               p = a.pool_cap - 1;
             }
             sm.pid[i] = p;

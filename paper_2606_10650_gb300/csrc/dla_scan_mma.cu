@@ -84,7 +84,7 @@ __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int
         break;
       }
       if (*abort) return false;
-      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::kWaitCycles) {
+      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::wait_limit(status)) {
         *abort = 1;
         atomicCAS(status, 0, sm100::kStatusTimeout);
         return false;
@@ -115,7 +115,7 @@ __device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16*
     const long long t0 = clock64();
     while ((piece_known = ld_acquire_gpu(piece_ready)) < piece_need) {
       if (*abort) break;
-      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::kWaitCycles) {
+      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::wait_limit(status)) {
         *abort = 1;
         atomicCAS(status, 0, sm100::kStatusTimeout);
         break;
@@ -1333,9 +1333,9 @@ int scan_mma_resident_streams(int BH, int d) {  // cached per device and kernel 
 }
 
 __global__ void gate_kernel(const int32_t* started, int n, int32_t* status) {
-  const long long t0 = clock64();
+  const long long t0 = clock64(), lim = sm100::wait_limit(status);
   while (ld_acquire_gpu(started) < n)
-    if (*(volatile int32_t*)status != 0 || clock64() - t0 > 4000000000LL) {  // ~2 s
+    if (*(volatile int32_t*)status != 0 || clock64() - t0 > lim) {
       atomicCAS(status, 0, 5);  // a failure reported elsewhere keeps its code
       return;
     }

@@ -16,6 +16,15 @@ namespace sm100 {
 constexpr int kStatusTimeout = 5;  // DLA_ERR_TIMEOUT
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
+// Limit of a bounded wait in SM clocks.  The word after a call's status word
+// (status[1]) may hold a shorter limit in units of 1024 clocks, written by the
+// host before the call's kernels run (a debugging knob that makes a wait give
+// up quickly); 0 selects the default of about 2 s.
+__device__ __forceinline__ long long wait_limit(const int32_t* status) {
+  const int u = status ? *(volatile const int32_t*)(status + 1) : 0;
+  return u > 0 ? ((long long)u << 10) : kWaitCycles;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -55,11 +64,11 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
 }
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, volatile int* abort, int32_t* status) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
-  const long long t0 = clock64();
+  const long long t0 = clock64(), lim = wait_limit(status);
   while (true) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > lim) {
       *abort = 1;
       if (status) atomicExch(status, kStatusTimeout);
       return false;
@@ -71,11 +80,11 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
 // another warp has already aborted.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, int32_t* status) {
   if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
+  const long long t0 = clock64(), lim = wait_limit(status);
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > lim) {
       *abort = 1;
       if (status) atomicExch(status, kStatusTimeout);
       return false;

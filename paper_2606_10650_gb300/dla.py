@@ -22,8 +22,8 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
             "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc",
-            "dla_forward_host_workspace", "dla_forward_host"]
-KERNELS = ["scan", "readout", "decode", "init", "gram", "gate"]
+            "dla_forward_host_workspace", "dla_forward_host", "dla_sync_status"]
+KERNELS = ["scan", "readout", "decode", "init", "gram", "gate", "status"]
 
 
 class DLAError(RuntimeError):
@@ -76,6 +76,7 @@ def lib():
         L.dla_forward_host_workspace.restype = sz
         L.dla_forward_host_workspace.argtypes = [P, ci, ci, ci, ci, ci, ci, ci]
         L.dla_forward_host.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp, sz, vp]
+        L.dla_sync_status.argtypes = [vp]
         L.dla_timing_enable.argtypes = [ci]
         L.dla_timing_read.argtypes = [ctypes.POINTER(ci), ctypes.POINTER(ctypes.c_double), ci]
         _LIB = L
@@ -275,6 +276,16 @@ def dla_forward_host(params, q, k, v, lam=None, o=None, cache=None, boundary=Non
                                 _ptr(merge_log), ctypes.c_void_p(base), nb, _stream(stream))
     _check(st)
     return workspace
+
+
+def dla_sync_status(stream=None):
+    """Waits for the stream and returns the device status of the library's
+    calls on it since the last read (0 ok, 5 a bounded wait gave up, 6 a device
+    check failed), clearing it.  Returns the code; does not raise for 5 or 6."""
+    st = lib().dla_sync_status(_stream(stream))
+    if st not in (0, 5, 6):
+        _check(st)
+    return st
 
 
 def workspace_status(workspace):

@@ -194,6 +194,34 @@ def host_batch(w: Workload, with_lam: bool = True, seed: int | None = None, T: i
     return q, k, v, lam
 
 
+def _stream_job(job):
+    """Worker of host_batch_parallel: one (b, h) stream as float32 arrays."""
+    w, b, h, seed, T = job
+    g = StreamGen(w, b, h, seed)
+    qq, kk, vv = g.tokens()
+    return b, h, qq[:T].astype(np.float32), kk[:T].astype(np.float32), vv[:T].astype(np.float32), \
+        g.lam()[:T].astype(np.float32)
+
+
+def host_batch_parallel(w: Workload, seed: int | None = None, T: int | None = None, procs: int | None = None):
+    """host_batch drawn by a pool of spawned processes, one stream per task,
+    returned as float32 arrays (exact: the values are bf16 or fp32 numbers).
+    The same values as host_batch."""
+    import multiprocessing as mp
+    import os
+    T = w.total_tokens if T is None else T
+    q = np.empty((w.B, T, w.H, w.d), np.float32)
+    k = np.empty_like(q)
+    v = np.empty_like(q)
+    lam = np.empty((w.B, T, w.H, w.C), np.float32)
+    jobs = [(w, b, h, seed, T) for b in range(w.B) for h in range(w.H)]
+    n = procs or min(len(jobs), os.cpu_count() or 1)
+    with mp.get_context("spawn").Pool(n) as pool:
+        for b, h, qq, kk, vv, ll in pool.imap_unordered(_stream_job, jobs):
+            q[b, :, h], k[b, :, h], v[b, :, h], lam[b, :, h] = qq, kk, vv, ll
+    return q, k, v, lam
+
+
 def to_device(x: np.ndarray, dtype: str, device):
     """Upload exact values as the device input dtype."""
     tdt = torch.float32 if dtype == "f32" else torch.bfloat16

@@ -9,8 +9,10 @@ oracle and
       of tau;
   G2  when token t would merge and the best and runner-up adjacent-pair
       densities lie within ``TIE_MARGIN`` (relative) of each other, rolls back
-      to the first token of the newest state among the two pairs, redraws that
-      token and replays from a checkpoint (G3).
+      to the last token of the newest state among the two pairs (changing
+      that token's score changes the state's summed score, the shortest
+      rollback that moves one of the tied densities), redraws it and replays
+      from a checkpoint (G3).
 
 Redraws come from generators keyed by (seed, b, h, t, attempt), so the result
 is reproducible.  THR_MARGIN is 1e-3 relative.  TIE_MARGIN is 1e-5 relative:
@@ -38,14 +40,15 @@ class RejectionFailed(RuntimeError):
 
 def safe_stream(w: W.Workload, b: int, h: int, T: int | None = None, seed: int | None = None,
                 thr: float = THR_MARGIN, tie: float = TIE_MARGIN, score_mode: int = 0,
-                max_rollbacks: int = 20000, max_attempts: int = 64):
+                max_rollbacks: int = 100000, max_attempts: int = 64):
     g = W.StreamGen(w, b, h, seed)
     q, k, v = g.tokens()
     lam = g.lam()
     T = w.total_tokens if T is None else int(T)
     q, k, v, lam = q[:T].copy(), k[:T].copy(), v[:T].copy(), lam[:T].copy()
     attempts = np.zeros(T, np.int64)
-    ck_every = max(256, T // 32)
+    # checkpoints: every FINE tokens, the last NFINE of them kept, plus every COARSE tokens
+    FINE, NFINE, COARSE = 16, 32, 1024
     st = oracle.Stream(w.C, w.d, w.d, w.tau, w.eps, w.rms_eps, score_mode)
     ckpts = {0: st.copy()}
     redraws = rollbacks = 0
@@ -55,9 +58,10 @@ def safe_stream(w: W.Workload, b: int, h: int, T: int | None = None, seed: int |
         k[t], v[t] = g.redraw(t, int(attempts[t]))
 
     def restore(t0):
-        nonlocal st, ckpts
+        nonlocal st
         c = max(c for c in ckpts if c <= t0)
-        ckpts = {kk: vv for kk, vv in ckpts.items() if kk <= c}
+        for kk in [kk for kk in ckpts if kk > c]:
+            del ckpts[kk]
         st = ckpts[c].copy()
         for s in range(c, t0):
             st.step(k[s], v[s])
@@ -79,15 +83,18 @@ def safe_stream(w: W.Workload, b: int, h: int, T: int | None = None, seed: int |
             rollbacks += 1
             if rollbacks > max_rollbacks:
                 raise RejectionFailed(f"{w.name} stream ({b},{h}): too many rollbacks")
-            t0 = r["rollback_to"]
+            t0 = r["rollback_last"]
             redraw(t0)
             restore(t0)
             t = t0
             continue
         st.step(k[t], v[t])
         t += 1
-        if t % ck_every == 0:
+        if t % FINE == 0:
             ckpts[t] = st.copy()
+            old = t - FINE * NFINE
+            if old > 0 and old % COARSE != 0:
+                ckpts.pop(old, None)
     return dict(q=q, k=k, v=v, lam=lam, redraws=redraws, rollbacks=rollbacks)
 
 
@@ -114,3 +121,53 @@ def safe_batch(w: W.Workload, T: int | None = None, streams=None, seed: int | No
 
 def shrink(w: W.Workload, **kw) -> W.Workload:
     return dataclasses.replace(w, **kw)
+
+
+def _safe_and_oracle(job):
+    """Worker of safe_oracle_streams (a separate process): one decision-safe
+    stream and the oracle's results on it."""
+    w, b, h, T, seed, score_mode, want_o = job
+    r = safe_stream(w, b, h, T=T, seed=seed, score_mode=score_mode)
+    st = oracle.Stream(w.C, w.d, w.d, w.tau, w.eps, w.rms_eps, score_mode)
+    o, bnd, ml, _ = st.run(r["q"], r["k"], r["v"], r["lam"], want_o=want_o)
+    ex = st.export()
+    f32 = lambda x: x.astype(np.float32)  # exact: the inputs are bf16 / fp32 values
+    return dict(b=b, h=h, q=f32(r["q"]), k=f32(r["k"]), v=f32(r["v"]), lam=f32(r["lam"]), bnd=bnd, ml=ml,
+                o=None if o is None else (o if want_o is None else o[np.asarray(want_o, bool)]),
+                cache=dict(states=ex["states"], n=ex["n"], ibar=ex["ibar"], m=ex["m"]),
+                rollbacks=r["rollbacks"], redraws=r["redraws"])
+
+
+def safe_oracle_streams(w: W.Workload, T: int | None = None, streams=None, seed: int | None = None,
+                        score_mode: int = 0, want_o=None, procs: int | None = None):
+    """Decision-safe inputs and the oracle's results for the listed streams of
+    a batch (default all), one stream per worker process (spawned, so that it
+    is safe after CUDA was initialised in this process).
+
+    Returns (q, k, v, lam) host arrays [B, T, H, *] (float64 values; streams
+    not listed keep the plain seeded draws) and the oracle's results in the
+    layout of ``oracle.forward``: o [B, T, H, d] (NaN where not computed),
+    boundary, merge_log and caches."""
+    import multiprocessing as mp
+    import os
+    T = w.total_tokens if T is None else int(T)
+    streams = [(b, h) for b in range(w.B) for h in range(w.H)] if streams is None else list(streams)
+    q, k, v, lam = W.host_batch(w, seed=seed, T=T)
+    o = np.full(q.shape, np.nan)
+    bnd = np.zeros((w.B, w.H, T), np.uint8)
+    ml = np.full((w.B, w.H, T), -2, np.int32)
+    caches = {}
+    n = procs or min(len(streams), os.cpu_count() or 1)
+    jobs = [(w, b, h, T, seed, score_mode, want_o) for (b, h) in streams]
+    with mp.get_context("spawn").Pool(n) as pool:
+        for res in pool.imap_unordered(_safe_and_oracle, jobs):
+            b, h = res["b"], res["h"]
+            q[b, :, h], k[b, :, h], v[b, :, h], lam[b, :, h] = res["q"], res["k"], res["v"], res["lam"]
+            bnd[b, h], ml[b, h] = res["bnd"], res["ml"]
+            if res["o"] is not None:
+                if want_o is None:
+                    o[b, :, h] = res["o"]
+                else:
+                    o[b, np.asarray(want_o, bool), h] = res["o"]
+            caches[(b, h)] = res["cache"]
+    return (q, k, v, lam), dict(o=o, boundary=bnd, merge_log=ml, caches=caches)

@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     for n in _declared():
         assert hasattr(L, n), n
     assert set(_declared()) == set(dla.EXPORTED)
-    assert L.dla_version() == 1
+    assert L.dla_version() == 2
 
 
 def _fake(addr=1 << 20):
@@ -106,3 +106,12 @@ def test_params_layout_and_seq_lens_checks(L):
     q.seq_lens = (1 << 20) + 2  # not 4-byte aligned
     assert _fwd(L, q) == 1
     assert b"seq_lens" in L.dla_last_error()
+
+
+def test_kernel_kinds_match_the_header():
+    """dla_timing_read fills DLA_K_COUNT entries; the binding names each kind."""
+    src = open(os.path.join(ROOT, "include", "dla.h")).read()
+    count = int(re.search(r"DLA_K_COUNT\s*=\s*(\d+)", src).group(1))
+    assert count == len(dla.KERNELS)
+    for i, name in enumerate(dla.KERNELS):
+        assert re.search(rf"DLA_K_{name.upper()}\s*=\s*{i}\b", src) or (name == "readout" and "DLA_K_READOUT = 1" in src)

@@ -299,9 +299,9 @@ def test_probe_runner_up_gap_and_rollback_brute_force(C, mode):
     relies on: at every token that merges, recompute from the exported cache
     all C - 1 adjacent pair densities (Algorithm 2's definition), order them by
     (density, index) and check the best pair, the runner-up density, the
-    relative gap (runner-up - best) / |best| and the first token of the newest
-    state among the two pairs (from the states' token counts, not from the
-    oracle's own token ranges).  The probe must leave the stream unchanged and
+    relative gap (runner-up - best) / |best| and the first and last tokens of
+    the newest state among the two pairs (from the states' token counts, not
+    from the oracle's own token ranges).  The probe must leave the stream unchanged and
     announce the decision the next step takes, with |I - tau| / tau as margin."""
     rng = np.random.default_rng(300 + 7 * C + mode)
     T, d = 96, 3
@@ -319,7 +319,7 @@ def test_probe_runner_up_gap_and_rollback_brute_force(C, mode):
         if t > 0:
             assert r["thr_margin"] == pytest.approx(abs(I - tau) / tau, rel=1e-12)
         if j < 0:
-            assert r["rollback_to"] == -1 and math.isinf(r["tie_gap"])
+            assert r["rollback_to"] == -1 and r["rollback_last"] == -1 and math.isinf(r["tie_gap"])
             continue
         n, ib = pre["n"].astype(np.int64), pre["ibar"]
         dens = [((ib[i] + ib[i + 1]) / (n[i] + n[i + 1]), i) for i in range(C - 1)]
@@ -329,6 +329,7 @@ def test_probe_runner_up_gap_and_rollback_brute_force(C, mode):
         assert r["tie_gap"] == pytest.approx((sd - bd) / abs(bd), rel=1e-12, abs=1e-300)
         newest = max(bi, si) + 1
         assert r["rollback_to"] == int(n[:newest].sum())
+        assert r["rollback_last"] == int(n[:newest + 1].sum()) - 1
         checked += 1
     assert checked >= 5
 

@@ -20,8 +20,8 @@ from parity_util import TOL
 pytestmark = pytest.mark.gpu
 
 
-def _inputs(seed, dev):
-    w = W.get("regime", B=1, H=2, T=900)
+def _inputs(seed, dev, T=900):
+    w = W.get("regime", B=1, H=2, T=T)
     q, k, v, lam = W.host_batch(w, seed=seed, T=w.T)
     t = [W.to_device(x, w.dtype, dev) for x in (q, k, v)]
     t.append(torch.from_numpy(lam.astype(np.float32)).to(dev))
@@ -40,7 +40,9 @@ def _run(entry, w, t, dev):
         dla.dla_forward_noalloc(p, q, k, v, lam, o, cache, bnd, ml)
     else:
         dla.dla_forward(p, q, k, v, lam, o, cache, bnd, ml)
-    torch.cuda.synchronize()
+    # the call's device status (its workspace word is inside the library's
+    # static array, so it is read through the stream's status word)
+    assert dla.dla_sync_status() == 0
     return o.cpu(), bnd.cpu(), ml.cpu(), cache.export()
 
 
@@ -55,6 +57,23 @@ def test_noalloc_matches_dla_forward_two_calls_in_a_row():
         assert (o - o_ref).abs().max().item() <= TOL[w.dtype]
         assert torch.equal(c["m"], c_ref["m"]) and torch.equal(c["n"], c_ref["n"])
         assert (c["states"] - c_ref["states"]).abs().max().item() <= TOL[w.dtype]
+
+
+def test_noalloc_with_a_plan_limited_by_its_scratch():
+    """A sequence whose preferred workspace exceeds the 64 MiB scratch (but whose
+    smallest one fits) runs with fewer rounds of snapshots; results equal
+    dla_forward's with its preferred workspace."""
+    dev = torch.device("cuda:0")
+    w, t = _inputs(13, dev, T=6000)
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    B, T, H, d = t[1].shape
+    assert dla.dla_forward_workspace(p, B, T, H, d, d, dla.DLA_BF16, True) > (64 << 20)
+    assert dla.dla_forward_min_workspace(p, B, T, H, d, d, dla.DLA_BF16, True) <= (64 << 20)
+    o_ref, b_ref, m_ref, c_ref = _run("workspace", w, t, dev)
+    o, b, m, c = _run("noalloc", w, t, dev)
+    assert torch.equal(b, b_ref) and torch.equal(m, m_ref)
+    assert (o - o_ref).abs().max().item() <= TOL[w.dtype]
+    assert torch.equal(c["m"], c_ref["m"]) and torch.equal(c["n"], c_ref["n"])
 
 
 def test_noalloc_rejects_calls_beyond_its_scratch():
