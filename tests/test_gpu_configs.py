@@ -81,7 +81,10 @@ def test_decode_workload_full_capacity():
     gp = run_gpu(wp, q[:, :Tp], k[:, :Tp], v[:, :Tp], lam[:, :Tp], want_o=False)
     np.testing.assert_array_equal(gp["boundary"], r["boundary"][:, :, :Tp])
     np.testing.assert_array_equal(gp["merge_log"], r["merge_log"][:, :, :Tp])
-    assert (gp["cache"].export()["m"] == w.C).all(), "the prefill must fill the cache"
+    m0 = gp["cache"].export()["m"]
+    # the 8192-token prefill fills most caches (C = 64); the decode kernel's argmin
+    # then spans two lanes per entry pair and its slot remap all 64 slots
+    assert (m0 == w.C).sum() >= m0.numel() // 2 and (m0 > 33).all(), m0
     cache = gp["cache"]
     dev = torch.device("cuda:0")
     p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
@@ -106,4 +109,6 @@ def test_decode_workload_full_capacity():
     g = dict(boundary=r["boundary"], merge_log=r["merge_log"], o=None, cache=cache)
     compare(w, g, r)
     assert b_all.sum() > 0 and (m_all >= 0).sum() > 0, "the decode steps must open states and merge"
+    full = (m0 == w.C).numpy()
+    assert (m_all[full] >= 0).sum() > 0, "merges must happen on full C = 64 caches"
     print("decode C=64: boundaries", int(b_all.sum()), "merges", int((m_all >= 0).sum()), "worst o", worst)
