@@ -185,7 +185,12 @@ dla_status dla_sync_status(void* stream);
  *   (pre-pass, whole scan and read-out one after another, each kernel alone on
  *   the device: for timing and profiling).  The concurrent schedule needs
  *   every scan CTA resident at once with SMs to spare; calls with more streams
- *   than that take the rounds schedule.  All give the same results. */
+ *   than that take the rounds schedule.  All give the same results.
+ *   DLA_SCAN (read at every call): unset selects the scan on warp-level tensor
+ *   cores (CTA pairs, the open state in registers); "tc" selects, for calls
+ *   with a read-out over whole rows of device-resident inputs, the scan on
+ *   tcgen05 with the open state in tensor memory (one CTA per stream; same
+ *   results, currently slower). */
 dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk,
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,

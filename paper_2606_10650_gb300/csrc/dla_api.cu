@@ -120,9 +120,9 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   P.off_lists_m0 = off;  if (with_output) off = align256(off + BH * P.nsnap_total * sizeof(int32_t));
   P.off_lists_ids = off; if (with_output) off = align256(off + BH * P.nsnap_total * C * sizeof(int32_t));
   P.off_pstate = off;    if (with_output) off = align256(off + (BH + BH * C) * sizeof(int32_t));
-  // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramBlock floats per 64-token chunk
+  // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramStride floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
-  P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramBlock * 4);
+  P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramStride * 4);
   // scan progress per (stream, CTA), the count of started scan CTAs (concurrent read-out),
   // the count of input pieces streamed in by the host, and the Gram pre-pass's per-block
   // chunk counters (a pre-pass running beside the scan)
@@ -174,6 +174,11 @@ namespace {
 // kernel waits for another: for timing and profiling single kernels).  All
 // compute the same results.
 enum Schedule { kConcurrent, kRounds, kSerial };
+// DLA_SCAN=tc (read at every call) selects the tcgen05 scan where it applies.
+bool scan_tc_requested() {
+  const char* v = getenv("DLA_SCAN");
+  return v && strcmp(v, "tc") == 0;
+}
 Schedule schedule() {
   const char* v = getenv("DLA_SCHEDULE");
   if (v && strcmp(v, "rounds") == 0) return kRounds;
@@ -598,12 +603,13 @@ size_t dla_forward_min_workspace(const dla_params* p, int B, int T, int H, int d
 
 // SMs the scan leaves to the rest on the concurrent schedule when all its CTAs
 // are resident (0: they are not)
-static int concurrent_free_sms(int B, int H, int d, cudaError_t* err) {
+static int concurrent_free_sms(int B, int H, int d, bool scan_tc, cudaError_t* err) {
   int dev = 0, sms = 0;
   if ((*err = cudaGetDevice(&dev)) != cudaSuccess ||
       (*err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
     return 0;
   const int BH = B * H;
+  if (scan_tc) return (dla::scan_tc_resident_streams() >= BH) ? sms - BH : 0;
   return (dla::scan_mma_resident_streams(BH, d) >= BH) ? sms - BH * dla::scan_mma_ctas_per_stream(BH, d) : 0;
 }
 
@@ -672,7 +678,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   if (io) {
     cudaError_t qe = cudaSuccess;
     stream_in = with_output && use_tc(in_dtype, d) && P.persistent && (P.nsnap_total + 1) / 2 <= 65535 &&
-                schedule() == kConcurrent && concurrent_free_sms(B, H, d, &qe) >= kMinFreeSms && write_value_fn();
+                schedule() == kConcurrent && concurrent_free_sms(B, H, d, false, &qe) >= kMinFreeSms && write_value_fn();
     if (qe != cudaSuccess) return cuda_fail(qe, "device query");
     if (!stream_in) {
       const cudaError_t ce = h2d_tokens(*io, B, T, H, d, C, 0, T, st);
@@ -744,6 +750,16 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   sa.pstate = P.persistent ? (int32_t*)(ws + P.off_pstate) : nullptr;
   sa.gram = P.gram_chunks ? (const float*)(ws + P.off_gram) : nullptr;
   sa.gram_chunks = P.gram_chunks;
+  // The scan: the mma.sync scan (CTA pairs, the open state in registers) by
+  // default; with DLA_SCAN=tc, on tcgen05 with the open state in tensor memory
+  // (one CTA per stream) where the Gram pre-pass runs over whole rows of
+  // resident inputs (it is correct but slower on the benchmark workloads:
+  // its per-chunk chain is bound by the latency of small tensor-core groups).
+  const bool scan_tc = tc && P.gram_chunks > 0 && !p->seq_lens && !stream_in && scan_tc_requested();
+  auto launch_main_scan = [&](cudaStream_t s_) -> cudaError_t {
+    return scan_tc ? dla::launch_scan_tc(sa, s_) : dla::launch_scan_mma(sa, d, pool_bf16, s_);
+  };
+  const int gram_per_sm = scan_tc ? dla::kGramTcCtasPerSm : dla::kGramCtasPerSm;
   // Round r: the scan (high-priority stream) appends to the pool, then the
   // read-out of round r (low-priority stream) runs while the scan of round
   // r + 1 proceeds.  In reset mode pool b is reused by round r + 2 only after
@@ -761,10 +777,11 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     ga.out = (float*)(ws + P.off_gram);
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = nullptr;
+    ga.packed = scan_tc ? 1 : 0;
     int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_fail(e, "device query");
-    dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
+    dla::gram_blocks(B * H, P.gram_chunks, gram_per_sm * sms, &ga.nblk, &ga.per_blk);
     if (P.gram_chunks) {
       e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
@@ -773,7 +790,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     sa.t_begin = 0; sa.t_end = T;
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
     sa.carry_in = 0; sa.snap_at_end = 0;
-    e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
+    e = timed(DLA_K_SCAN, S->hi, [&] { return launch_main_scan(S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     ra.pool = sa.pool;
     ra.t_begin = 0; ra.t_end = T;
@@ -786,7 +803,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   }
   int free_sms = 0;  // SMs the scan leaves to the rest when all its CTAs are resident (0: they are not)
   if (one_readout && sched == kConcurrent) {
-    free_sms = concurrent_free_sms(B, H, d, &e);
+    free_sms = concurrent_free_sms(B, H, d, scan_tc, &e);
     if (e != cudaSuccess) return cuda_fail(e, "device query");
   }
   if (free_sms >= kMinFreeSms) {
@@ -807,7 +824,8 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
       if ((e = cudaGetDevice(&dev)) != cudaSuccess || dev < 0 || dev >= kMaxDev) return cuda_fail(e, "device query");
       std::lock_guard<std::mutex> g(mu);
       if (!loaded[dev]) {
-        if ((e = dla::preload_scan_kernels()) != cudaSuccess || (e = dla::preload_readout_kernels()) != cudaSuccess)
+        if ((e = dla::preload_scan_kernels()) != cudaSuccess || (e = dla::preload_scan_tc_kernel()) != cudaSuccess ||
+            (e = dla::preload_readout_kernels()) != cudaSuccess)
           return cuda_fail(e, "kernel load");
         loaded[dev] = true;
       }
@@ -820,13 +838,14 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     // with streamed inputs the scan forms its Gram entries itself: a pre-pass
     // waiting for the pieces would hold back the read-out behind it
     const bool run_gram = P.gram_chunks && !stream_in;
-    const int ctas = dla::scan_mma_ctas_per_stream(B * H, d);
+    const int ctas = scan_tc ? 1 : dla::scan_mma_ctas_per_stream(B * H, d);
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
     ga.out = (float*)(ws + P.off_gram);
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = gram_ready;
-    dla::gram_blocks(B * H, P.gram_chunks, dla::kGramCtasPerSm * free_sms, &ga.nblk, &ga.per_blk);
+    ga.packed = scan_tc ? 1 : 0;
+    dla::gram_blocks(B * H, P.gram_chunks, gram_per_sm * free_sms, &ga.nblk, &ga.per_blk);
     if ((e = cudaMemsetAsync(progress, 0, (2 * B * H + 2 + kOutPieces + B * H * ga.nblk) * sizeof(int32_t), S->hi)) !=
         cudaSuccess)
       return cuda_fail(e, "progress reset");
@@ -866,7 +885,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
       if ((e = cudaStreamWaitEvent(S->cp, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       if ((s = put_piece(0)) != DLA_OK) return s;
     }
-    e = timed(DLA_K_SCAN, S->hi, [&] { return dla::launch_scan_mma(sa, d, pool_bf16, S->hi); });
+    e = timed(DLA_K_SCAN, S->hi, [&] { return launch_main_scan(S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     e = timed(DLA_K_GATE, S->lo, [&] { return dla::launch_gate(started, B * H * ctas, status, S->lo); });
     if (e != cudaSuccess) return cuda_fail(e, "gate launch");
@@ -935,17 +954,18 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
     ga.out = (float*)(ws + P.off_gram);
     ga.ready = nullptr;
+    ga.packed = scan_tc ? 1 : 0;
     int dev = 0, sms = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess || (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
       return cuda_fail(e, "device query");
     const int first = std::min(P.gram_chunks, sizes[0] * P.interval / dla::kScanL);
     ga.chunk0 = 0; ga.count = first;
-    dla::gram_blocks(B * H, ga.count, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
+    dla::gram_blocks(B * H, ga.count, gram_per_sm * sms, &ga.nblk, &ga.per_blk);
     e = timed(DLA_K_GRAM, S->hi, [&] { return dla::launch_gram(ga, d, S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     if (first < P.gram_chunks) {
       ga.chunk0 = first; ga.count = P.gram_chunks - first;
-      dla::gram_blocks(B * H, ga.count, dla::kGramCtasPerSm * sms, &ga.nblk, &ga.per_blk);
+      dla::gram_blocks(B * H, ga.count, gram_per_sm * sms, &ga.nblk, &ga.per_blk);
       if ((e = cudaStreamWaitEvent(S->lo, S->in, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
       e = timed(DLA_K_GRAM, S->lo, [&] { return dla::launch_gram(ga, d, S->lo); });
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
@@ -971,7 +991,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     if (r == 1 && gram_rest && (e = cudaStreamWaitEvent(S->hi, S->gram_done, 0)) != cudaSuccess)
       return cuda_fail(e, "stream wait");
     e = timed(DLA_K_SCAN, S->hi, [&] {
-      return in_bf16 ? dla::launch_scan_mma(sa, d, pool_bf16, S->hi) : dla::launch_scan(sa, d, false, pool_bf16, S->hi);
+      return in_bf16 ? launch_main_scan(S->hi) : dla::launch_scan(sa, d, false, pool_bf16, S->hi);
     });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     if ((e = cudaEventRecord(S->scan_done[r % 2], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");

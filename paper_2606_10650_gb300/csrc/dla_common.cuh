@@ -103,11 +103,12 @@ __device__ __forceinline__ void fill_padding_trace(uint8_t* bnd, int32_t* mlog, 
 // copy of the line.
 __device__ __forceinline__ void wait_progress(const int32_t* progress, int ctas, int bh, int need, int32_t* status) {
   if (!progress || threadIdx.x != 0) return;
-  const long long t0 = clock64(), lim = sm100::wait_limit(status);
+  const long long t0 = clock64();
+  long long lim = -1;
   for (int r = 0; r < ctas; ++r)
     while (ld_acquire_gpu(progress + 2 * bh + r) < need) {
       if (*(volatile int32_t*)status != 0) return;  // the call has failed already
-      if (clock64() - t0 > lim) {
+      if (sm100::wait_expired(t0, lim, status)) {
         atomicCAS(status, 0, sm100::kStatusTimeout);
         return;
       }
@@ -157,6 +158,27 @@ __device__ __forceinline__ double warp_sum(double v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
+}
+
+// Cache metadata of the live entries, held in registers by one warp: entry i
+// in lane i % 32, element i / 32 (C <= 64).  i is warp-uniform.
+template <typename T>
+__device__ __forceinline__ T entry_get(const T (&f)[2], int i) {
+  return __shfl_sync(0xffffffffu, (i < 32) ? f[0] : f[1], i & 31);
+}
+template <typename T>
+__device__ __forceinline__ void entry_set(T (&f)[2], int i, T v) {
+  if ((i & 31) == (int)(threadIdx.x & 31)) {
+    if (i < 32) f[0] = v;
+    else f[1] = v;
+  }
+}
+// Entry i + 1's field for both of this lane's entries (i = lane, lane + 32).
+template <typename T>
+__device__ __forceinline__ void entry_next(const T (&f)[2], T (&nx)[2]) {
+  const int lane = threadIdx.x & 31;
+  nx[0] = __shfl_sync(0xffffffffu, lane == 0 ? f[1] : f[0], (lane + 1) & 31);
+  nx[1] = __shfl_down_sync(0xffffffffu, f[1], 1);
 }
 
 // Warp argmin over (value, index) pairs; lowest index wins exact ties.

@@ -16,6 +16,20 @@ constexpr int kScanL = 64;  // tokens per scan chunk (K1)
 // prefix table Q[j][t] and a_t (see GramArgs).
 constexpr int kGramBlock = 2 * kScanL * kScanL + kScanL;
 
+// Gram block of the tensor-core scan (K0 with GramArgs::packed = 1), per chunk:
+//   gs[j][t], j <= t <= 64   packed by rows (row j starts at 65 j - j (j - 1) / 2)
+//   Q[j][t],  j <= t <= 64   the same packing (Q[j][64] is the whole chunk's running sum)
+//   a[t]                     64
+//   cs[j][t] = sum_{j <= s < 64} (k_t.k'_s)(v_t.v'_s), t in this chunk, s in the
+//            previous chunk (k', v'): beta_t of a segment opened at j of the
+//            previous chunk, 64 x 64 row-major
+constexpr int kPackTri = 65 * kScanL - kScanL * (kScanL - 1) / 2;  // 2144
+constexpr int kGramBlockTc = 2 * kPackTri + kScanL + kScanL * kScanL;
+__host__ __device__ constexpr int pack_row(int j) { return 65 * j - j * (j - 1) / 2; }
+// Floats between consecutive chunks' blocks in the Gram pre-pass output (either
+// layout).
+constexpr int kGramStride = kGramBlockTc;
+
 // Method parameters of the score / boundary test (Sec. 3.1).
 struct ScoreParams {
   double tau, eps, rms_eps;
@@ -90,11 +104,13 @@ struct GramArgs {
   int nchunks;           // chunks of the whole sequence
   int chunk0, count;     // this launch: chunks chunk0 .. chunk0 + count - 1
   int nblk, per_blk;     // blocks of this launch and chunks per block at most (nblk * per_blk >= count)
-  float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64)
+  float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64); packed: [kGramBlockTc]
   int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after its first four, then every fourth), or nullptr
+  int packed;            // 1: the tensor-core scan's layout (kGramBlockTc floats per chunk, with the cross table)
 };
 constexpr int kMaxGramBlk = 64;  // blocks per stream of one Gram launch, at most
 constexpr int kGramCtasPerSm = 3;  // resident Gram CTAs per SM (shared memory)
+constexpr int kGramTcCtasPerSm = 2;  // the same for the packed layout (two chunks of k, v in shared memory)
 
 // K2: read-out of one round, one CTA per (snapshot interval, stream).
 struct ReadoutArgs {
@@ -177,6 +193,13 @@ cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStre
 cudaError_t preload_scan_kernels();
 cudaError_t preload_readout_kernels();
 cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s);
+// K1 on tcgen05 (dla_scan_tc.cu): bf16 inputs, d = 128, one CTA per stream, the
+// open state in tensor memory; needs the packed Gram pre-pass output, whole rows
+// (no per-row lengths) and resident inputs.
+cudaError_t launch_scan_tc(const ScanArgs& a, cudaStream_t s);
+// Streams whose launch_scan_tc CTAs can all be resident at once.
+int scan_tc_resident_streams();
+cudaError_t preload_scan_tc_kernel();
 size_t scan_smem_bytes(int d);
 cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;

@@ -77,6 +77,7 @@ __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int
   const int blk = gc % f.nblk, need = gc / f.nblk + 1;
   if (f.cnt[blk] < need) {
     const long long t0 = clock64();
+    long long lim = -1;
     while (true) {
       const int c = ld_acquire_gpu(f.ready + blk);
       if (c >= need) {
@@ -84,7 +85,7 @@ __device__ __forceinline__ bool gram_feed_wait(GramFeed& f, int gc, volatile int
         break;
       }
       if (*abort) return false;
-      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::wait_limit(status)) {
+      if (*(volatile int32_t*)status != 0 || sm100::wait_expired(t0, lim, status)) {
         *abort = 1;
         atomicCAS(status, 0, sm100::kStatusTimeout);
         return false;
@@ -113,9 +114,10 @@ __device__ __forceinline__ void prefetch_chunk(__nv_bfloat16* dk, __nv_bfloat16*
   constexpr int V16 = D / 8;
   if (piece_ready && piece_known < piece_need) {
     const long long t0 = clock64();
+    long long lim = -1;
     while ((piece_known = ld_acquire_gpu(piece_ready)) < piece_need) {
       if (*abort) break;
-      if (*(volatile int32_t*)status != 0 || clock64() - t0 > sm100::wait_limit(status)) {
+      if (*(volatile int32_t*)status != 0 || sm100::wait_expired(t0, lim, status)) {
         *abort = 1;
         atomicCAS(status, 0, sm100::kStatusTimeout);
         break;
@@ -418,27 +420,6 @@ __device__ __forceinline__ void put_pair(float* entry, int D, int j, int k, floa
 template <typename Tpool>
 constexpr int parts_of() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
-// Cache metadata of the live entries, held in registers by one warp: entry i
-// in lane i % 32, element i / 32 (C <= 64).  i is warp-uniform.
-template <typename T>
-__device__ __forceinline__ T entry_get(const T (&f)[2], int i) {
-  return __shfl_sync(0xffffffffu, (i < 32) ? f[0] : f[1], i & 31);
-}
-template <typename T>
-__device__ __forceinline__ void entry_set(T (&f)[2], int i, T v) {
-  if ((i & 31) == (int)(threadIdx.x & 31)) {
-    if (i < 32) f[0] = v;
-    else f[1] = v;
-  }
-}
-// Entry i + 1's field for both of this lane's entries (i = lane, lane + 32).
-template <typename T>
-__device__ __forceinline__ void entry_next(const T (&f)[2], T (&nx)[2]) {
-  const int lane = threadIdx.x & 31;
-  nx[0] = __shfl_sync(0xffffffffu, lane == 0 ? f[1] : f[0], (lane + 1) & 31);
-  nx[1] = __shfl_down_sync(0xffffffffu, f[1], 1);
-}
-
 }  // namespace
 
 // One stream per CTA (CL = 1) or per CTA pair (CL = 2, a thread-block
@@ -671,7 +652,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   if (!kRagged || ntok > 0)  // a row that ended before this round has no chunk to load
   prefetch_chunk<D>(sm.kv[0][0], sm.kv[0][1], kbase + (long long)a.t_begin * row_stride,
                       vbase + (long long)a.t_begin * row_stride, row_stride, min(L, ntok), sm.gq[0],
-                      a.gram ? a.gram + gchunk0 * kGramBlock : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
+                      a.gram ? a.gram + gchunk0 * kGramStride : nullptr, &sm.kvbar[0], feed, a.t_begin / L,
                       &sm.abort_flag, a.status, tid, NT, a.piece_ready,
                       a.piece_chunks ? a.t_begin / L / a.piece_chunks + 1 : 0, piece_known);
   int rel_pending = 0;  // thread NT - 32: progress value not yet released
@@ -797,7 +778,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const int t1 = t0 + L;
       prefetch_chunk<D>(sm.kv[st ^ 1][0], sm.kv[st ^ 1][1], kbase + (long long)t1 * row_stride,
                         vbase + (long long)t1 * row_stride, row_stride, min(L, DLA_T_END - t1), sm.gq[st ^ 1],
-                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramBlock : nullptr, &sm.kvbar[st ^ 1], feed,
+                        a.gram ? a.gram + (gchunk0 + c + 1) * kGramStride : nullptr, &sm.kvbar[st ^ 1], feed,
                         a.t_begin / L + c + 1, &sm.abort_flag, a.status, tid - 32, NT - 32, a.piece_ready,
                         a.piece_chunks ? (a.t_begin / L + c + 1) / a.piece_chunks + 1 : 0, piece_known);
     }
@@ -1188,7 +1169,7 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
     prefix_rows_ilp(sm.G, 1, L + 1, sm.Q, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u]
     __syncthreads();
     // out: gs[j][t], Q[j][t] (four consecutive t per thread), a[t]
-    float* out = a.out + ((long long)bh * a.nchunks + c) * kGramBlock;
+    float* out = a.out + ((long long)bh * a.nchunks + c) * kGramStride;
     for (int e = threadIdx.x; e < L * L / 4; e += NT) {
       const int j = e / (L / 4), t = (e % (L / 4)) * 4;
       const float4 g4 = make_float4(sm.G[t * (L + 1) + j], sm.G[(t + 1) * (L + 1) + j], sm.G[(t + 2) * (L + 1) + j],
@@ -1211,10 +1192,148 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   }
 }
 
+// Cross Gram block of two chunks with mma.sync: Gout[t][s] = (k_t.k'_s)(v_t.v'_s)
+// for every t of this chunk (K, V) and s of the previous one (Kp, Vp), row
+// stride L + 1.  All 8 warps; warp w takes the 16-token band w % 4 and the 32
+// columns w / 4.
+template <int D>
+__device__ __forceinline__ void gram_cross(const __nv_bfloat16* Ks, const __nv_bfloat16* Vs, const __nv_bfloat16* Kp,
+                                           const __nv_bfloat16* Vp, float* Gout) {
+  constexpr int RP = D + 8;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> 2, tg = lane & 3, q = lane >> 3, r8 = lane & 7;
+  const int mt = warp & 3, sb = 32 * (warp >> 2);
+  float kk4[4][4], vv4[4][4];
+#pragma unroll
+  for (int n = 0; n < 4; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) kk4[n][e] = vv4[n][e] = 0.f;
+#pragma unroll 2
+  for (int kk = 0; kk < D; kk += 16) {
+    uint32_t ak[4], av[4];
+    ldsm4(ak, Ks + (16 * mt + (q & 1) * 8 + r8) * RP + kk + (q >> 1) * 8);
+    ldsm4(av, Vs + (16 * mt + (q & 1) * 8 + r8) * RP + kk + (q >> 1) * 8);
+#pragma unroll
+    for (int np = 0; np < 2; ++np) {
+      uint32_t bk[4], bv[4];
+      ldsm4(bk, Kp + (sb + 16 * np + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8);
+      ldsm4(bv, Vp + (sb + 16 * np + (q >> 1) * 8 + r8) * RP + kk + (q & 1) * 8);
+      mma16816(kk4[2 * np], ak, bk[0], bk[1]);
+      mma16816(kk4[2 * np + 1], ak, bk[2], bk[3]);
+      mma16816(vv4[2 * np], av, bv[0], bv[1]);
+      mma16816(vv4[2 * np + 1], av, bv[2], bv[3]);
+    }
+  }
+#pragma unroll
+  for (int n = 0; n < 4; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int t = 16 * mt + g + 8 * (e >> 1);
+      const int s2 = sb + 8 * n + 2 * tg + (e & 1);
+      Gout[t * (L + 1) + s2] = kk4[n][e] * vv4[n][e];
+    }
+}
+
+// K0 for the tensor-core scan: the same tables as gram_kernel in the packed
+// layout (kGramBlockTc floats per chunk) plus the cross table cs of the chunk
+// against the previous one.  Each CTA walks its block's chunks like
+// gram_kernel, loading the chunk and the one before it.
+template <int D>
+struct GramTcSmem {
+  static constexpr int RP = D + 8;
+  __nv_bfloat16 k[L * RP], v[L * RP];    // this chunk
+  __nv_bfloat16 kp[L * RP], vp[L * RP];  // the previous chunk (zero rows before the sequence)
+  float G[L * (L + 1)];                  // G[t][s], then in place gs[s][t]
+  float X[L * (L + 1)];                  // cross G'[t][s], then in place cs[s][t]
+  float a[L];
+  // Q[j][t] lives in the previous chunk's k and v rows (adjacent), free once the
+  // Gram blocks are formed
+  __device__ float* Q() { return reinterpret_cast<float*>(kp); }
+  static_assert(2 * sizeof(__nv_bfloat16) * L * RP >= sizeof(float) * L * (L + 1), "Q fits the k, v rows");
+};
+
+template <int D>
+__global__ void __launch_bounds__(NT) gram_tc_kernel(GramArgs a) {
+  constexpr int RP = D + 8;
+  constexpr int V16 = D / 8;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  GramTcSmem<D>& sm = *reinterpret_cast<GramTcSmem<D>*>(smem_raw);
+  const int bh = blockIdx.x, blk = blockIdx.y;
+  const int b = bh / a.H, h = bh % a.H;
+  if (blk >= a.count) return;
+  const int n_mine = (a.count - blk + a.nblk - 1) / a.nblk;
+  auto chunk_of = [&](int i) { return a.chunk0 + blk + i * a.nblk; };
+  const int row_stride = a.H * D;
+  const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
+  const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
+  // rows of chunk c (c >= 0) into (dk, dv); rows outside [0, T) zero-filled
+  auto load = [&](int c, __nv_bfloat16* dk, __nv_bfloat16* dv) {
+    const int t0 = c * L;
+    for (int e = threadIdx.x; e < L * V16; e += NT) {
+      const int r = e / V16, cc = (e % V16) * 8;
+      const int t = t0 + r;
+      const bool ok = (c >= 0) && (t < a.T);
+      const long long off = (long long)(ok ? t : 0) * row_stride + cc;
+      const int nbytes = ok ? 16 : 0;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dk + r * RP + cc)), "l"(k0 + off),
+                   "r"(nbytes) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(dv + r * RP + cc)), "l"(v0 + off),
+                   "r"(nbytes) : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  for (int i = 0; i < n_mine; ++i) {
+    const int c = chunk_of(i);
+    __syncthreads();  // the buffers of the previous chunk are no longer read
+    load(c, sm.k, sm.v);
+    load(c - 1, sm.kp, sm.vp);
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    gram_tile_lower<D>(sm.k, sm.v, sm.G, sm.a);
+    gram_cross<D>(sm.k, sm.v, sm.kp, sm.vp, sm.X);
+    __syncthreads();
+    suffix_rows_ilp(sm.G);  // G[t][j] = gs[j][t]
+    suffix_rows_ilp(sm.X);  // X[t][j] = cs[j][t]
+    __syncthreads();
+    float* const Qs = sm.Q();
+    prefix_rows_ilp(sm.G, 1, L + 1, Qs, L + 1);  // Q[j][t] = sum_{u < t} gs[j][u], t < L
+    __syncthreads();
+    float* out = a.out + ((long long)bh * a.nchunks + c) * kGramStride;
+    float* ogs = out;
+    float* oq = out + kPackTri;
+    float* oa = out + 2 * kPackTri;
+    float* ocs = oa + L;
+    // packed rows j (a warp each), t in [j, 64]; Q[j][64] = Q[j][63] + gs[j][63]
+    {
+      const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+      for (int j = warp; j < L; j += NW) {
+        const int base = pack_row(j);
+        for (int t = j + lane; t <= L; t += 32) {
+          ogs[base + t - j] = (t < L) ? sm.G[t * (L + 1) + j] : 0.f;
+          oq[base + t - j] = (t < L) ? Qs[j * (L + 1) + t] : Qs[j * (L + 1) + L - 1] + sm.G[(L - 1) * (L + 1) + j];
+        }
+      }
+    }
+    if (threadIdx.x < L) oa[threadIdx.x] = sm.a[threadIdx.x];
+    for (int e = threadIdx.x; e < L * L / 4; e += NT) {
+      const int j = e / (L / 4), t = (e % (L / 4)) * 4;
+      *reinterpret_cast<float4*>(ocs + j * L + t) = make_float4(sm.X[t * (L + 1) + j], sm.X[(t + 1) * (L + 1) + j],
+                                                                sm.X[(t + 2) * (L + 1) + j], sm.X[(t + 3) * (L + 1) + j]);
+    }
+    const bool publish = a.ready && (i < 4 || (i & 3) == 3 || i + 1 == n_mine);
+    if (publish) asm volatile("fence.proxy.async.global;" ::: "memory");
+    __syncthreads();
+    if (publish && threadIdx.x == 0) {
+      __threadfence();
+      st_release_gpu(a.ready + (long long)bh * a.nblk + blk, i + 1);
+    }
+  }
+}
+
 template <int D>
 static cudaError_t launch_gram_t(const GramArgs& a, cudaStream_t s) {
-  const size_t smem = sizeof(GramSmem<D>);
-  auto kern = gram_kernel<D>;
+  const size_t smem = a.packed ? sizeof(GramTcSmem<D>) : sizeof(GramSmem<D>);
+  auto kern = a.packed ? gram_tc_kernel<D> : gram_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   if (a.nblk < 1 || a.nblk > kMaxGramBlk || (long long)a.nblk * a.per_blk < a.count) return cudaErrorInvalidValue;
@@ -1333,9 +1452,10 @@ int scan_mma_resident_streams(int BH, int d) {  // cached per device and kernel 
 }
 
 __global__ void gate_kernel(const int32_t* started, int n, int32_t* status) {
-  const long long t0 = clock64(), lim = sm100::wait_limit(status);
+  const long long t0 = clock64();
+  long long lim = -1;
   while (ld_acquire_gpu(started) < n)
-    if (*(volatile int32_t*)status != 0 || clock64() - t0 > lim) {
+    if (*(volatile int32_t*)status != 0 || sm100::wait_expired(t0, lim, status)) {
       atomicCAS(status, 0, 5);  // a failure reported elsewhere keeps its code
       return;
     }
@@ -1348,6 +1468,7 @@ cudaError_t preload_scan_kernels() {
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2, true>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1, true>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_kernel<128>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, gram_tc_kernel<128>)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, gate_kernel);
 }
 cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStream_t s) {

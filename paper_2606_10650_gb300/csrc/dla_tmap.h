@@ -50,4 +50,19 @@ inline bool tmap_pool(CUtensorMap* m, const void* base, long long rows) {
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// fp32 states as rows of 128 floats (the cache's [d_v][d_k] states): box (32, 128)
+// with the 128-byte swizzle (a 128-row tile of 32 columns, 16 KB).
+inline bool tmap_states(CUtensorMap* m, const void* base, long long rows) {
+  auto fn = tmap_encode_fn();
+  if (!fn) return false;
+  constexpr int D = 128;
+  cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)D * 4};
+  cuuint32_t box[2] = {32, 128};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace dla

@@ -25,6 +25,9 @@ from safe_inputs import safe_oracle_streams
 pytestmark = pytest.mark.gpu
 
 
+_ORACLE_CACHE = {}
+
+
 def _prefill_case(name, want_every=1):
     w = W.get(name)
     want = None
@@ -32,7 +35,10 @@ def _prefill_case(name, want_every=1):
         want = np.zeros(w.T, bool)
         want[::want_every] = True
         want[-1] = True
-    (q, k, v, lam), r = safe_oracle_streams(w, T=w.T, want_o=want)
+    key = (name, want_every)
+    if key not in _ORACLE_CACHE:  # the safe inputs and the oracle's results, once per workload
+        _ORACLE_CACHE[key] = safe_oracle_streams(w, T=w.T, want_o=want)
+    (q, k, v, lam), r = _ORACLE_CACHE[key]
     g = run_gpu(w, q, k, v, lam)
     rep = {}
     compare(w, g, r, report=rep)
@@ -50,9 +56,12 @@ def test_standard_workload_full_shape():
 
 
 @pytest.mark.timeout(900)
-def test_regime_workload_full_shape():
+@pytest.mark.parametrize("scan", ["mma", "tc"])
+def test_regime_workload_full_shape(scan, monkeypatch):
     """All 32 streams of 16384 tokens: the C = 32 cache fills and merges inside
-    read-out intervals on the tensor-core read-out."""
+    read-out intervals on the tensor-core read-out; with either scan."""
+    if scan == "tc":
+        monkeypatch.setenv("DLA_SCAN", "tc")
     _, nb, nm = _prefill_case("regime")
     assert nb > 32 * 40 and nm > 32 * 10
 

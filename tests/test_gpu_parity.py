@@ -318,3 +318,33 @@ def test_ragged_rows(case, sched, monkeypatch):
         np.testing.assert_array_equal(g["merge_log"][b, :, n:], -1)
         if n == 0:
             assert (ex["m"][b] == 0).all()
+
+
+@pytest.mark.parametrize("sched", ["concurrent", "rounds", "serial"])
+@pytest.mark.parametrize("case", ["standard_bf16", "regime_bf16", "long_churn_bf16", "many_streams_bf16"])
+def test_forward_parity_tcgen05_scan(case, sched, monkeypatch):
+    """DLA_SCAN=tc: the scan with the open state in tensor memory and its state
+    builds and y contractions on tcgen05 (the opt-in scan) gives the oracle's
+    results on every schedule."""
+    monkeypatch.setenv("DLA_SCAN", "tc")
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
+    name, ov = CASES[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+    structural_checks(w, g, w.T)
+
+
+def test_tcgen05_scan_small_workspace(monkeypatch):
+    """DLA_SCAN=tc with the smallest workspace: one read-out interval per round,
+    pools reset every round."""
+    monkeypatch.setenv("DLA_SCAN", "tc")
+    w = W.get("regime", B=1, H=2, T=1100)
+    q, k, v, lam = _safe(w)
+    p = dla.make_params(w.tau, w.C)
+    nb = dla.dla_forward_min_workspace(p, w.B, w.T, w.H, w.d, w.d, dla.DLA_BF16, True)
+    g = run_gpu(w, q, k, v, lam, ws_bytes=nb)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
