@@ -67,7 +67,7 @@
 extern "C" {
 #endif
 
-#define DLA_VERSION 2
+#define DLA_VERSION 3
 
 typedef enum {
   DLA_OK = 0,
@@ -195,6 +195,33 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
                        int dv, const void* q, const void* k, const void* v, const float* lam,
                        void* o, const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
                        void* workspace, size_t ws_bytes, void* stream);
+
+/* dla_forward over a packed batch of B rows of different lengths (ragged
+ * batches without padding, as in serving; Sec. 3.2's fixed-size memory per
+ * sequence makes each row an independent stream per head).  Row b holds tokens
+ * cu_seqlens[b] .. cu_seqlens[b+1] - 1 of
+ *   q, k, v   [total_tokens, H, d]   (bf16 or fp32)
+ *   lam       [total_tokens, H, C]   fp32, or NULL (all ones)
+ *   o         [total_tokens, H, d_v] (p->out_dtype), or NULL
+ * and runs exactly as a call on its own tokens would (Algorithm 1 and 2 per
+ * (row, head) stream, the read-out of Eq. capacity_bounded_output).
+ *   cu_seqlens  device int32 [B + 1], 4-byte aligned: non-decreasing offsets
+ *               with 0 <= cu_seqlens[b] and cu_seqlens[B] <= total_tokens.
+ *   max_seqlen  an upper bound of every row's length; it takes the place of T
+ *               in the workspace size (dla_forward_workspace(p, B, max_seqlen,
+ *               ...)) and in the trace layout: boundary and merge_log are
+ *               [B, H, max_seqlen], the row's tokens first, then padding
+ *               (boundary 0, merge_log -1).
+ *   cache       as in dla_forward ([B, H, C] streams, one per row and head).
+ *   p->seq_lens must be NULL.  Offsets that break the rules above are found
+ *   on the device: the row is clamped into range and the call's status is
+ *   DLA_ERR_DEVICE_CHECK (dla_sync_status).  Inputs must be device-resident
+ *   (there is no host-buffer variant).  DLA_SCAN=tc does not apply. */
+dla_status dla_forward_varlen(const dla_params* p, dla_dtype in_dtype, int B, int max_seqlen,
+                              long long total_tokens, const int32_t* cu_seqlens, int H, int dk, int dv,
+                              const void* q, const void* k, const void* v, const float* lam, void* o,
+                              const dla_cache* cache, uint8_t* boundary, int32_t* merge_log,
+                              void* workspace, size_t ws_bytes, void* stream);
 
 /* dla_forward for callers that cannot allocate device memory (the paper has
  * no counterpart: this is a deployment convenience).  Some callers cannot

@@ -79,7 +79,7 @@ struct FwdPlan {
   int persistent;
   int nbuf;          // pools (1 persistent, 2 reset with several rounds)
   int pool_cap;      // pool entries per stream, per pool
-  size_t off_status, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram,
+  size_t off_status, off_rows, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram,
       off_progress, off_pool, pool_bytes;
   int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
   size_t total;
@@ -114,6 +114,8 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   }
   size_t off = 0;
   P.off_status = off;    off = align256(off + 256);
+  // packed batches: each row's length and first token row (2 x B int32)
+  P.off_rows = off;      off = align256(off + 2 * (size_t)B * sizeof(int32_t));
   P.off_bnd = off;       if (need_trace) off = align256(off + BH * T);
   P.off_mlog = off;      if (need_trace) off = align256(off + BH * T * sizeof(int32_t));
   P.off_cache = off;     if (need_cache) off = align256(off + cache_layout(B, H, C, d, d).total);
@@ -616,20 +618,27 @@ static int concurrent_free_sms(int B, int H, int d, bool scan_tc, cudaError_t* e
 // dla_forward; with io, q, k, v and lambda come from host memory into the
 // device buffers q, k, v, lam (workspace), streamed beside the scan on the
 // concurrent schedule, otherwise copied before anything else.
+// A packed batch: row b holds tokens cu[b] .. cu[b+1] - 1 of q, k, v, lambda and o
+// (device int32 offsets), `total` token rows in all.
+struct Varlen {
+  const int32_t* cu;
+  long long total;
+};
+
 static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
                                  const void* q, const void* k, const void* v, const float* lam, void* o,
                                  const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
-                                 size_t ws_bytes, void* stream, HostIO* io, int32_t** word);
+                                 size_t ws_bytes, void* stream, HostIO* io, const Varlen* vl, int32_t** word);
 
 // forward_launch, then the call's device status folded into its stream's status
 // word once every kernel of the call has run (the stream waits for them).
 static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
                                const void* q, const void* k, const void* v, const float* lam, void* o,
                                const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
-                               size_t ws_bytes, void* stream, HostIO* io) {
+                               size_t ws_bytes, void* stream, HostIO* io, const Varlen* vl = nullptr) {
   int32_t* word = nullptr;
   dla_status s = forward_launch(p, in_dtype, B, T, H, dk, dv, q, k, v, lam, o, cache, boundary, merge_log, workspace,
-                                ws_bytes, stream, io, &word);
+                                ws_bytes, stream, io, vl, &word);
   if (s != DLA_OK) return s;
   cudaError_t e = timed(DLA_K_STATUS, (cudaStream_t)stream, [&] {
     status_fold_kernel<<<1, 1, 0, (cudaStream_t)stream>>>((const int32_t*)workspace, word);
@@ -642,7 +651,7 @@ static dla_status forward_impl(const dla_params* p, dla_dtype in_dtype, int B, i
 static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
                                  const void* q, const void* k, const void* v, const float* lam, void* o,
                                  const dla_cache* cache, uint8_t* boundary, int32_t* merge_log, void* workspace,
-                                 size_t ws_bytes, void* stream, HostIO* io, int32_t** word) {
+                                 size_t ws_bytes, void* stream, HostIO* io, const Varlen* vl, int32_t** word) {
   dla_status s = check_params(p);
   if (s != DLA_OK) return s;
   if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
@@ -650,6 +659,13 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   if ((s = check_shape(dk, dv)) != DLA_OK) return s;
   const int d = dk, C = p->capacity;
   if ((long long)B * T * H * d >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
+  if (vl) {
+    if (!vl->cu || !aligned(vl->cu, 4)) return fail(DLA_ERR_INVALID_ARG, "cu_seqlens must be non-NULL and 4-byte aligned");
+    if (p->seq_lens) return fail(DLA_ERR_INVALID_ARG, "a packed batch takes its lengths from cu_seqlens: seq_lens must be NULL");
+    if (vl->total < 0 || vl->total >= (1LL << 31)) return fail(DLA_ERR_UNSUPPORTED, "total_tokens must be in [0, 2^31)");
+    if (vl->total * H * d >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
+    if (io) return fail(DLA_ERR_UNSUPPORTED, "packed batches take device-resident inputs");
+  }
   if (!k || !v) return fail(DLA_ERR_INVALID_ARG, "k and v must be non-NULL");
   const bool with_output = (o != nullptr);
   if (with_output && !q) return fail(DLA_ERR_INVALID_ARG, "q must be non-NULL when o is requested");
@@ -708,6 +724,18 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     e = timed(DLA_K_INIT, st, [&] { return dla::launch_init_cache(live.slot, live.n, live.ibar, live.m, B * H, C, st); });
     if (e != cudaSuccess) return cuda_fail(e, "init_cache launch");
   }
+  // per-row lengths (ragged rows in the padded layout, or a packed batch's rows,
+  // checked on the device) and, for a packed batch, each row's first token row
+  const int32_t* seq_lens = p->seq_lens;
+  const int32_t* row_start = nullptr;
+  if (vl) {
+    int32_t* lens_ws = (int32_t*)(ws + P.off_rows);
+    int32_t* start_ws = lens_ws + B;
+    e = timed(DLA_K_INIT, st, [&] { return dla::launch_varlen_rows(vl->cu, B, T, vl->total, lens_ws, start_ws, status, st); });
+    if (e != cudaSuccess) return cuda_fail(e, "packed rows launch");
+    seq_lens = lens_ws;
+    row_start = start_ws;
+  }
 
   dla::ScanArgs sa;
   memset(&sa, 0, sizeof(sa));
@@ -719,7 +747,8 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   sa.states = live.states; sa.slot = live.slot; sa.n = live.n; sa.ibar = live.ibar; sa.m = live.m;
   sa.boundary = bnd; sa.merge_log = mlog;
   sa.status = status;
-  sa.seq_lens = p->seq_lens;
+  sa.seq_lens = seq_lens;
+  sa.row_start = row_start;
   const bool in_bf16 = (in_dtype == DLA_BF16);
   const bool tc = use_tc(in_dtype, d);
   const bool pool_bf16 = tc;
@@ -737,7 +766,9 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   ra.B = B; ra.T = T; ra.H = H; ra.C = C;
   ra.boundary = bnd; ra.merge_log = mlog;
   ra.status = status;
-  ra.seq_lens = p->seq_lens;
+  ra.seq_lens = seq_lens;
+  ra.row_start = row_start;
+  ra.total_rows = vl ? vl->total : 0;
   ra.interval = P.interval;
   sa.snap_chunks = P.interval / dla::kScanL;
   sa.pool_cap = P.pool_cap;
@@ -755,7 +786,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   // (one CTA per stream) where the Gram pre-pass runs over whole rows of
   // resident inputs (it is correct but slower on the benchmark workloads:
   // its per-chunk chain is bound by the latency of small tensor-core groups).
-  const bool scan_tc = tc && P.gram_chunks > 0 && !p->seq_lens && !stream_in && scan_tc_requested();
+  const bool scan_tc = tc && P.gram_chunks > 0 && !seq_lens && !stream_in && scan_tc_requested();
   auto launch_main_scan = [&](cudaStream_t s_) -> cudaError_t {
     return scan_tc ? dla::launch_scan_tc(sa, s_) : dla::launch_scan_mma(sa, d, pool_bf16, s_);
   };
@@ -774,6 +805,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     // pre-pass, whole scan, read-out, one after another on the scan stream
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.seq_lens = seq_lens; ga.row_start = row_start;
     ga.out = (float*)(ws + P.off_gram);
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = nullptr;
@@ -841,6 +873,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     const int ctas = scan_tc ? 1 : dla::scan_mma_ctas_per_stream(B * H, d);
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.seq_lens = seq_lens; ga.row_start = row_start;
     ga.out = (float*)(ws + P.off_gram);
     ga.chunk0 = 0; ga.count = P.gram_chunks;
     ga.ready = gram_ready;
@@ -952,6 +985,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     // the scan stream; the rest run on the read-out stream while that scan goes.
     dla::GramArgs ga;
     ga.k = k; ga.v = v; ga.B = B; ga.T = T; ga.H = H; ga.nchunks = P.gram_chunks;
+    ga.seq_lens = seq_lens; ga.row_start = row_start;
     ga.out = (float*)(ws + P.off_gram);
     ga.ready = nullptr;
     ga.packed = scan_tc ? 1 : 0;
@@ -1018,6 +1052,15 @@ dla_status dla_forward(const dla_params* p, dla_dtype in_dtype, int B, int T, in
                        uint8_t* boundary, int32_t* merge_log, void* workspace, size_t ws_bytes, void* stream) {
   return forward_impl(p, in_dtype, B, T, H, dk, dv, q, k, v, lam, o, cache, boundary, merge_log, workspace, ws_bytes,
                       stream, nullptr);
+}
+
+dla_status dla_forward_varlen(const dla_params* p, dla_dtype in_dtype, int B, int max_seqlen, long long total_tokens,
+                              const int32_t* cu_seqlens, int H, int dk, int dv, const void* q, const void* k,
+                              const void* v, const float* lam, void* o, const dla_cache* cache, uint8_t* boundary,
+                              int32_t* merge_log, void* workspace, size_t ws_bytes, void* stream) {
+  const Varlen vl{cu_seqlens, total_tokens};
+  return forward_impl(p, in_dtype, B, max_seqlen, H, dk, dv, q, k, v, lam, o, cache, boundary, merge_log, workspace,
+                      ws_bytes, stream, nullptr, &vl);
 }
 
 // Device buffers of dla_forward_host at the end of its workspace: q, k, v,

@@ -87,6 +87,11 @@ __device__ __forceinline__ int row_t_end(const int32_t* seq_lens, int b, int t_b
   if (!seq_lens) return t_end;
   return max(t_begin, min(t_end, __ldg(seq_lens + b)));
 }
+// Token row of the first token of batch row b: b * T in the padded layout, or
+// row_start[b] in the packed one.
+__device__ __forceinline__ long long row_tok0(const int32_t* row_start, int b, int T) {
+  return row_start ? (long long)__ldg(row_start + b) : (long long)b * T;
+}
 // Decision trace of padding tokens [t0, t1) of one stream: no boundary, no merge.
 __device__ __forceinline__ void fill_padding_trace(uint8_t* bnd, int32_t* mlog, int t0, int t1, int i0, int ni) {
   for (int t = t0 + i0; t < t1; t += ni) {

@@ -321,4 +321,31 @@ cudaError_t launch_init_cache(int32_t* slot, int32_t* n, double* ibar, int32_t* 
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- packed rows
+// Row lengths and first token rows of a packed batch from its cumulative
+// offsets (see launch_varlen_rows).
+__global__ void varlen_rows_kernel(const int32_t* cu, int B, int T, long long total, int32_t* lens, int32_t* start,
+                                   int32_t* status) {
+  for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < B; b += gridDim.x * blockDim.x) {
+    long long s0 = cu[b], s1 = cu[b + 1];
+    const bool bad = s0 < 0 || s1 < s0 || s1 > total || s1 - s0 > T;
+    if (bad) {
+      atomicCAS(status, 0, 6);
+      s0 = s0 < 0 ? 0 : (s0 > total ? total : s0);
+      s1 = s1 < s0 ? s0 : (s1 > total ? total : s1);
+      if (s1 - s0 > T) s1 = s0 + T;
+    }
+    start[b] = (int32_t)s0;
+    lens[b] = (int32_t)(s1 - s0);
+  }
+}
+
+cudaError_t launch_varlen_rows(const int32_t* cu, int B, int T, long long total, int32_t* lens, int32_t* start,
+                               int32_t* status, cudaStream_t s) {
+  int blocks = (B + 255) / 256;
+  if (blocks > 1024) blocks = 1024;
+  varlen_rows_kernel<<<blocks, 256, 0, s>>>(cu, B, T, total, lens, start, status);
+  return cudaGetLastError();
+}
+
 }  // namespace dla

@@ -85,6 +85,10 @@ struct ScanArgs {
   const int32_t* piece_ready;
   int piece_chunks;
   const int32_t* seq_lens;  // [B] tokens of each row (padding after them), or nullptr: T each
+  // [B] token row of each batch row's first token (the packed layout: rows of
+  // seq_lens[b] tokens one after another), or nullptr: b * T (the padded layout).
+  // Set only together with seq_lens.
+  const int32_t* row_start;
   int32_t* progress;     // [B*H][2] intervals completed by each CTA of the stream, or nullptr
   int32_t* started;      // counter of the scan CTAs that have started, or nullptr
   int32_t* status;       // device status word (0 = ok)
@@ -107,6 +111,10 @@ struct GramArgs {
   float* out;            // [B*H][nchunks][kGramBlock]: gs (64 x 64), Q (64 x 64), a (64); packed: [kGramBlockTc]
   int32_t* ready;        // [B*H][nblk] chunks of the block written so far (published after its first four, then every fourth), or nullptr
   int packed;            // 1: the tensor-core scan's layout (kGramBlockTc floats per chunk, with the cross table)
+  // per-row lengths and first token rows (as in ScanArgs), or nullptr: rows of T
+  // tokens at b * T.  Rows past a row's length are zero-filled, not read.
+  const int32_t* seq_lens;
+  const int32_t* row_start;
 };
 constexpr int kMaxGramBlk = 64;  // blocks per stream of one Gram launch, at most
 constexpr int kGramCtasPerSm = 3;  // resident Gram CTAs per SM (shared memory)
@@ -140,6 +148,8 @@ struct ReadoutArgs {
   int32_t* out_done;
   int out_piece_pairs;
   const int32_t* seq_lens;  // [B] tokens of each row (padding after them), or nullptr: T each
+  const int32_t* row_start; // [B] first token row of each batch row (packed layout), or nullptr: b * T
+  long long total_rows;     // token rows of q, k, v, lambda and o in the packed layout (row_start set)
   int lam_l2;  // 1: lambda arrives while the kernel runs (streamed inputs): read it through L2
   int32_t* status;          // device status word
 };
@@ -163,6 +173,14 @@ struct DecodeArgs {
   int32_t* merge_idx;    // [B, H] or nullptr
   int32_t* status;       // device status word of the call's stream (6 when the cache is inconsistent)
 };
+
+// Per-row lengths and first token rows of a packed batch from its cumulative
+// offsets cu[0..B] (device int32): lens[b] = cu[b+1] - cu[b] and start[b] = cu[b],
+// checked (0 <= cu[b] <= cu[b+1] <= total, length <= T); a row that fails the
+// check sets status 6 and is clamped into range, so no kernel reads outside
+// the total rows.
+cudaError_t launch_varlen_rows(const int32_t* cu, int B, int T, long long total, int32_t* lens, int32_t* start,
+                               int32_t* status, cudaStream_t s);
 
 // Records a formatted message as the calling thread's dla_last_error() and
 // returns s (for entry points defined outside dla_api.cu).

@@ -68,7 +68,7 @@ __global__ void __launch_bounds__(NT, 1) readout_simt_kernel(ReadoutArgs a) {
   const int Lc = min(L, row_t_end(a.seq_lens, b, a.t_begin, a.t_end) - c0);
   if (Lc <= 0) return;  // the interval lies past this row's length: padding, o not written
   const int row_stride = a.H * D;
-  const long long tok0 = ((long long)b * a.T + c0) * a.H + h;  // row index of token c0
+  const long long tok0 = (row_tok0(a.row_start, b, a.T) + c0) * a.H + h;  // row index of token c0
   const int m0 = a.snap_m0[(long long)bh * a.snap_stride + a.snap_base + s];
   const uint8_t* bnd = a.boundary + (long long)bh * a.T + c0;
   const int32_t* mlog = a.merge_log + (long long)bh * a.T + c0;

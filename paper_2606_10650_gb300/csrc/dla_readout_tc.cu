@@ -172,6 +172,12 @@ __global__ void __launch_bounds__(NT, 1)
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const int sA = 2 * pair;
+  // token row of the row's token 0, and the TMA coordinates of it: (token, batch)
+  // = (t, b) in the padded layout, (row_start[b] + t, 0) in the packed one (the
+  // per-row-length instance only)
+  const long long tok0 = kRagged ? row_tok0(a.row_start, b, a.T) : (long long)b * a.T;
+  const bool packed = kRagged && a.row_start != nullptr;
+  const int tma_t = packed ? (int)tok0 : 0, tma_b = packed ? 0 : b;
   // this row's end (padding after it)
   const int t_end = kRagged ? row_t_end(a.seq_lens, b, a.t_begin, a.t_end) : a.t_end;
   if constexpr (kRagged) {
@@ -238,11 +244,11 @@ __global__ void __launch_bounds__(NT, 1)
     prefetch_tmap(&tmV);
     prefetch_tmap(&tmS);
     mbar_expect_tx(&sm.bar_q, (hasB ? 4 : 2) * kTile);
-    tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, c0A, b);
-    tma_load_4d(sm.Q[0][1], &tmQ, &sm.bar_q, 64, h, c0A, b);
+    tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, tma_t + c0A, tma_b);
+    tma_load_4d(sm.Q[0][1], &tmQ, &sm.bar_q, 64, h, tma_t + c0A, tma_b);
     if (hasB) {
-      tma_load_4d(sm.Q[1][0], &tmQ, &sm.bar_q, 0, h, c0B, b);
-      tma_load_4d(sm.Q[1][1], &tmQ, &sm.bar_q, 64, h, c0B, b);
+      tma_load_4d(sm.Q[1][0], &tmQ, &sm.bar_q, 0, h, tma_t + c0B, tma_b);
+      tma_load_4d(sm.Q[1][1], &tmQ, &sm.bar_q, 64, h, tma_t + c0B, tma_b);
     }
   }
   for (int i = tid; i < 2 * kMaxC; i += NT) {
@@ -306,18 +312,18 @@ __global__ void __launch_bounds__(NT, 1)
     if (lane == 0) {
       int issued[NHS];  // uses of each stage so far
       mbar_expect_tx(&sm.full[0], 2 * kTile);
-      tma_load_4d(sm.hs[0][0], &tmK, &sm.full[0], 0, h, c0A, b);
-      tma_load_4d(sm.hs[0][1], &tmK, &sm.full[0], 64, h, c0A, b);
+      tma_load_4d(sm.hs[0][0], &tmK, &sm.full[0], 0, h, tma_t + c0A, tma_b);
+      tma_load_4d(sm.hs[0][1], &tmK, &sm.full[0], 64, h, tma_t + c0A, tma_b);
       mbar_expect_tx(&sm.full[2], 2 * kTile);
-      tma_load_4d(sm.hs[2][0], &tmV, &sm.full[2], 0, h, c0A, b);
-      tma_load_4d(sm.hs[2][1], &tmV, &sm.full[2], 64, h, c0A, b);
+      tma_load_4d(sm.hs[2][0], &tmV, &sm.full[2], 0, h, tma_t + c0A, tma_b);
+      tma_load_4d(sm.hs[2][1], &tmV, &sm.full[2], 64, h, tma_t + c0A, tma_b);
       if (hasB) {
         mbar_expect_tx(&sm.full[1], 2 * kTile);
-        tma_load_4d(sm.hs[1][0], &tmK, &sm.full[1], 0, h, c0B, b);
-        tma_load_4d(sm.hs[1][1], &tmK, &sm.full[1], 64, h, c0B, b);
+        tma_load_4d(sm.hs[1][0], &tmK, &sm.full[1], 0, h, tma_t + c0B, tma_b);
+        tma_load_4d(sm.hs[1][1], &tmK, &sm.full[1], 64, h, tma_t + c0B, tma_b);
         mbar_expect_tx(&sm.full[3], 2 * kTile);
-        tma_load_4d(sm.hs[3][0], &tmV, &sm.full[3], 0, h, c0B, b);
-        tma_load_4d(sm.hs[3][1], &tmV, &sm.full[3], 64, h, c0B, b);
+        tma_load_4d(sm.hs[3][0], &tmV, &sm.full[3], 0, h, tma_t + c0B, tma_b);
+        tma_load_4d(sm.hs[3][1], &tmV, &sm.full[3], 64, h, tma_t + c0B, tma_b);
       } else {  // first phase complete without data: the stages' later uses keep their parity
         mbar_arrive(&sm.full[1]);
         mbar_arrive(&sm.full[3]);
@@ -427,7 +433,7 @@ __global__ void __launch_bounds__(NT, 1)
     const int etid = ew * 32 + lane;      // 0..511
     const int c0s = c0_of(side), Lcs = Lc_of(side);
     const bool side_in = (side == 0 || hasB);  // warp-uniform
-    const long long rowbase = ((long long)b * a.T + c0s) * a.H + h;
+    const long long rowbase = (tok0 + c0s) * a.H + h;
 
     if (etid < 2 * L) {  // both intervals' boundary flags and merge indices
       const int sd = etid / L, tt = etid % L;
@@ -597,9 +603,14 @@ __global__ void __launch_bounds__(NT, 1)
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
   CUtensorMap mq, mk, mv, ms;
   const long long rows = (long long)a.B * a.H * a.pool_cap * 2 * D;
-  if (!tmap_tokens(&mq, a.q, a.B, a.T, a.H) || !tmap_tokens(&mk, a.k, a.B, a.T, a.H) ||
-      !tmap_tokens(&mv, a.v, a.B, a.T, a.H) || !tmap_pool(&ms, a.pool, rows))
+  // packed layout: one batch coordinate over all token rows
+  const int mb = a.row_start ? 1 : a.B;
+  const long long mt = a.row_start ? (a.total_rows > 0 ? a.total_rows : 1) : a.T;
+  if (mt >= (1LL << 31)) return cudaErrorInvalidValue;
+  if (!tmap_tokens(&mq, a.q, mb, (int)mt, a.H) || !tmap_tokens(&mk, a.k, mb, (int)mt, a.H) ||
+      !tmap_tokens(&mv, a.v, mb, (int)mt, a.H) || !tmap_pool(&ms, a.pool, rows))
     return cudaErrorInvalidValue;
+  if (a.row_start && !a.seq_lens) return cudaErrorInvalidValue;  // the packed layout needs per-row lengths
   const size_t smem = sizeof(TcSmem) + 1024;
   const bool stream = a.lam_l2 || a.out_done, ragged = a.seq_lens != nullptr;
   auto kern = stream ? (ragged ? readout_tc_kernel<true, true> : readout_tc_kernel<true, false>)

@@ -128,8 +128,9 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const float Df = (float)(D * D);
-  const Tin* kbase = reinterpret_cast<const Tin*>(a.k) + ((long long)b * a.T * a.H + h) * D;
-  const Tin* vbase = reinterpret_cast<const Tin*>(a.v) + ((long long)b * a.T * a.H + h) * D;
+  const long long tok0 = row_tok0(a.row_start, b, a.T);  // token row of the row's first token
+  const Tin* kbase = reinterpret_cast<const Tin*>(a.k) + (tok0 * a.H + h) * D;
+  const Tin* vbase = reinterpret_cast<const Tin*>(a.v) + (tok0 * a.H + h) * D;
   const int row_stride = a.H * D;
   float* states = a.states + (long long)bh * C * D * D;
   constexpr long long kEntry = (long long)pool_parts<Tpool>() * D * D;  // elements per pool entry

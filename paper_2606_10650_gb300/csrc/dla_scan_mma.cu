@@ -450,8 +450,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
   const float Df = (float)(D * D);
-  const __nv_bfloat16* kbase = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
-  const __nv_bfloat16* vbase = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
+  // token row of the row's first token (the packed layout only in the per-row-length instance)
+  const long long tok0 = kRagged ? row_tok0(a.row_start, b, a.T) : (long long)b * a.T;
+  const __nv_bfloat16* kbase = reinterpret_cast<const __nv_bfloat16*>(a.k) + (tok0 * a.H + h) * D;
+  const __nv_bfloat16* vbase = reinterpret_cast<const __nv_bfloat16*>(a.v) + (tok0 * a.H + h) * D;
   const int row_stride = a.H * D;
   const int rbase = rank * R;         // first state row of this CTA
   float* states = a.states + (long long)bh * C * D * D;
@@ -1141,18 +1143,23 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
   const int n_mine = (a.count - blk + a.nblk - 1) / a.nblk;
   auto chunk_of = [&](int i) { return a.chunk0 + blk + i * a.nblk; };
   const int row_stride = a.H * D;
-  const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + ((long long)b * a.T * a.H + h) * D;
-  const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + ((long long)b * a.T * a.H + h) * D;
-  auto load = [&](int c) {  // rows past the sequence end are zero-filled
-    const int t0 = c * L, valid = min(L, a.T - t0);
+  const long long tok0 = row_tok0(a.row_start, b, a.T);
+  const __nv_bfloat16* k0 = reinterpret_cast<const __nv_bfloat16*>(a.k) + (tok0 * a.H + h) * D;
+  const __nv_bfloat16* v0 = reinterpret_cast<const __nv_bfloat16*>(a.v) + (tok0 * a.H + h) * D;
+  const int row_len = a.seq_lens ? max(0, min(a.T, __ldg(a.seq_lens + b))) : a.T;
+  auto load = [&](int c) {  // rows past the row's end are zero-filled, not read
+    const int t0 = c * L, valid = min(L, row_len - t0);
+    const __nv_bfloat16* kz = reinterpret_cast<const __nv_bfloat16*>(a.k);  // address of a zero-filled row
+    const __nv_bfloat16* vz = reinterpret_cast<const __nv_bfloat16*>(a.v);
     for (int e = threadIdx.x; e < L * V16; e += NT) {
       const int r = e / V16, cc = (e % V16) * 8;
-      const long long off = (long long)(t0 + (r < valid ? r : 0)) * row_stride + cc;
-      const int nbytes = (r < valid) ? 16 : 0;
+      const bool in = r < valid;
+      const long long off = (long long)(t0 + r) * row_stride + cc;
+      const int nbytes = in ? 16 : 0;
       asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.k + r * RP + cc)),
-                   "l"(k0 + off), "r"(nbytes) : "memory");
+                   "l"(in ? k0 + off : kz), "r"(nbytes) : "memory");
       asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(su32(sm.v + r * RP + cc)),
-                   "l"(v0 + off), "r"(nbytes) : "memory");
+                   "l"(in ? v0 + off : vz), "r"(nbytes) : "memory");
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };

@@ -22,7 +22,7 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
             "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc",
-            "dla_forward_host_workspace", "dla_forward_host", "dla_sync_status"]
+            "dla_forward_host_workspace", "dla_forward_host", "dla_sync_status", "dla_forward_varlen"]
 KERNELS = ["scan", "readout", "decode", "init", "gram", "gate", "status"]
 
 
@@ -77,6 +77,8 @@ def lib():
         L.dla_forward_host_workspace.argtypes = [P, ci, ci, ci, ci, ci, ci, ci]
         L.dla_forward_host.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp, sz, vp]
         L.dla_sync_status.argtypes = [vp]
+        L.dla_forward_varlen.argtypes = [P, ci, ci, ci, ctypes.c_longlong, vp, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp,
+                                         vp, vp, sz, vp]
         L.dla_timing_enable.argtypes = [ci]
         L.dla_timing_read.argtypes = [ctypes.POINTER(ci), ctypes.POINTER(ctypes.c_double), ci]
         _LIB = L
@@ -238,6 +240,34 @@ def dla_forward(params, q, k, v, lam=None, o=None, cache=None, boundary=None, me
     st = lib().dla_forward(ctypes.byref(params), dt, B, T, H, d, d, _ptr(q), _ptr(k), _ptr(v), _ptr(lam), _ptr(o),
                            ctypes.byref(cache.c) if cache is not None else None, _ptr(boundary), _ptr(merge_log),
                            ctypes.c_void_p(base), nb, _stream(stream))
+    _check(st)
+    return workspace
+
+
+def dla_forward_varlen(params, cu_seqlens, max_seqlen, q, k, v, lam=None, o=None, cache=None, boundary=None,
+                       merge_log=None, workspace=None, stream=None):
+    """Raw call of dla_forward_varlen (a packed batch).  cu_seqlens: int32 CUDA
+    tensor [B + 1]; q, k, v: [total_tokens, H, d] contiguous CUDA tensors (bf16
+    or fp32); lam [total_tokens, H, C] fp32 or None; o [total_tokens, H, d] or
+    None; boundary [B, H, max_seqlen] uint8, merge_log [B, H, max_seqlen] int32
+    or None; workspace as for dla_forward (sized with T = max_seqlen)."""
+    Ttot, H, d = k.shape
+    B = cu_seqlens.numel() - 1
+    dt = _dtype_code(k)
+    if cu_seqlens.dtype != torch.int32:
+        raise ValueError("cu_seqlens must be int32")
+    for t in (q, k, v, lam, o, boundary, merge_log, cu_seqlens):
+        if t is not None and not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    if workspace is None:
+        nb = dla_forward_workspace(params, B, max_seqlen, H, d, d, dt, o is not None)
+        buf, base = _aligned_workspace(nb, k.device)
+        workspace = (buf, base, nb)
+    _, base, nb = workspace
+    st = lib().dla_forward_varlen(ctypes.byref(params), dt, B, int(max_seqlen), int(Ttot), _ptr(cu_seqlens), H, d, d,
+                                  _ptr(q), _ptr(k), _ptr(v), _ptr(lam), _ptr(o),
+                                  ctypes.byref(cache.c) if cache is not None else None, _ptr(boundary),
+                                  _ptr(merge_log), ctypes.c_void_p(base), nb, _stream(stream))
     _check(st)
     return workspace
 

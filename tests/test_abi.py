@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     for n in _declared():
         assert hasattr(L, n), n
     assert set(_declared()) == set(dla.EXPORTED)
-    assert L.dla_version() == 2
+    assert L.dla_version() == 3
 
 
 def _fake(addr=1 << 20):
@@ -106,6 +106,25 @@ def test_params_layout_and_seq_lens_checks(L):
     q.seq_lens = (1 << 20) + 2  # not 4-byte aligned
     assert _fwd(L, q) == 1
     assert b"seq_lens" in L.dla_last_error()
+
+
+def test_packed_batch_argument_errors(L):
+    p = dla.make_params(0.6, 8)
+
+    def fv(q=p, cu=True, total=100, ws_bytes=1 << 40, cu_addr=1 << 22):
+        return L.dla_forward_varlen(ctypes.byref(q), dla.DLA_BF16, 2, 64, total, _fake(cu_addr) if cu else None, 2,
+                                    128, 128, _fake(), _fake(), _fake(), None, _fake(), None, None, None,
+                                    _fake(1 << 24), ws_bytes, None)
+    assert fv(cu=False) == 1
+    assert b"cu_seqlens" in L.dla_last_error()
+    assert fv(cu_addr=(1 << 22) + 2) == 1          # offsets not 4-byte aligned
+    assert fv(total=-1) == 2
+    assert fv(total=1 << 31) == 2
+    r = dla.make_params(0.6, 8)
+    r.seq_lens = 1 << 21
+    assert fv(q=r) == 1                             # lengths come from the offsets only
+    assert b"seq_lens" in L.dla_last_error()
+    assert fv(ws_bytes=1024) == 3
 
 
 def test_kernel_kinds_match_the_header():

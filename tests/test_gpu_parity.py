@@ -320,6 +320,117 @@ def test_ragged_rows(case, sched, monkeypatch):
             assert (ex["m"][b] == 0).all()
 
 
+PACKED = {
+    # name: (workload, overrides, per-row lengths); max_seqlen = T
+    "regime_bf16": ("regime", dict(B=4, H=2, T=1300), [1300, 517, 1, 640]),
+    "standard_bf16": ("standard", dict(B=4, H=2, T=700), [0, 700, 333, 64]),
+    "d64_bf16": ("standard", dict(B=3, H=2, T=700, d=64, C=8, tau=1.4215), [257, 0, 700]),
+    "d128_fp32": ("tiny", dict(B=2, H=2, T=300, d=128, C=6, tau=1.4142), [129, 300]),
+}
+
+
+def _pack(x, lens):
+    """Rows x[b, :lens[b]] one after another: [sum(lens), ...]."""
+    return np.ascontiguousarray(np.concatenate([x[b, :n] for b, n in enumerate(lens)], axis=0))
+
+
+@pytest.mark.parametrize("sched", ["concurrent", "rounds", "serial"])
+@pytest.mark.parametrize("case", list(PACKED))
+def test_packed_rows(case, sched, monkeypatch):
+    """Packed batches (dla_forward_varlen): the rows of different lengths lie one
+    after another in q, k, v, lambda and o ([total_tokens, H, ...], offsets
+    cu_seqlens); each row gives the oracle's results on its own tokens, the
+    trace is padded per stream, and every value equals the padded layout's
+    (dla_params.seq_lens) on the same rows."""
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
+    name, ov, lens = PACKED[case]
+    w = W.get(name, **ov)
+    q, k, v, lam = _safe(w)
+    dev = torch.device("cuda:0")
+    B, T, H = w.B, w.T, w.H
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    total = int(cu[-1])
+    qt, kt, vt, lt = upload(w, _pack(q, lens), _pack(k, lens), _pack(v, lens), _pack(lam, lens))
+    d = kt.shape[-1]
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    o = torch.full((total, H, d), float("nan"), dtype=torch.float32, device=dev)
+    bnd = torch.full((B, H, T), 7, dtype=torch.uint8, device=dev)
+    ml = torch.full((B, H, T), -7, dtype=torch.int32, device=dev)
+    cut = torch.from_numpy(cu).to(dev)
+    dla.dla_forward_varlen(p, cut, T, qt, kt, vt, lt, o, cache, bnd, ml)
+    assert dla.dla_sync_status() == 0, "device status reports a failure"
+    og = o.double().cpu().numpy()
+    assert not np.isnan(og).any(), "an output row of the packed batch was not written"
+    o_rows = np.full((B, T, H, d), np.nan)
+    for b, n in enumerate(lens):
+        o_rows[b, :n] = og[cu[b]:cu[b + 1]]
+    g = dict(o=o_rows, boundary=bnd.cpu().numpy(), merge_log=ml.cpu().numpy(), cache=cache)
+    r = dict(o=np.full((B, T, H, d), np.nan), boundary=np.zeros((B, H, T), np.uint8),
+             merge_log=np.full((B, H, T), -1, np.int32), caches={})
+    live = []
+    for b, n in enumerate(lens):
+        if n == 0:
+            continue
+        rb = oracle.forward(q[b:b + 1, :n], k[b:b + 1, :n], v[b:b + 1, :n], lam[b:b + 1, :n], tau=w.tau, C=w.C,
+                            eps=w.eps, rms_eps=w.rms_eps)
+        r["o"][b, :n] = rb["o"][0]
+        r["boundary"][b, :, :n] = rb["boundary"][0]
+        r["merge_log"][b, :, :n] = rb["merge_log"][0]
+        for h in range(H):
+            r["caches"][(b, h)] = rb["caches"][(0, h)]
+            live.append((b, h))
+    compare(w, g, r, streams=live)
+    ex = cache.export()
+    for b, n in enumerate(lens):
+        np.testing.assert_array_equal(g["boundary"][b, :, n:], 0)
+        np.testing.assert_array_equal(g["merge_log"][b, :, n:], -1)
+        if n == 0:
+            assert (ex["m"][b] == 0).all()
+    # the padded layout with the same row lengths: the same values, bit for bit
+    qp, kp, vp, lp = upload(w, q, k, v, lam)
+    cache2 = dla.Cache(B, H, w.C, d, device=dev)
+    sl = torch.tensor(lens, dtype=torch.int32, device=dev)  # must outlive the call
+    p2 = dla.make_params(w.tau, w.C, w.eps, w.rms_eps, seq_lens=sl)
+    o2 = torch.full((B, T, H, d), float("nan"), dtype=torch.float32, device=dev)
+    bnd2 = torch.empty((B, H, T), dtype=torch.uint8, device=dev)
+    ml2 = torch.empty((B, H, T), dtype=torch.int32, device=dev)
+    dla.dla_forward(p2, qp, kp, vp, lp, o2, cache2, bnd2, ml2)
+    assert dla.dla_sync_status() == 0
+    o2n = o2.double().cpu().numpy()
+    for b, n in enumerate(lens):
+        np.testing.assert_array_equal(o_rows[b, :n], o2n[b, :n])
+    np.testing.assert_array_equal(g["boundary"], bnd2.cpu().numpy())
+    np.testing.assert_array_equal(g["merge_log"], ml2.cpu().numpy())
+    ex2 = cache2.export()
+    for key in ("m", "n"):
+        np.testing.assert_array_equal(ex[key], ex2[key])
+
+
+def test_packed_offsets_out_of_range_are_reported(monkeypatch):
+    """Offsets that decrease, pass total_tokens or give a row longer than
+    max_seqlen are found on the device: those rows are clamped into range
+    (nothing is read past the packed tensors) and the call's status is 6."""
+    w = W.get("standard", B=3, H=2, T=256)
+    q, k, v, lam = _safe(w)
+    dev = torch.device("cuda:0")
+    total = 300
+    qt, kt, vt, lt = upload(w, _pack(q, [256, 44]), _pack(k, [256, 44]), _pack(v, [256, 44]), _pack(lam, [256, 44]))
+    d = kt.shape[-1]
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    for cu in ([0, 280, 300, 300], [0, 200, 150, 300], [0, 100, 300, 400]):
+        o = torch.zeros((total, w.H, d), dtype=torch.float32, device=dev)
+        cache = dla.Cache(w.B, w.H, w.C, d, device=dev)
+        dla.dla_forward_varlen(p, torch.tensor(cu, dtype=torch.int32, device=dev), w.T, qt, kt, vt, lt, o, cache)
+        assert dla.dla_sync_status() == 6, cu
+        assert torch.isfinite(o).all()
+    # a correct call on the same stream afterwards
+    o = torch.zeros((total, w.H, d), dtype=torch.float32, device=dev)
+    dla.dla_forward_varlen(p, torch.tensor([0, 256, 300, 300], dtype=torch.int32, device=dev), w.T, qt, kt, vt, lt,
+                           o, dla.Cache(w.B, w.H, w.C, d, device=dev))
+    assert dla.dla_sync_status() == 0
+
+
 @pytest.mark.parametrize("sched", ["concurrent", "rounds", "serial"])
 @pytest.mark.parametrize("case", ["standard_bf16", "regime_bf16", "long_churn_bf16", "many_streams_bf16"])
 def test_forward_parity_tcgen05_scan(case, sched, monkeypatch):
