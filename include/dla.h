@@ -67,7 +67,7 @@
 extern "C" {
 #endif
 
-#define DLA_VERSION 3
+#define DLA_VERSION 4
 
 typedef enum {
   DLA_OK = 0,
@@ -291,10 +291,41 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
                            const void* q, const void* k, const void* v, const float* lam,
                            void* o, uint8_t* boundary, int32_t* merge_idx, void* stream);
 
+/* Gradients of the read-out with the forward pass's decisions held fixed
+ * (training-shaped sequences).  The boundary and merge decisions of Algorithm 1
+ * and 2 are piecewise constant in k and v, so their derivative is zero almost
+ * everywhere; with them fixed, every state is a sum of token states over a
+ * contiguous token range and Eq. capacity_bounded_output reads
+ *   o_t = sum_{s <= t} lambda_{t, slot_t(s)} (q_t . k_s) v_s,
+ * slot_t(s) the logical slot of the state holding token s after token t.  For
+ * a loss L with grad_o = dL/do this call writes
+ *   grad_q, grad_k, grad_v [B, T, H, d] fp32 and grad_lam [B, T, H, C] fp32
+ *   (NULL: not computed; 0 for slots >= m_t),
+ * taking q, k, v [B, T, H, d] (bf16 only: DLA_ERR_UNSUPPORTED otherwise), lam
+ * [B, T, H, C] fp32 or NULL (all ones), grad_o [B, T, H, d] fp32 and the
+ * decision trace of the forward call on the same inputs (boundary [B, H, T]
+ * uint8, merge_log [B, H, T] int32).  p->capacity is the C of lam and of the
+ * trace; p->from_cache must be 0 (the sequence starts from an empty cache) and
+ * p->seq_lens NULL.  The work is quadratic in T per stream (every token pair).
+ * A trace that is not a valid replay of Algorithm 2 (a merge index outside the
+ * live pairs, a boundary into a full cache without a merge) is reported as
+ * DLA_ERR_DEVICE_CHECK through the stream's status word; the gradients are
+ * then undefined.  workspace: device memory of at least
+ * dla_backward_workspace(...) bytes, 256-byte aligned; its first 4 bytes
+ * receive the call's device status.  All pointers 16-byte aligned (lam and
+ * grad_lam 4-byte). */
+size_t dla_backward_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype);
+dla_status dla_backward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv,
+                        const void* q, const void* k, const void* v, const float* lam,
+                        const uint8_t* boundary, const int32_t* merge_log, const float* grad_o,
+                        float* grad_q, float* grad_k, float* grad_v, float* grad_lam,
+                        void* workspace, size_t ws_bytes, void* stream);
+
 /* Instrumentation (no counterpart in the paper).  Kernel kinds of the
  * library: K1 scan, K2 read-out, K3 decode, cache init, K0 Gram pre-pass, the
- * one-thread gate of the concurrent schedule, and the one-thread kernel that
- * folds a forward call's status into its stream's status word. */
+ * one-thread gate of the concurrent schedule, the one-thread kernel that
+ * folds a call's status into its stream's status word, and K4 (the three
+ * kernels of dla_backward). */
 typedef enum {
   DLA_K_SCAN = 0,
   DLA_K_READOUT = 1,
@@ -303,7 +334,8 @@ typedef enum {
   DLA_K_GRAM = 4,
   DLA_K_GATE = 5,
   DLA_K_STATUS = 6,
-  DLA_K_COUNT = 7
+  DLA_K_BACKWARD = 7,
+  DLA_K_COUNT = 8
 } dla_kernel_kind;
 
 /* enable = 1: from now on, every kernel this host thread launches through the

@@ -21,7 +21,7 @@ LIB = os.path.join(BUILD, "libdla.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 SOURCES = ["dla_api.cu", "dla_scan.cu", "dla_readout_simt.cu", "dla_decode.cu", "dla_noalloc.cu",
-           "dla_readout_tc.cu", "dla_scan_mma.cu", "dla_scan_tc.cu"]
+           "dla_readout_tc.cu", "dla_scan_mma.cu", "dla_scan_tc.cu", "dla_backward.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-ffp-contract=off",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -1161,4 +1161,63 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
   return ok();
 }
 
+size_t dla_backward_workspace(const dla_params* p, int B, int T, int H, int dk, int dv, dla_dtype in_dtype) {
+  if (!p || B < 1 || T < 1 || H < 1 || dk < 1 || dv < 1 || in_dtype != DLA_BF16) return 0;
+  return 256 + align256(dla::backward_slot_bytes((int)((long long)B * H), T));
+}
+
+dla_status dla_backward(const dla_params* p, dla_dtype in_dtype, int B, int T, int H, int dk, int dv, const void* q,
+                        const void* k, const void* v, const float* lam, const uint8_t* boundary,
+                        const int32_t* merge_log, const float* grad_o, float* grad_q, float* grad_k, float* grad_v,
+                        float* grad_lam, void* workspace, size_t ws_bytes, void* stream) {
+  dla_status s = check_params(p);
+  if (s != DLA_OK) return s;
+  if (in_dtype != DLA_BF16 && in_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad in_dtype");
+  if (in_dtype != DLA_BF16) return fail(DLA_ERR_UNSUPPORTED, "dla_backward takes bf16 q, k, v");
+  if (B < 1 || T < 1 || H < 1) return fail(DLA_ERR_INVALID_ARG, "B, T, H must be >= 1");
+  if ((s = check_shape(dk, dv)) != DLA_OK) return s;
+  if ((long long)B * H > 65535) return fail(DLA_ERR_UNSUPPORTED, "B * H must be at most 65535");
+  if ((long long)B * T * H * dk >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
+  if (p->from_cache) return fail(DLA_ERR_UNSUPPORTED, "dla_backward starts from an empty cache (from_cache = 0)");
+  if (p->seq_lens) return fail(DLA_ERR_UNSUPPORTED, "dla_backward takes whole rows (seq_lens = NULL)");
+  if (!q || !k || !v || !boundary || !merge_log || !grad_o || !grad_q || !grad_k || !grad_v)
+    return fail(DLA_ERR_INVALID_ARG, "q, k, v, boundary, merge_log, grad_o, grad_q, grad_k, grad_v must be non-NULL");
+  const void* a16[] = {q, k, v, grad_o, grad_q, grad_k, grad_v};
+  for (const void* x : a16)
+    if (!aligned(x, 16)) return fail(DLA_ERR_INVALID_ARG, "q, k, v and the gradients of o, q, k, v must be 16-byte aligned");
+  if ((lam && !aligned(lam, 4)) || (grad_lam && !aligned(grad_lam, 4)))
+    return fail(DLA_ERR_INVALID_ARG, "lambda and its gradient must be 4-byte aligned");
+  if (!workspace) return fail(DLA_ERR_WORKSPACE, "workspace is NULL");
+  if (!aligned(workspace, 256)) return fail(DLA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  const size_t need = dla_backward_workspace(p, B, T, H, dk, dv, in_dtype);
+  if (ws_bytes < need) return fail(DLA_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", ws_bytes, need);
+  cudaStream_t st = (cudaStream_t)stream;
+  char* ws = (char*)workspace;
+  int32_t* word = nullptr;
+  cudaError_t e = status_word(st, &word);
+  if (e != cudaSuccess) return cuda_fail(e, "status word");
+  dla::BackwardArgs ba;
+  memset(&ba, 0, sizeof(ba));
+  ba.q = q; ba.k = k; ba.v = v; ba.lam = lam; ba.g = grad_o;
+  ba.boundary = boundary; ba.merge_log = merge_log;
+  ba.dq = grad_q; ba.dk = grad_k; ba.dv = grad_v; ba.dlam = grad_lam;
+  ba.B = B; ba.T = T; ba.H = H; ba.C = p->capacity;
+  ba.status = (int32_t*)ws;
+  ba.evt = (int32_t*)(ws + 256);
+  ba.firsts = ba.evt + (size_t)B * H * T;
+  if ((e = cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), st)) != cudaSuccess) return cuda_fail(e, "status reset");
+  if ((e = timed(DLA_K_BACKWARD, st, [&] { return dla::launch_backward_slots(ba, st); })) != cudaSuccess)
+    return cuda_fail(e, "backward slot lists launch");
+  if ((e = timed(DLA_K_BACKWARD, st, [&] { return dla::launch_backward_dkv(ba, dk, st); })) != cudaSuccess)
+    return cuda_fail(e, "backward dK, dV launch");
+  if ((e = timed(DLA_K_BACKWARD, st, [&] { return dla::launch_backward_dq(ba, dk, st); })) != cudaSuccess)
+    return cuda_fail(e, "backward dQ launch");
+  e = timed(DLA_K_STATUS, st, [&] {
+    status_fold_kernel<<<1, 1, 0, st>>>((const int32_t*)ws, word);
+    return cudaGetLastError();
+  });
+  if (e != cudaSuccess) return cuda_fail(e, "status fold launch");
+  return ok();
+}
+
 }  // extern "C"

@@ -174,6 +174,33 @@ struct DecodeArgs {
   int32_t* status;       // device status word of the call's stream (6 when the cache is inconsistent)
 };
 
+// K4: gradients of the read-out with the forward pass's decisions held fixed
+// (dla_backward.cu).  bf16 q, k, v [B, T, H, d]; fp32 g = dL/do and gradients.
+struct BackwardArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const float* lam;          // [B, T, H, C] or nullptr (ones)
+  const float* g;            // [B, T, H, d]
+  const uint8_t* boundary;   // [B, H, T] of the forward pass
+  const int32_t* merge_log;  // [B, H, T]
+  float* dq;
+  float* dk;
+  float* dv;
+  float* dlam;               // [B, T, H, C] or nullptr
+  int B, T, H, C;
+  int32_t* evt;              // workspace: [B*H][T] boundary events at or before each token
+  int32_t* firsts;           // workspace: [B*H][T + 1][kMaxC] first tokens of the live states after each event
+  int32_t* status;           // device status word (6: an inconsistent trace)
+};
+// The three kernels of K4, in this order on one stream: the slot lists, then
+// dK and dV, then dQ and dlambda.
+cudaError_t launch_backward_slots(const BackwardArgs& a, cudaStream_t s);
+cudaError_t launch_backward_dkv(const BackwardArgs& a, int d, cudaStream_t s);
+cudaError_t launch_backward_dq(const BackwardArgs& a, int d, cudaStream_t s);
+// Workspace bytes of the slot lists of launch_backward.
+size_t backward_slot_bytes(int BH, int T);
+
 // Per-row lengths and first token rows of a packed batch from its cumulative
 // offsets cu[0..B] (device int32): lens[b] = cu[b+1] - cu[b] and start[b] = cu[b],
 // checked (0 <= cu[b] <= cu[b+1] <= total, length <= T); a row that fails the

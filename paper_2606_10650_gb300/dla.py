@@ -22,8 +22,9 @@ STATUS = {0: "DLA_OK", 1: "DLA_ERR_INVALID_ARG", 2: "DLA_ERR_UNSUPPORTED", 3: "D
 EXPORTED = ["dla_default_params", "dla_cache_bytes", "dla_cache_carve", "dla_init_cache",
             "dla_forward_workspace", "dla_forward_min_workspace", "dla_forward", "dla_decode_step",
             "dla_last_error", "dla_status_string", "dla_version", "dla_timing_enable", "dla_timing_read", "dla_forward_noalloc",
-            "dla_forward_host_workspace", "dla_forward_host", "dla_sync_status", "dla_forward_varlen"]
-KERNELS = ["scan", "readout", "decode", "init", "gram", "gate", "status"]
+            "dla_forward_host_workspace", "dla_forward_host", "dla_sync_status", "dla_forward_varlen",
+            "dla_backward_workspace", "dla_backward"]
+KERNELS = ["scan", "readout", "decode", "init", "gram", "gate", "status", "backward"]
 
 
 class DLAError(RuntimeError):
@@ -77,6 +78,9 @@ def lib():
         L.dla_forward_host_workspace.argtypes = [P, ci, ci, ci, ci, ci, ci, ci]
         L.dla_forward_host.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp, vp, vp, sz, vp]
         L.dla_sync_status.argtypes = [vp]
+        L.dla_backward_workspace.restype = sz
+        L.dla_backward_workspace.argtypes = [P, ci, ci, ci, ci, ci, ci]
+        L.dla_backward.argtypes = [P, ci, ci, ci, ci, ci, ci, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.dla_forward_varlen.argtypes = [P, ci, ci, ci, ctypes.c_longlong, vp, ci, ci, ci, vp, vp, vp, vp, vp, Cp, vp,
                                          vp, vp, sz, vp]
         L.dla_timing_enable.argtypes = [ci]
@@ -270,6 +274,43 @@ def dla_forward_varlen(params, cu_seqlens, max_seqlen, q, k, v, lam=None, o=None
                                   _ptr(merge_log), ctypes.c_void_p(base), nb, _stream(stream))
     _check(st)
     return workspace
+
+
+def dla_backward(params, q, k, v, lam, boundary, merge_log, grad_o, grad_q, grad_k, grad_v, grad_lam=None,
+                 workspace=None, stream=None):
+    """Raw call of dla_backward: q, k, v [B, T, H, d] bf16; lam [B, T, H, C] fp32
+    or None; boundary [B, H, T] uint8 and merge_log [B, H, T] int32 from the
+    forward call; grad_o and the outputs grad_q, grad_k, grad_v [B, T, H, d]
+    fp32; grad_lam [B, T, H, C] fp32 or None (all contiguous CUDA tensors)."""
+    B, T, H, d = k.shape
+    dt = _dtype_code(k)
+    for t in (q, k, v, lam, boundary, merge_log, grad_o, grad_q, grad_k, grad_v, grad_lam):
+        if t is not None and not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+    if workspace is None:
+        nb = lib().dla_backward_workspace(ctypes.byref(params), B, T, H, d, d, dt)
+        if nb == 0:
+            raise DLAError(1, "dla_backward_workspace: unsupported arguments")
+        buf, base = _aligned_workspace(nb, k.device)
+        workspace = (buf, base, nb)
+    _, base, nb = workspace
+    st = lib().dla_backward(ctypes.byref(params), dt, B, T, H, d, d, _ptr(q), _ptr(k), _ptr(v), _ptr(lam),
+                            _ptr(boundary), _ptr(merge_log), _ptr(grad_o), _ptr(grad_q), _ptr(grad_k), _ptr(grad_v),
+                            _ptr(grad_lam), ctypes.c_void_p(base), nb, _stream(stream))
+    _check(st)
+    return workspace
+
+
+def backward(q, k, v, lam, boundary, merge_log, grad_o, *, capacity, want_lam=True, stream=None):
+    """Convenience gradients of the read-out (decisions of the forward call held
+    fixed): allocates the outputs with torch.  Returns dict(dq, dk, dv, dlam)."""
+    B, T, H, d = k.shape
+    dev = k.device
+    p = make_params(0.0, capacity)
+    dq, dk, dv = (torch.empty((B, T, H, d), dtype=torch.float32, device=dev) for _ in range(3))
+    dlam = torch.empty((B, T, H, capacity), dtype=torch.float32, device=dev) if want_lam else None
+    dla_backward(p, q, k, v, lam, boundary, merge_log, grad_o, dq, dk, dv, dlam, stream=stream)
+    return dict(dq=dq, dk=dk, dv=dv, dlam=dlam)
 
 
 def dla_forward_noalloc(params, q, k, v, lam=None, o=None, cache=None, boundary=None, merge_log=None, stream=None):

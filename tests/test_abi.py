@@ -35,7 +35,7 @@ def test_library_exports_every_declared_symbol(L):
     for n in _declared():
         assert hasattr(L, n), n
     assert set(_declared()) == set(dla.EXPORTED)
-    assert L.dla_version() == 3
+    assert L.dla_version() == 4
 
 
 def _fake(addr=1 << 20):
@@ -125,6 +125,25 @@ def test_packed_batch_argument_errors(L):
     assert fv(q=r) == 1                             # lengths come from the offsets only
     assert b"seq_lens" in L.dla_last_error()
     assert fv(ws_bytes=1024) == 3
+
+
+def test_backward_argument_errors(L):
+    p = dla.make_params(0.6, 8)
+    nb = L.dla_backward_workspace(ctypes.byref(p), 1, 64, 2, 128, 128, dla.DLA_BF16)
+    assert nb >= 256 + 2 * 64 * 4 + 2 * 65 * 64 * 4
+    assert L.dla_backward_workspace(ctypes.byref(p), 1, 64, 2, 128, 128, dla.DLA_F32) == 0
+
+    def fb(q=p, dt=dla.DLA_BF16, d=128, k=True, ws_bytes=1 << 30, go=True):
+        f = _fake
+        return L.dla_backward(ctypes.byref(q), dt, 1, 64, 2, d, d, f(), f() if k else None, f(), None, f(), f(),
+                              f() if go else None, f(), f(), f(), None, f(1 << 24), ws_bytes, None)
+    assert fb(dt=dla.DLA_F32) == 2
+    assert fb(d=96) == 2
+    assert fb(k=False) == 1
+    assert fb(go=False) == 1
+    assert fb(ws_bytes=1024) == 3
+    assert fb(q=dla.make_params(0.6, 8, from_cache=1)) == 2
+    assert b"from_cache" in L.dla_last_error()
 
 
 def test_kernel_kinds_match_the_header():
