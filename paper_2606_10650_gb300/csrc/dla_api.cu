@@ -55,8 +55,8 @@ CacheLayout cache_layout(int B, int H, int C, int dk, int dv) {
 }
 
 // The read-out kernel of a configuration: bf16 inputs with d = 128 run on the
-// tensor cores (128-token intervals, bf16 hi/lo snapshots); everything else on
-// CUDA cores (64-token intervals, fp32 snapshots).
+// tensor cores (128-token intervals, fp16 snapshots with a power-of-two scale
+// per entry); everything else on CUDA cores (64-token intervals, fp32 snapshots).
 bool use_tc(dla_dtype in_dtype, int d) { return in_dtype == DLA_BF16 && d == 128; }
 int readout_interval(dla_dtype in_dtype, int d) {
   return use_tc(in_dtype, d) ? dla::kReadoutTcInterval : dla::kReadoutSimtInterval;
@@ -79,17 +79,18 @@ struct FwdPlan {
   int persistent;
   int nbuf;          // pools (1 persistent, 2 reset with several rounds)
   int pool_cap;      // pool entries per stream, per pool
-  size_t off_status, off_rows, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_gram,
-      off_progress, off_pool, pool_bytes;
+  size_t off_status, off_rows, off_bnd, off_mlog, off_cache, off_lists_m0, off_lists_ids, off_pstate, off_nbound,
+      off_gram, off_progress, off_pool, pool_bytes, pool_scale_off;
   int gram_chunks;   // chunks of the Gram pre-pass output (0: the scan forms its Gram entries itself)
   size_t total;
 };
 
-// Bytes per snapshot element: fp32 (CUDA-core read-out) or bf16 hi + lo
-// (tensor-core read-out).  A single bf16 rounding of the states (2^-9
-// relative) already reaches the 2e-2 output tolerance on coherent (regime)
-// streams, hence the hi/lo pair.
-size_t pool_elt(dla_dtype /*in_dtype*/) { return 4; }
+// Bytes per snapshot element: fp32 (CUDA-core read-out) or fp16 (tensor-core
+// read-out: S / s in fp16 with s a power of two per entry, kept beside the
+// entries).  A single bf16 rounding of the states (2^-9 relative) already
+// reaches the 2e-2 output tolerance on coherent (regime) streams; fp16 keeps
+// 2^-12, eight times less.
+size_t pool_elt(dla_dtype in_dtype, int d) { return use_tc(in_dtype, d) ? 2 : 4; }
 
 FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int H, int d, dla_dtype in_dtype,
                  bool with_output, bool need_trace, bool need_cache) {
@@ -122,6 +123,8 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   P.off_lists_m0 = off;  if (with_output) off = align256(off + BH * P.nsnap_total * sizeof(int32_t));
   P.off_lists_ids = off; if (with_output) off = align256(off + BH * P.nsnap_total * C * sizeof(int32_t));
   P.off_pstate = off;    if (with_output) off = align256(off + (BH + BH * C) * sizeof(int32_t));
+  // norm bounds of the live entries between rounds (tensor-core read-out: the scale of a snapshot)
+  P.off_nbound = off;    if (with_output) off = align256(off + BH * C * sizeof(float));
   // Gram pre-pass output (bf16 inputs, calls with a read-out): kGramStride floats per 64-token chunk
   P.gram_chunks = (with_output && in_dtype == DLA_BF16) ? (T + dla::kScanL - 1) / dla::kScanL : 0;
   P.off_gram = off;      off = align256(off + BH * (size_t)P.gram_chunks * dla::kGramStride * 4);
@@ -130,7 +133,10 @@ FwdPlan plan_for(int R, bool persistent, const dla_params* p, int B, int T, int 
   // chunk counters (a pre-pass running beside the scan)
   P.off_progress = off;
   if (with_output) off = align256(off + (2 * BH + 2 + kOutPieces + BH * dla::kMaxGramBlk) * sizeof(int32_t));
-  P.pool_bytes = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype)) : 0;
+  // a pool: its entries, then (tensor-core read-out) one scale per entry
+  P.pool_scale_off = with_output ? align256(BH * (size_t)P.pool_cap * d * d * pool_elt(in_dtype, d)) : 0;
+  P.pool_bytes = P.pool_scale_off +
+                 ((with_output && use_tc(in_dtype, d)) ? align256(BH * (size_t)P.pool_cap * sizeof(float)) : 0);
   P.off_pool = off;      off += (size_t)P.nbuf * P.pool_bytes;
   P.total = off;
   return P;
@@ -779,6 +785,13 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   ra.snap_m0 = sa.snap_m0;
   ra.snap_ids = sa.snap_ids;
   sa.pstate = P.persistent ? (int32_t*)(ws + P.off_pstate) : nullptr;
+  sa.nbound = (float*)(ws + P.off_nbound);
+  if (tc && p->from_cache) {  // the continued cache's norm bounds, for the scales of its snapshots
+    e = timed(DLA_K_INIT, st, [&] {
+      return dla::launch_cache_bounds(live.states, live.slot, live.m, B * H, C, d, sa.nbound, st);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "cache bounds launch");
+  }
   sa.gram = P.gram_chunks ? (const float*)(ws + P.off_gram) : nullptr;
   sa.gram_chunks = P.gram_chunks;
   // The scan: the mma.sync scan (CTA pairs, the open state in registers) by
@@ -819,12 +832,14 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     }
     sa.pool = ws + P.off_pool;
+    sa.pool_scale = (float*)((char*)sa.pool + P.pool_scale_off);
     sa.t_begin = 0; sa.t_end = T;
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
     sa.carry_in = 0; sa.snap_at_end = 0;
     e = timed(DLA_K_SCAN, S->hi, [&] { return launch_main_scan(S->hi); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     ra.pool = sa.pool;
+    ra.pool_scale = sa.pool_scale;
     ra.t_begin = 0; ra.t_end = T;
     ra.nsnap = P.nsnap_total; ra.snap_base = 0;
     e = timed(DLA_K_READOUT, S->hi, [&] { return dla::launch_readout_tc(ra, status, S->hi); });
@@ -885,6 +900,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     if ((e = cudaEventRecord(S->prep_done, S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
     if ((e = cudaStreamWaitEvent(S->lo, S->prep_done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
     sa.pool = ws + P.off_pool;
+    sa.pool_scale = (float*)((char*)sa.pool + P.pool_scale_off);
     sa.t_begin = 0; sa.t_end = T;
     sa.nsnap = P.nsnap_total; sa.snap_base = 0;
     sa.carry_in = 0; sa.snap_at_end = 0;
@@ -927,6 +943,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
       if (e != cudaSuccess) return cuda_fail(e, "gram launch");
     }
     ra.pool = sa.pool;
+    ra.pool_scale = sa.pool_scale;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
     // the read-out follows the pre-pass on the read-out stream: one launch over
     // the whole sequence, its CTAs dispatched interval pair by interval pair
@@ -1014,7 +1031,9 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     const int t1 = std::min(T, t0 + sizes[r] * P.interval);
     const int bsel = P.persistent ? 0 : (r % 2) % P.nbuf;
     sa.pool = ws + P.off_pool + (size_t)bsel * P.pool_bytes;
+    sa.pool_scale = (float*)((char*)sa.pool + P.pool_scale_off);
     ra.pool = sa.pool;
+    ra.pool_scale = sa.pool_scale;
     sa.t_begin = t0; sa.t_end = t1;
     sa.nsnap = (t1 - t0 + P.interval - 1) / P.interval;
     sa.snap_base = ra.snap_base = snap0;

@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -86,6 +87,21 @@ __device__ __forceinline__ void st_release_gpu(int32_t* p, int v) {
 __device__ __forceinline__ int row_t_end(const int32_t* seq_lens, int b, int t_begin, int t_end) {
   if (!seq_lens) return t_end;
   return max(t_begin, min(t_end, __ldg(seq_lens + b)));
+}
+// fp16 pool entries: an entry holds S / s in fp16, s a power of two chosen from
+// an upper bound of |S|_F (f16_scale), so that no element exceeds 2^13 (eight
+// times below the fp16 range) and every element keeps fp16's 2^-12 relative
+// rounding.  The bounds come from the triangle inequality over exact norms, so
+// the range needs no check per element.
+__device__ __forceinline__ float f16_scale(float bound) {
+  if (!(bound > 0.f) || !isfinite(bound)) return 1.f;  // an infinite state is caught by the range check
+  int ex;
+  frexpf(bound, &ex);               // bound < 2^ex
+  return ldexpf(1.f, ex - 13);      // bound / s < 2^13
+}
+__device__ __forceinline__ uint2 f16x4(float4 x, float inv) {
+  const __half2 a = __floats2half2_rn(x.x * inv, x.y * inv), b = __floats2half2_rn(x.z * inv, x.w * inv);
+  return make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&b));
 }
 // Token row of the first token of batch row b: b * T in the padded layout, or
 // row_start[b] in the packed one.

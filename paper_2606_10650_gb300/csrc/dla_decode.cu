@@ -321,6 +321,39 @@ cudaError_t launch_init_cache(int32_t* slot, int32_t* n, double* ibar, int32_t* 
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- cache norm bounds
+__global__ void __launch_bounds__(256) cache_bounds_kernel(const float* states, const int32_t* slot, const int32_t* m,
+                                                           int C, int d, float* out) {
+  const int i = blockIdx.x, bh = blockIdx.y;
+  const int mm = m[bh];
+  if (i >= mm || i >= C) return;
+  int sl = slot[(long long)bh * C + i];
+  if (sl < 0 || sl >= C) sl = i;  // an invalid slot map is reported by the kernels that use it
+  const float* S = states + ((long long)bh * C + sl) * d * d;
+  float acc = 0.f;
+  for (int e = threadIdx.x; e < d * d / 4; e += blockDim.x) {
+    const float4 x = reinterpret_cast<const float4*>(S)[e];
+    acc += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
+  }
+  __shared__ float red[8];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += red[w];
+    out[(long long)bh * C + i] = sqrtf(t) * 1.001f;  // fp32 summation error: a bound, not the norm
+  }
+}
+
+cudaError_t launch_cache_bounds(const float* states, const int32_t* slot, const int32_t* m, int BH, int C, int d,
+                                float* out, cudaStream_t s) {
+  if (BH > 65535) return cudaErrorInvalidConfiguration;
+  cache_bounds_kernel<<<dim3(C, BH), 256, 0, s>>>(states, slot, m, C, d, out);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------- packed rows
 // Row lengths and first token rows of a packed batch from its cumulative
 // offsets (see launch_varlen_rows).

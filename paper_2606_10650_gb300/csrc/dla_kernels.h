@@ -13,8 +13,11 @@ namespace dla {
 constexpr int kMaxC = 64;   // largest supported capacity C
 constexpr int kScanL = 64;  // tokens per scan chunk (K1)
 // Floats per chunk of the Gram pre-pass output: suffix table gs[j][t], its
-// prefix table Q[j][t] and a_t (see GramArgs).
-constexpr int kGramBlock = 2 * kScanL * kScanL + kScanL;
+// prefix table Q[j][t], a_t, and the exclusive prefix sums
+// SA[t] = sum_{u < t} sqrt(a_u) for t = 0 .. 64 (|v_u| |k_u| = sqrt(a_u): the
+// growth of a state's norm bound), padded to a multiple of four (see GramArgs).
+constexpr int kGramSA = 2 * kScanL * kScanL + kScanL;
+constexpr int kGramBlock = kGramSA + kScanL + 4;
 
 // Gram block of the tensor-core scan (K0 with GramArgs::packed = 1), per chunk:
 //   gs[j][t], j <= t <= 64   packed by rows (row j starts at 65 j - j (j - 1) / 2)
@@ -29,6 +32,7 @@ __host__ __device__ constexpr int pack_row(int j) { return 65 * j - j * (j - 1) 
 // Floats between consecutive chunks' blocks in the Gram pre-pass output (either
 // layout).
 constexpr int kGramStride = kGramBlockTc;
+static_assert(kGramStride >= kGramBlock && (kGramBlock * 4) % 16 == 0, "Gram block layout");
 
 // Method parameters of the score / boundary test (Sec. 3.1).
 struct ScoreParams {
@@ -71,6 +75,12 @@ struct ScanArgs {
   int carry_in;          // 1: the pool continues from the previous round (pstate holds its counters)
   int snap_at_end;       // 1: also snapshot at this round's last interval end (for the next round)
   int32_t* pstate;       // [B*H] next free pool entry, then [B*H][C] pool ids of the live entries
+  // fp16 pool (tensor-core read-out): the scale s of each entry (S / s is stored),
+  // [B*H][pool_cap], and upper bounds of the live entries' norms |S|_F, [B*H][C]
+  // (read at a round's start, written at its end; a call continuing from a
+  // cache gets them from launch_cache_bounds first)
+  float* pool_scale;
+  float* nbound;
   const float* gram;     // Gram pre-pass output [B*H][gram_chunks][kGramBlock], or nullptr
   int gram_chunks;       // 64-token chunks of the whole sequence
   // Gram pre-pass running beside the scan (nullptr: it finished before the
@@ -133,6 +143,7 @@ struct ReadoutArgs {
   const uint8_t* boundary;
   const int32_t* merge_log;
   const void* pool;
+  const float* pool_scale;  // fp16 pool: the scale of each entry ([B*H][pool_cap])
   int pool_cap;
   const int32_t* snap_m0;
   const int32_t* snap_ids;
@@ -200,6 +211,12 @@ cudaError_t launch_backward_dkv(const BackwardArgs& a, int d, cudaStream_t s);
 cudaError_t launch_backward_dq(const BackwardArgs& a, int d, cudaStream_t s);
 // Workspace bytes of the slot lists of launch_backward.
 size_t backward_slot_bytes(int BH, int T);
+
+// Norms |S_i|_F of the live states of a cache (logical order, i < m), rounded
+// up, into out[B*H][C]: the norm bounds a forward call that continues from the
+// cache starts with.
+cudaError_t launch_cache_bounds(const float* states, const int32_t* slot, const int32_t* m, int BH, int C, int d,
+                                float* out, cudaStream_t s);
 
 // Per-row lengths and first token rows of a packed batch from its cumulative
 // offsets cu[0..B] (device int32): lens[b] = cu[b+1] - cu[b] and start[b] = cu[b],

@@ -14,15 +14,19 @@
 // snapshot lists share most of their states (only entries that changed get new
 // pool entries), so the CTA loads the union of the two lists once and applies
 // each state to the tokens of both intervals: D_x^A = Q_A S_x^T and
-// D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128), with
-// S_x = S_hi + S_lo, the fp32 snapshot split into bf16 parts by K1 (two MMAs
-// per state and interval keep the state rounding near 2^-17 instead of 2^-9).
-// An interval's MMAs are skipped for a state that is not in its list.  Before
+// D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128) in fp16: K1 stores
+// each snapshot as S_x / s_x in fp16 (s_x a power of two from a bound of
+// |S_x|_F, so that no element overflows and every element keeps 2^-12
+// relative rounding), and Q is converted in place to fp16 with a power-of-two
+// scale per row once the intra part has used it (exact: bf16 values fit fp16's
+// significand); the epilogue multiplies D_x by s_x and the row's inverse scale
+// together with lambda.  An interval's MMAs are skipped for a state that is
+// not in its list.  Before
 // the states, the intra part of each interval: P = Q K^T, Pt = P o W
 // (W_ts = lambda_{t, L_t(e(s))} for s <= t, else 0) written as bf16 over the K
 // tile, O = Pt V with V as loaded (an MN-major operand), which o starts from.
-// Roles: warp 0 issues TMA loads (the two Q, K and V tiles, then the
-// hi and lo parts of each union state through four 32 KB stages), warp 1
+// Roles: warp 0 issues TMA loads (the two Q, K and V tiles, then each union
+// state, 32 KB in fp16, through four 32 KB stages), warp 1
 // issues tcgen05.mma (one thread) into two TMEM buffers of two 128-column
 // accumulators (A, B), warps 2..17 read TMEM, weight by lambda and accumulate o
 // in registers (one token row, one interval and one 64-column half per thread;
@@ -42,7 +46,7 @@ constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
 constexpr int NT = 576;   // 18 warps
 constexpr int NEPI = 16;  // epilogue warps
-constexpr int NHS = 4;   // shared-memory stages (32 KB: a hi or lo state part, a K / Pt tile or a V tile)
+constexpr int NHS = 4;   // shared-memory stages (32 KB: an fp16 state, a K / Pt tile or a V tile)
 constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
 constexpr int MAXU = 2 * kMaxC;  // union of two lists
 constexpr uint32_t kTmemCols = 512;
@@ -69,6 +73,8 @@ struct TcSmem {
   int ids[2][kMaxC];           // pool ids of the two lists
   int uid[MAXU];               // union: pool id
   int uxa[MAXU], uxb[MAXU];    // union: index in list A / list B, or -1
+  float uscale[MAXU];          // union: scale s_x of the fp16 entry (S_x / s_x is stored)
+  float qmax[2][2][L];         // [interval][k-half][row]: max |q| of the half row (Q's fp16 scales)
   int logi[2][kRows];          // table-build scratch, per interval
   int nu;                      // union size
   uint64_t bar_q, bar_pt, bar_done;
@@ -295,6 +301,9 @@ __global__ void __launch_bounds__(NT, 1)
       nb_only += __popc(only);
     }
     if (lane == 0) sm.nu = m0A + nb_only;
+    __syncwarp();
+    const int nu_w = m0A + nb_only;
+    for (int u = lane; u < nu_w; u += 32) sm.uscale[u] = __ldcg(a.pool_scale + (long long)bh * a.pool_cap + sm.uid[u]);
   }
   tc_fence_before();
   __syncthreads();
@@ -302,10 +311,10 @@ __global__ void __launch_bounds__(NT, 1)
   const uint32_t tmem = sm.tmem_base;
   const int nu = sm.nu;
   // Ring units: g = 0, 1 the K tiles of intervals A and B (then Pt over them),
-  // g = 2, 3 their V tiles (the MN-major B operand of O), g = 4 + u the hi / lo part
-  // u & 1 of union state u >> 1.  Unit g uses stage g % NHS for the
-  // (g / NHS)-th time.  Accumulators (TMEM buffer n % NBUF): n = 0 P = Q K^T,
-  // n = 1 O = Pt V, n = 2 + x union state x.
+  // g = 2, 3 their V tiles (the MN-major B operand of O), g = 4 + x union state
+  // x (fp16).  Unit g uses stage g % NHS for the (g / NHS)-th time.
+  // Accumulators (TMEM buffer n % NBUF): n = 0 P = Q K^T, n = 1 O = Pt V,
+  // n = 2 + x union state x.
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -329,11 +338,11 @@ __global__ void __launch_bounds__(NT, 1)
         mbar_arrive(&sm.full[3]);
       }
       for (int i = 0; i < NHS; ++i) issued[i] = 1;
-      for (int u = 0; u < 2 * nu; ++u) {
+      for (int u = 0; u < nu; ++u) {
         const int g = 4 + u, hsi = g % NHS, k = g / NHS;
         if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
-        const int row = (int)((((long long)bh * a.pool_cap + sm.uid[u >> 1]) * 2 + (u & 1)) * D);
+        const int row = (int)(((long long)bh * a.pool_cap + sm.uid[u]) * D);
         tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
         tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
         issued[hsi] = k + 1;
@@ -391,31 +400,30 @@ __global__ void __launch_bounds__(NT, 1)
         mma_commit(&sm.acc_full[1]);
       }
       for (int i = 0; i < NHS; ++i) mma_commit(&sm.empty[i]);  // every stage is free once O is done
+      // the state products, fp16 Q (converted by the epilogue before bar_pt) and fp16 states
+      constexpr uint32_t idesc_h = idesc_f16_f32(L, D);
       for (int x = 0; ok && x < nu; ++x) {
         const int buf = x % NBUF;
         const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
         if (!(ok = acc_acquire(x + 2))) break;
         const uint32_t dA = tmem + 256u * buf, dB = dA + 128u;
-        for (int part = 0; part < 2; ++part) {
-          const int g = 4 + 2 * x + part, hsi = g % NHS;
-          if (!(ok = unit_wait(g))) break;
-          const uint64_t bd = hd0 + (uint64_t)hsi * kStage;
-          if (inA && inB) {
+        const int g = 4 + x, hsi = g % NHS;
+        if (!(ok = unit_wait(g))) break;
+        const uint64_t bd = hd0 + (uint64_t)hsi * kStage;
+        if (inA && inB) {
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              const uint32_t acc = (part | kk) > 0;
-              mma_bf16(dA, qd0 + kstep(kk), bd + kstep(kk), idesc, acc);
-              mma_bf16(dB, qd1 + kstep(kk), bd + kstep(kk), idesc, acc);
-            }
-          } else if (inA || inB) {
-            const uint32_t dd = inA ? dA : dB;
-            const uint64_t qd = inA ? qd0 : qd1;
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) mma_bf16(dd, qd + kstep(kk), bd + kstep(kk), idesc, (part | kk) > 0);
+          for (int kk = 0; kk < 8; ++kk) {
+            mma_bf16(dA, qd0 + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
+            mma_bf16(dB, qd1 + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
           }
-          mma_commit(&sm.empty[hsi]);
+        } else if (inA || inB) {
+          const uint32_t dd = inA ? dA : dB;
+          const uint64_t qd = inA ? qd0 : qd1;
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) mma_bf16(dd, qd + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
         }
-        if (ok) mma_commit(&sm.acc_full[buf]);
+        mma_commit(&sm.empty[hsi]);
+        mma_commit(&sm.acc_full[buf]);
       }
       mma_commit(&sm.bar_done);  // every MMA issued above has completed once this fires
       mbar_wait_drain(&sm.bar_done, 0);
@@ -510,7 +518,52 @@ __global__ void __launch_bounds__(NT, 1)
           }
         }
       }
-      fence_proxy_async();  // the generic-proxy writes (Pt) feed the tensor core
+    }
+    // This row's half of Q into fp16 in place (the P MMAs, the only bf16 use of Q,
+    // are complete): a power-of-two scale per row, agreed on by the two k-halves
+    // through qmax, keeps every element below 2^14 and in fp16's normal range
+    // (bf16 values fit fp16's significand, so only values below 2^-14 of the
+    // row's scale round); the epilogue multiplies D by its inverse, qinv.
+    float qinv = 1.f;
+    {
+      uint8_t* qtile = sm.Q[side][ch];
+      const bool conv = ok && side_in;  // warp-uniform
+      float mx = 0.f;
+      if (conv) {
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          const uint4 w = *reinterpret_cast<const uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4));
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ws[i]));
+            mx = fmaxf(mx, fmaxf(fabsf(f.x), fabsf(f.y)));
+          }
+        }
+      }
+      sm.qmax[side][ch][t] = mx;
+      asm volatile("bar.sync 1, 512;" ::: "memory");
+      if (conv) {
+        const float rm = fmaxf(sm.qmax[side][0][t], sm.qmax[side][1][t]);
+        int ex = 0;
+        if (rm > 0.f) frexpf(rm, &ex);  // rm < 2^ex
+        const float sc = ldexpf(1.f, 14 - ex);
+        qinv = ldexpf(1.f, ex - 14);
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          uint4* ptr = reinterpret_cast<uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4));
+          const uint4 w = *ptr;
+          uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ws[i]));
+            const __half2 hh = __floats2half2_rn(f.x * sc, f.y * sc);
+            ws[i] = *reinterpret_cast<const uint32_t*>(&hh);
+          }
+          *ptr = make_uint4(ws[0], ws[1], ws[2], ws[3]);
+        }
+      }
+      fence_proxy_async();  // the generic-proxy writes (Pt, fp16 Q) feed the tensor core
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -541,12 +594,13 @@ __global__ void __launch_bounds__(NT, 1)
     const int* ux = side ? sm.uxb : sm.uxa;
     {  // snapshot part
       const unsigned char* tab_t = sm.tab[side] + evt_t * kMaxC;
-      // weight of union state x for this token (0 when not in its interval's list)
+      // weight of union state x for this token (0 when not in its interval's list):
+      // lambda times the entry's scale s_x and the row's inverse Q scale
       auto weight = [&](int x) -> float {
         if (x >= nu || t >= Lcs) return 0.f;
         const int xi = ux[x];
         if (xi < 0) return 0.f;
-        return lam_t ? lam_at(tab_t[xi]) : 1.f;
+        return (lam_t ? lam_at(tab_t[xi]) : 1.f) * sm.uscale[x] * qinv;
       };
       float wn = weight(0);
       for (int x = 0; ok && x < nu; ++x) {
@@ -602,13 +656,13 @@ __global__ void __launch_bounds__(NT, 1)
 // ---------------------------------------------------------------- host side
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
   CUtensorMap mq, mk, mv, ms;
-  const long long rows = (long long)a.B * a.H * a.pool_cap * 2 * D;
+  const long long rows = (long long)a.B * a.H * a.pool_cap * D;  // fp16 entries of D rows
   // packed layout: one batch coordinate over all token rows
   const int mb = a.row_start ? 1 : a.B;
   const long long mt = a.row_start ? (a.total_rows > 0 ? a.total_rows : 1) : a.T;
   if (mt >= (1LL << 31)) return cudaErrorInvalidValue;
   if (!tmap_tokens(&mq, a.q, mb, (int)mt, a.H) || !tmap_tokens(&mk, a.k, mb, (int)mt, a.H) ||
-      !tmap_tokens(&mv, a.v, mb, (int)mt, a.H) || !tmap_pool(&ms, a.pool, rows))
+      !tmap_tokens(&mv, a.v, mb, (int)mt, a.H) || !tmap_pool(&ms, a.pool, rows, true))
     return cudaErrorInvalidValue;
   if (a.row_start && !a.seq_lens) return cudaErrorInvalidValue;  // the packed layout needs per-row lengths
   const size_t smem = sizeof(TcSmem) + 1024;

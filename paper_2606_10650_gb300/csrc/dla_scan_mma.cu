@@ -50,11 +50,29 @@ struct MmaSmem {
   int mlog[L];
   int ops[3 * L + 4][4];
   int snap_src[kMaxC][2];
+  float snap_scale[kMaxC];          // scale s of each snapshot job (fp16 pool: S / s is stored)
   int nops, nsnapjobs;
   int pend;                         // snapshot copies waiting for the next chunk's idle warps (bf16 pool)
   int gcnt[kMaxGramBlk];            // Gram pre-pass counters last read (thread 0)
   int m, cur, js, seg_pre, pool_next;
 };
+
+// SA[t] = sum_{u < t} sqrt(a_u), t = 0 .. 64, of a chunk's a values (one warp;
+// lane l takes tokens 2l and 2l + 1), and three zeros of padding.
+__device__ __forceinline__ void norm_prefix_warp(const float* a, float* sa, int lane) {
+  const float s0 = sqrtf(a[2 * lane]), s1 = sqrtf(a[2 * lane + 1]);
+  float inc = s0 + s1;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float u = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += u;
+  }
+  const float ex = inc - s0 - s1;
+  sa[2 * lane] = ex;
+  sa[2 * lane + 1] = ex + s0;
+  if (lane == 31) sa[kScanL] = inc;
+  if (lane < 3) sa[kScanL + 1 + lane] = 0.f;
+}
 
 // Keep the bf16 halves of a packed pair whose token index lies in [u0, u1).
 __device__ __forceinline__ uint32_t mask_pair(uint32_t v, int t, int u0, int u1) {
@@ -340,28 +358,10 @@ __device__ __forceinline__ void copy_state_g(float* dst, const float* src) {
     for (int i = 0; i < 4; ++i) store4(dst + ((base + i) * NT + threadIdx.x) * 4, v[i]);
   }
 }
-template <int D, int NR = D>
-__device__ __forceinline__ void copy_state_g(__nv_bfloat16* dst, const float* src) {
-  constexpr int PER = NR * D / 4 / NT;
-  for (int base = 0; base < PER; base += 4) {
-    float4 v[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) v[i] = load4(src + ((base + i) * NT + threadIdx.x) * 4);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int e = ((base + i) * NT + threadIdx.x) * 4;
-      const float4 x = v[i];
-      const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
-      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-      store4(dst + e, make_float4(f01.x, f01.y, f23.x, f23.y));
-      store4(dst + D * D + e, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
-    }
-  }
-}
-// The same conversion by threads i0, i0 + ni, ... (any count: the deferred
-// snapshot copies run on the warps that idle during the boundary passes).
+// NR rows of an fp32 state into an fp16 pool entry (scaled by inv = 1 / s), by
+// threads i0, i0 + ni, ...
 template <int D, int NR>
-__device__ __forceinline__ void copy_state_split(__nv_bfloat16* dst, const float* src, int i0, int ni) {
+__device__ __forceinline__ void copy_state_f16(__half* dst, const float* src, float inv, int i0, int ni) {
   constexpr int N4 = NR * D / 4;
   for (int base = i0; base < N4; base += 4 * ni) {
     float4 v[4];
@@ -373,13 +373,7 @@ __device__ __forceinline__ void copy_state_split(__nv_bfloat16* dst, const float
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int e4 = base + i * ni;
-      if (e4 < N4) {
-        const float4 x = v[i];
-        const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
-        const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-        store4(dst + e4 * 4, make_float4(f01.x, f01.y, f23.x, f23.y));
-        store4(dst + D * D + e4 * 4, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
-      }
+      if (e4 < N4) *reinterpret_cast<uint2*>(dst + e4 * 4) = f16x4(v[i], inv);
     }
   }
 }
@@ -416,9 +410,6 @@ __device__ __forceinline__ void add_state_g(float* dst, const float* src) {
 __device__ __forceinline__ void put_pair(float* entry, int D, int j, int k, float v0, float v1) {
   *reinterpret_cast<float2*>(entry + j * D + k) = make_float2(v0, v1);
 }
-
-template <typename Tpool>
-constexpr int parts_of() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
 }  // namespace
 
@@ -457,7 +448,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   const int row_stride = a.H * D;
   const int rbase = rank * R;         // first state row of this CTA
   float* states = a.states + (long long)bh * C * D * D;
-  constexpr long long kEntry = (long long)parts_of<Tpool>() * D * D;
+  constexpr long long kEntry = (long long)D * D;
+  constexpr bool kF16 = sizeof(Tpool) == 2;  // fp16 pool entries (tensor-core read-out)
   Tpool* pool = a.pool ? reinterpret_cast<Tpool*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
   uint8_t* bnd_out = a.boundary + (long long)bh * a.T;
   int32_t* mlog_out = a.merge_log + (long long)bh * a.T;
@@ -502,10 +494,12 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   __syncthreads();
   const int m_start = sm.m;
   if (tid == 0) sm.open_slot = (m_start > 0) ? sm.slot[m_start - 1] : 0;  // rewritten by every replay
-  // Warp 0 keeps n, Ibar, physical slot, pool id and "changed since the last
-  // snapshot" of every entry in registers (entry i: lane i % 32, element i / 32).
+  // Warp 0 keeps n, Ibar, physical slot, pool id, "changed since the last
+  // snapshot" and (fp16 pool) an upper bound of |S|_F of every entry in
+  // registers (entry i: lane i % 32, element i / 32).
   int e_n[2] = {0, 0}, e_slot[2] = {0, 0}, e_pid[2] = {-1, -1}, e_dirty[2] = {0, 0};
   double e_ib[2] = {0.0, 0.0};
+  float e_nb[2] = {0.f, 0.f};
   if (warp == 0) {
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
@@ -514,6 +508,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         e_n[r] = a.n[(long long)bh * C + i];
         e_ib[r] = a.ibar[(long long)bh * C + i];
         e_slot[r] = sm.slot[i];
+        if (kF16 && pool && i < m_start) e_nb[r] = a.nbound[(long long)bh * C + i];
       }
     }
   }
@@ -539,8 +534,25 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         for (int r = 0; r < 2; ++r)
           if (lane + 32 * r < m_start) e_pid[r] = a.pstate[a.B * a.H + (long long)bh * C + lane + 32 * r];
     } else {  // snapshot 0: every live entry at the start of the round
-      for (int i = 0; i < m_start && i < a.pool_cap; ++i)
-        copy_state_g<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]));
+      if constexpr (kF16) {
+        if (warp == 0)
+#pragma unroll
+          for (int r = 0; r < 2; ++r) {
+            const int i = lane + 32 * r;
+            if (i < m_start && i < a.pool_cap) {
+              const float sc = f16_scale(e_nb[r]);
+              sm.snap_scale[i] = sc;
+              if (lead) a.pool_scale[(long long)bh * a.pool_cap + i] = sc;
+            }
+          }
+        __syncthreads();
+        for (int i = 0; i < m_start && i < a.pool_cap; ++i)
+          copy_state_f16<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]),
+                               1.f / sm.snap_scale[i], tid, NT);
+      } else {
+        for (int i = 0; i < m_start && i < a.pool_cap; ++i)
+          copy_state_g<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]));
+      }
       if (warp == 0)
 #pragma unroll
         for (int r = 0; r < 2; ++r)
@@ -603,23 +615,36 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
     }
   };
-  // The snapshot copies listed in sm.snap_src[0 .. n): the open state from its
-  // bf16 hi / lo operand in shared memory, closed states from their fp32 slots.
-  // Threads i0, i0 + ni, ...
+  // The snapshot copies listed in sm.snap_src[0 .. n) into fp16 pool entries
+  // (scaled by 1 / sm.snap_scale): the open state from its bf16 hi / lo operand
+  // in shared memory (hi + lo is the fp32 value to 2^-17), closed states from
+  // their fp32 slots.  Threads i0, i0 + ni, ...
   auto snapshot_copies = [&](int n, int i0, int ni) {
     for (int jj = 0; jj < n; ++jj) {
       const int p = sm.snap_src[jj][0], srcslot = sm.snap_src[jj][1];
+      const float inv = 1.f / sm.snap_scale[jj];
       Tpool* entry = pool + (long long)p * kEntry;
-      if constexpr (sizeof(Tpool) == 2) {
-        if (srcslot < 0) {  // coalesced 16-byte copies of the staged hi / lo rows
-          for (int e = i0; e < 2 * R * (D / 8); e += ni) {
-            const int part = e / (R * (D / 8)), rem = e % (R * (D / 8));
-            const int j = rem / (D / 8), k8 = (rem % (D / 8)) * 8;
-            *reinterpret_cast<uint4*>(entry + part * D * D + (rbase + j) * D + k8) =
-                *reinterpret_cast<const uint4*>(&sm.S2[part][j * RP + k8]);
+      if constexpr (kF16) {
+        if (srcslot < 0) {  // 8 elements per 16-byte store, rows in order
+          for (int e = i0; e < R * (D / 8); e += ni) {
+            const int j = e / (D / 8), k8 = (e % (D / 8)) * 8;
+            const uint4 hv = *reinterpret_cast<const uint4*>(&sm.S2[0][j * RP + k8]);
+            const uint4 lv = *reinterpret_cast<const uint4*>(&sm.S2[1][j * RP + k8]);
+            const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w}, lw[4] = {lv.x, lv.y, lv.z, lv.w};
+            float f[8];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float2 h2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&hw[i]));
+              const float2 l2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&lw[i]));
+              f[2 * i] = h2.x + l2.x;
+              f[2 * i + 1] = h2.y + l2.y;
+            }
+            const uint2 a0 = f16x4(make_float4(f[0], f[1], f[2], f[3]), inv);
+            const uint2 a1 = f16x4(make_float4(f[4], f[5], f[6], f[7]), inv);
+            *reinterpret_cast<uint4*>(entry + (rbase + j) * D + k8) = make_uint4(a0.x, a0.y, a1.x, a1.y);
           }
         } else {
-          copy_state_split<D, R>(entry + (long long)rbase * D, srows(srcslot), i0, ni);
+          copy_state_f16<D, R>(entry + (long long)rbase * D, srows(srcslot), inv, i0, ni);
         }
       }
     }
@@ -750,6 +775,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       }
       __syncthreads();
       prefix_rows(sm.gq[st], GS, 1, sm.gq[st] + L * L, GS);
+      if (warp == 0) norm_prefix_warp(sm.gq[st] + 2 * L * L, sm.gq[st] + kGramSA, lane);
     }
     __syncthreads();
     if (tid < L) {  // this CTA's part of x_t
@@ -806,6 +832,8 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const float* gst = sm.gq[st];
       const float* qst = gst + L * L;
       const float aa = gst[2 * L * L + ta], ab = gst[2 * L * L + tb];
+      // fp16 pool: the open entry's norm bound restarts from its exact norm
+      if (kF16 && m_chunk > 0) entry_set(e_nb, m_chunk - 1, sqrtf(fmaxf(gam_open, 0.f)));
       // exclusive prefix sums of x_t and a_t over the chunk: with the table Q,
       // sum_{js <= u < t} (2 beta_u + a_u) = 2 (X(t) - X(js)) [open state] + 2 Q[js][t] + A(t) - A(js)
       float xpa, xpb, apa, apb;
@@ -867,6 +895,9 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         const float v = ((ta >= u0 && ta < u1) ? Ia : 0.f) + ((tb >= u0 && tb < u1) ? Ib : 0.f);
         return warp_sum(v);
       };
+      // fp16 pool: a run [u0, u1) grows its entry's norm bound by SA(u1) - SA(u0)
+      // (the chunk's prefix sums of |v_t| |k_t| = sqrt(a_t), in its Gram block)
+      const float* sa_blk = gst + kGramSA;
       int m = m_chunk;
       int seg_u0 = 0, nops = 0, run0 = 0;
       unsigned long long pend = bmask;
@@ -875,12 +906,15 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         pend &= pend - 1;
         if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
           const double part = (double)run_sum(run0, t);
+          // |S + sum v k^T|_F <= |S|_F + sum |v| |k|, and |v_t| |k_t| = sqrt(a_t)
+          float grow = 0.f;
+          if constexpr (kF16) grow = sa_blk[t] - sa_blk[run0];
           const int e = m - 1;
           if ((e & 31) == lane) {
             if (e < 32) {
-              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1;
+              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1; e_nb[0] += grow;
             } else {
-              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1;
+              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1; e_nb[1] += grow;
             }
           }
         }
@@ -901,8 +935,10 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           // pair densities (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}): fp64 sums, compared in fp32
           int nn[2], ns[2], np_[2], nd[2];
           double nb[2];
+          float nnb[2];
           entry_next(e_n, nn);
           entry_next(e_ib, nb);
+          entry_next(e_nb, nnb);
           entry_next(e_slot, ns);
           entry_next(e_pid, np_);
           entry_next(e_dirty, nd);
@@ -942,15 +978,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           for (int r = 0; r < 2; ++r) {
             const int i = lane + 32 * r;
             if (i == j) {
-              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1;
+              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1; e_nb[r] += nnb[r];
             } else if (i > j && i < m - 1) {
               e_n[r] = nn[r]; e_ib[r] = nb[r]; e_slot[r] = ns[r]; e_pid[r] = np_[r]; e_dirty[r] = nd[r];
+              e_nb[r] = nnb[r];
             }
           }
           phys_new = srcs;
           m -= 1;
         }
         const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
+        if constexpr (kF16) entry_set(e_nb, m, sa_blk[t + 1] - sa_blk[t]);
         entry_set(e_slot, m, phys_new);
         entry_set(e_n, m, 1);
         entry_set(e_ib, m, (double)it);
@@ -1022,6 +1060,11 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
             e_dirty[r] = 0;
             sm.snap_src[rank_][0] = p;
             sm.snap_src[rank_][1] = (i == m - 1) ? -1 : e_slot[r];
+            if constexpr (kF16) {
+              const float sc = f16_scale(e_nb[r]);
+              sm.snap_scale[rank_] = sc;
+              if (lead) a.pool_scale[(long long)bh * a.pool_cap + p] = sc;
+            }
           }
           nj += __popc(bal);
           if (lead && i < m) a.snap_ids[lrow * C + i] = e_pid[r];
@@ -1096,6 +1139,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
           a.ibar[(long long)bh * C + i] = (i < m) ? e_ib[r] : 0.0;
         }
         if (pool && a.pstate && i < m) a.pstate[a.B * a.H + (long long)bh * C + i] = e_pid[r];
+        if (kF16 && pool && i < m) a.nbound[(long long)bh * C + i] = e_nb[r];
       }
       if (lane == 0) {
         a.m[bh] = m;
@@ -1187,6 +1231,7 @@ __global__ void __launch_bounds__(NT) gram_kernel(GramArgs a) {
     }
     if (threadIdx.x < L / 4)
       *reinterpret_cast<float4*>(out + 2 * L * L + 4 * threadIdx.x) = *reinterpret_cast<const float4*>(sm.a + 4 * threadIdx.x);
+    if (threadIdx.x >= NT - 32) norm_prefix_warp(sm.a, out + kGramSA, threadIdx.x & 31);
     // published after the first chunk, then every fourth and after the last
     // (the scan reads the blocks by bulk copy: async proxy)
     const bool publish = a.ready && (i < 4 || (i & 3) == 3 || i + 1 == n_mine);
@@ -1402,7 +1447,7 @@ static int resident_streams_query(int BH, int d) {
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return 0;
   if (scan_mma_ctas_per_stream(BH, d) == 2) {
-    auto kern = scan_mma_kernel<128, __nv_bfloat16, 2>;
+    auto kern = scan_mma_kernel<128, __half, 2>;
     const size_t smem = sizeof(MmaSmem<128, 2>);
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) return 0;
     cudaLaunchConfig_t cfg = {};
@@ -1421,13 +1466,13 @@ static int resident_streams_query(int BH, int d) {
     return clusters;
   }
   if (d == 128) {
-    auto kern = scan_mma_kernel<128, __nv_bfloat16, 1>;
+    auto kern = scan_mma_kernel<128, __half, 1>;
     const size_t smem = sizeof(MmaSmem<128, 1>);
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, smem) != cudaSuccess)
       return 0;
   } else {
-    auto kern = scan_mma_kernel<64, __nv_bfloat16, 1>;
+    auto kern = scan_mma_kernel<64, __half, 1>;
     const size_t smem = sizeof(MmaSmem<64, 1>);
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess ||
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NT, smem) != cudaSuccess)
@@ -1470,10 +1515,10 @@ __global__ void gate_kernel(const int32_t* started, int n, int32_t* status) {
 cudaError_t preload_scan_kernels() {
   cudaFuncAttributes fa;
   cudaError_t e;
-  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 2, true>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __nv_bfloat16, 1, true>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 2>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 1>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 2, true>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 1, true>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_kernel<128>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_tc_kernel<128>)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, gate_kernel);
@@ -1486,10 +1531,10 @@ cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStre
 cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s) {
   if (d == 128) {
     if (use_pairs(a))
-      return pool_bf16 ? launch_scan_mma_t<128, __nv_bfloat16, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);
-    return pool_bf16 ? launch_scan_mma_t<128, __nv_bfloat16, 1>(a, s) : launch_scan_mma_t<128, float, 1>(a, s);
+      return pool_bf16 ? launch_scan_mma_t<128, __half, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);
+    return pool_bf16 ? launch_scan_mma_t<128, __half, 1>(a, s) : launch_scan_mma_t<128, float, 1>(a, s);
   }
-  return pool_bf16 ? launch_scan_mma_t<64, __nv_bfloat16, 1>(a, s) : launch_scan_mma_t<64, float, 1>(a, s);
+  return pool_bf16 ? launch_scan_mma_t<64, __half, 1>(a, s) : launch_scan_mma_t<64, float, 1>(a, s);
 }
 
 }  // namespace dla

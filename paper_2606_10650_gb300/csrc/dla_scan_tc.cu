@@ -71,6 +71,7 @@ struct DecBuf {         // decisions of one chunk (warp 0 -> state warps)
 };
 struct SnapBuf {        // snapshot jobs of one interval end
   int src[kMaxC][2];    // pool id, source physical slot (-1: the open entry)
+  float scale[kMaxC];   // scale s of each job's fp16 entry (S / s is stored)
   int ids[kMaxC];
   int njobs, m;
 };
@@ -86,6 +87,7 @@ struct TcScanSmem {
   float red[4][L];
   float gred[4];
   int slot0[kMaxC];
+  float scale0[kMaxC];             // scales of the round's first snapshot (every live entry)
   int gcnt[kMaxGramBlk];
   int cmd[2][8];                   // MMA commands: kind, stage, region, acc, source of each K step
   uint64_t kv_full[NKV], kv_empty[NKV], tab_full[2], tab_empty[2], dec_full[2], y_full[2], cmd_full[2],
@@ -165,8 +167,8 @@ __global__ void __launch_bounds__(NT, 1)
   const int ntok = a.t_end - a.t_begin;
   const int nchunks = (ntok + L - 1) / L;
   float* states = a.states + (long long)bh * C * D * D;
-  constexpr long long kEntry = 2LL * D * D;  // a pool entry: bf16 hi rows, then lo rows
-  __nv_bfloat16* pool = a.pool ? reinterpret_cast<__nv_bfloat16*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
+  constexpr long long kEntry = (long long)D * D;  // a pool entry: S / s in fp16, D rows
+  __half* pool = a.pool ? reinterpret_cast<__half*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
   uint8_t* bnd_out = a.boundary + (long long)bh * a.T;
   int32_t* mlog_out = a.merge_log + (long long)bh * a.T;
   volatile int* abort = &sm.abort_flag;
@@ -205,6 +207,8 @@ __global__ void __launch_bounds__(NT, 1)
       sl = i;
     }
     sm.slot0[i] = sl;
+    // a round that restarts its pool copies every live entry first
+    if (a.pool && !a.carry_in) sm.scale0[i] = f16_scale(a.nbound[(long long)bh * C + i]);
   }
   if (warp == W_MMA) tmem_alloc(&sm.tmem_base, kTmemCols);
   tc_fence_before();
@@ -218,6 +222,7 @@ __global__ void __launch_bounds__(NT, 1)
     const float Df = (float)(D * D), invDf = 1.f / Df;
     int e_n[2] = {0, 0}, e_slot[2] = {0, 0}, e_pid[2] = {-1, -1}, e_dirty[2] = {0, 0};
     double e_ib[2] = {0.0, 0.0};
+    float e_nb[2] = {0.f, 0.f};  // upper bounds of |S|_F (the scales of the fp16 snapshots)
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int i = lane + 32 * r;
@@ -225,6 +230,7 @@ __global__ void __launch_bounds__(NT, 1)
         e_n[r] = a.n[(long long)bh * C + i];
         e_ib[r] = a.ibar[(long long)bh * C + i];
         e_slot[r] = sm.slot0[i];
+        if (pool && i < m_start) e_nb[r] = a.nbound[(long long)bh * C + i];
       }
     }
     int pool_next = 0;
@@ -236,8 +242,13 @@ __global__ void __launch_bounds__(NT, 1)
           if (lane + 32 * r < m_start) e_pid[r] = a.pstate[a.B * a.H + (long long)bh * C + lane + 32 * r];
       } else {
 #pragma unroll
-        for (int r = 0; r < 2; ++r)
-          if (lane + 32 * r < m_start) e_pid[r] = lane + 32 * r;
+        for (int r = 0; r < 2; ++r) {
+          const int i = lane + 32 * r;
+          if (i < m_start) {
+            e_pid[r] = i;
+            a.pool_scale[(long long)bh * a.pool_cap + i] = sm.scale0[i];
+          }
+        }
         pool_next = m_start;
       }
     }
@@ -279,6 +290,7 @@ __global__ void __launch_bounds__(NT, 1)
       if (ta >= Lc) xa = 0.f;
       if (tb >= Lc) xb = 0.f;
       const float aa = (ta < Lc) ? av[ta] : 0.f, ab = (tb < Lc) ? av[tb] : 0.f;
+      if (m_chunk > 0) entry_set(e_nb, m_chunk - 1, sqrtf(fmaxf(gam_open, 0.f)));
       // exclusive prefix sums X, A of x and a over the chunk
       float xpa, xpb, apa, apb, xtot, atot;
       {
@@ -353,12 +365,15 @@ __global__ void __launch_bounds__(NT, 1)
         pend &= pend - 1;
         if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
           const double part = (double)run_sum(run0, t);
+          // |S + sum v k^T|_F <= |S|_F + sum |v| |k|, and |v_t| |k_t| = sqrt(a_t)
+          const float grow =
+              warp_sum(((ta >= run0 && ta < t) ? sqrtf(aa) : 0.f) + ((tb >= run0 && tb < t) ? sqrtf(ab) : 0.f));
           const int e = m - 1;
           if ((e & 31) == lane) {
             if (e < 32) {
-              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1;
+              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1; e_nb[0] += grow;
             } else {
-              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1;
+              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1; e_nb[1] += grow;
             }
           }
         }
@@ -379,8 +394,10 @@ __global__ void __launch_bounds__(NT, 1)
           // pair densities (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}): fp64 sums, compared in fp32
           int nn[2], ns[2], np_[2], nd[2];
           double nb[2];
+          float nnb[2];
           entry_next(e_n, nn);
           entry_next(e_ib, nb);
+          entry_next(e_nb, nnb);
           entry_next(e_slot, ns);
           entry_next(e_pid, np_);
           entry_next(e_dirty, nd);
@@ -419,15 +436,17 @@ __global__ void __launch_bounds__(NT, 1)
           for (int r = 0; r < 2; ++r) {
             const int i = lane + 32 * r;
             if (i == j) {
-              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1;
+              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1; e_nb[r] += nnb[r];
             } else if (i > j && i < m - 1) {
               e_n[r] = nn[r]; e_ib[r] = nb[r]; e_slot[r] = ns[r]; e_pid[r] = np_[r]; e_dirty[r] = nd[r];
+              e_nb[r] = nnb[r];
             }
           }
           phys_new = srcs;
           m -= 1;
         }
         const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
+        entry_set(e_nb, m, sqrtf(__shfl_sync(0xffffffffu, (t & 1) ? ab : aa, t >> 1)));
         entry_set(e_slot, m, phys_new);
         entry_set(e_n, m, 1);
         entry_set(e_ib, m, (double)it);
@@ -473,6 +492,9 @@ __global__ void __launch_bounds__(NT, 1)
             e_dirty[r] = 0;
             sb.src[rank_][0] = p;
             sb.src[rank_][1] = (i == m - 1) ? -1 : e_slot[r];
+            const float sc = f16_scale(e_nb[r]);
+            sb.scale[rank_] = sc;
+            a.pool_scale[(long long)bh * a.pool_cap + p] = sc;
           }
           nj += __popc(bal);
           if (i < m) sb.ids[i] = e_pid[r];
@@ -507,6 +529,7 @@ __global__ void __launch_bounds__(NT, 1)
         a.ibar[(long long)bh * C + i] = (i < m) ? e_ib[r] : 0.0;
       }
       if (pool && a.pstate && i < m) a.pstate[a.B * a.H + (long long)bh * C + i] = e_pid[r];
+      if (pool && i < m) a.nbound[(long long)bh * C + i] = e_nb[r];
     }
     if (lane == 0) {
       a.m[bh] = m;
@@ -788,8 +811,8 @@ __global__ void __launch_bounds__(NT, 1)
           store4(dst + (base + i * 128) * 4, make_float4(x[i].x + y[i].x, x[i].y + y[i].y, x[i].z + y[i].z, x[i].w + y[i].w));
       }
     };
-    // fp32 state -> pool entry (bf16 hi, then lo), coalesced
-    auto copy_split = [&](__nv_bfloat16* entry, const float* src) {
+    // fp32 state -> fp16 pool entry S / s (inv = 1 / s), coalesced
+    auto copy_f16 = [&](__half* entry, const float* src, float inv) {
       constexpr int N4 = D * D / 4;
 #pragma unroll 1
       for (int base = st; base < N4; base += 4 * 128) {
@@ -797,14 +820,7 @@ __global__ void __launch_bounds__(NT, 1)
 #pragma unroll
         for (int i = 0; i < 4; ++i) v[i] = load4(src + (base + i * 128) * 4);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int e = (base + i * 128) * 4;
-          const float4 x = v[i];
-          const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
-          const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-          store4(entry + e, make_float4(f01.x, f01.y, f23.x, f23.y));
-          store4(entry + D * D + e, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
-        }
+        for (int i = 0; i < 4; ++i) *reinterpret_cast<uint2*>(entry + (base + i * 128) * 4) = f16x4(v[i], inv);
       }
     };
 
@@ -830,7 +846,7 @@ __global__ void __launch_bounds__(NT, 1)
     if (pool && !a.carry_in) {  // snapshot 0: every live entry at the start of the round
       const long long lst = (long long)bh * a.snap_stride + a.snap_base;
       for (int i = 0; i < m_start && i < a.pool_cap; ++i)
-        copy_split(pool + (long long)i * kEntry, states + (long long)sm.slot0[i] * D * D);
+        copy_f16(pool + (long long)i * kEntry, states + (long long)sm.slot0[i] * D * D, 1.f / sm.scale0[i]);
       if (st == 0) a.snap_m0[lst] = m_start;
       if (st < m_start) a.snap_ids[lst * C + st] = st;
     }
@@ -886,7 +902,7 @@ __global__ void __launch_bounds__(NT, 1)
       const int snap_idx = (c + 1) / a.snap_chunks;
       const bool do_snap = pool && ivl_end && (snap_idx < a.nsnap || a.snap_at_end);
       float g = 0.f;
-      if (need_y || do_snap) g = split(cur);
+      if (need_y) g = split(cur);  // the y operand (snapshots take the fp32 state itself)
       if (need_y) {  // y of chunk c + 2 against S_open at the start of chunk c + 1
         const int s2 = (c + 2) % NKV;
         if (!(ok = state_all(mbar_wait(&sm.kv_full[s2], (uint32_t)(((c + 2) / NKV) & 1), abort, a.status)))) break;
@@ -904,21 +920,26 @@ __global__ void __launch_bounds__(NT, 1)
         const SnapBuf& sb = sm.snap[snap_idx & 1];
         const long long list_row = (long long)bh * a.snap_stride + a.snap_base + snap_idx;
         for (int jj = 0; jj < sb.njobs; ++jj) {
-          __nv_bfloat16* entry = pool + (long long)sb.src[jj][0] * kEntry;
+          __half* entry = pool + (long long)sb.src[jj][0] * kEntry;
           const int srcslot = sb.src[jj][1];
-          if (srcslot < 0) {  // the open entry: its hi / lo rows straight from TMEM (split above), by TMA
-            const int row0 = (bh * a.pool_cap + sb.src[jj][0]) * 2 * D;
+          const float inv = 1.f / sb.scale[jj];
+          if (srcslot < 0) {  // the open entry: its fp32 rows from TMEM, scaled into fp16, by TMA
+            const int row0 = (bh * a.pool_cap + sb.src[jj][0]) * D;
 #pragma unroll 1
-            for (int part = 0; part < 2; ++part) {
-              const uint32_t cols = part ? kColsLo : kColsHi;
-              float v[64];
-              tmem_ld32x2(tmem + lrow + cols, tmem + lrow + cols + 32, v);
-              stage_row(sm.out[0], v);
-              stage_row(sm.out[1], v + 32);
-              flush_tiles(&tmP, 0, row0 + part * D, 64, row0 + part * D);
+            for (int half = 0; half < 2; ++half) {
+              float v[64], w[32];
+              tmem_ld32x2(tmem + lrow + 128u * cur + 64 * half, tmem + lrow + 128u * cur + 64 * half + 32, v);
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const uint2 h = f16x4(make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]), inv);
+                w[2 * i] = __uint_as_float(h.x);
+                w[2 * i + 1] = __uint_as_float(h.y);
+              }
+              stage_row(sm.out[half], w);  // columns 64 * half .. + 63 of row j
             }
+            flush_tiles(&tmP, 0, row0, 64, row0);
           } else {
-            copy_split(entry, states + (long long)srcslot * D * D);
+            copy_f16(entry, states + (long long)srcslot * D * D, inv);
           }
         }
         if (st < sb.m) a.snap_ids[list_row * C + st] = sb.ids[st];
@@ -954,7 +975,7 @@ cudaError_t launch_scan_tc(const ScanArgs& a, cudaStream_t s) {
   CUtensorMap mk, mv, ms, mp;
   if (!a.pool || !tmap_tokens(&mk, a.k, a.B, a.T, a.H, L) || !tmap_tokens(&mv, a.v, a.B, a.T, a.H, L) ||
       !tmap_states(&ms, a.states, (long long)a.B * a.H * a.C * D) ||
-      !tmap_pool(&mp, a.pool, (long long)a.B * a.H * a.pool_cap * 2 * D))
+      !tmap_pool(&mp, a.pool, (long long)a.B * a.H * a.pool_cap * D, true))
     return cudaErrorInvalidValue;
   if (!a.gram || a.seq_lens || a.piece_ready || a.snap_chunks != 2) return cudaErrorInvalidValue;
   const size_t smem = scan_tc_smem_bytes();

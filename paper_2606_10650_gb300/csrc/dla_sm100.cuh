@@ -290,6 +290,12 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
 }
 // The same with B MN-major.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(int M, int N) { return idesc_bf16_f32(M, N) | (1u << 16); }
+// kind::f16 with fp16 A and B (format 0), fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4)                        // D format: f32
+         | ((uint32_t)(N >> 3) << 17)     // N / 8
+         | ((uint32_t)(M >> 4) << 24);    // M / 16
+}
 
 // Byte offset of element (row r, column c) of a K-major 128B-swizzled tile
 // whose rows hold 64 bf16 (c in 0..63).

@@ -36,8 +36,9 @@ inline bool tmap_tokens(CUtensorMap* m, const void* base, int B, int T, int H, i
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Snapshot pool as rows of 128 bf16: box (64, 128) with the 128-byte swizzle.
-inline bool tmap_pool(CUtensorMap* m, const void* base, long long rows) {
+// Snapshot pool as rows of 128 fp16 (the tensor-core read-out's entries) or
+// bf16: box (64, 128) with the 128-byte swizzle.
+inline bool tmap_pool(CUtensorMap* m, const void* base, long long rows, bool f16 = false) {
   auto fn = tmap_encode_fn();
   if (!fn) return false;
   constexpr int D = 128;
@@ -45,9 +46,9 @@ inline bool tmap_pool(CUtensorMap* m, const void* base, long long rows) {
   cuuint64_t strides[1] = {(cuuint64_t)D * 2};
   cuuint32_t box[2] = {64, 128};
   cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return fn(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+            dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // fp32 states as rows of 128 floats (the cache's [d_v][d_k] states): box (32, 128)
