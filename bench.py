@@ -283,8 +283,10 @@ def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headli
                 "peak_note": ("measured bf16 dense GEMM (burst) of MEASURED_PEAKS.json" if tc_path else
                               "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x sm_max_mhz"),
                 "work_per_launch": f"2*d^2*sum_t m_t / launches = {work:.4g} flop", "timing": timing_note,
-                "executed_note": ("each snapshot-state product runs as two bf16 MMAs (hi + lo split of the fp32 "
-                                  "state): executed tensor flops are about 2x the algorithmic count" if tc_path else "")}
+                "executed_note": ("each snapshot-state product runs as one fp16 MMA per interval (fp16 pool "
+                                  "entries, Q converted to fp16; fp16 runs at the bf16 dense rate), so the executed "
+                                  "snapshot flops equal the algorithmic count; the intra-interval products (Q K^T, "
+                                  "Pt V) come on top" if tc_path else "")}
             sm_ms[name] = t * n_launch * n_sms
         elif name == "scan":
             work = 4.0 * d * d * T * BH / max(n_launch, 1)  # x_t = v^T S k and the state build, 2 d^2 each per token
