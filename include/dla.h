@@ -56,6 +56,14 @@
  *   - Supported: d_k = d_v = d in {64, 128}; 2 <= C <= 64; T >= 1.  Anything
  *     else returns DLA_ERR_UNSUPPORTED (shape outside the built kernels) or
  *     DLA_ERR_INVALID_ARG (meaningless value).
+ *   - DLA(I), dynamic state merging without the capacity bound (Table 5): a
+ *     capacity C that no stream's segment count reaches gives exactly its
+ *     results.  dla_forward and dla_forward_noalloc also take 64 < C <= 256
+ *     for bf16 inputs with d = 128 over whole rows of device-resident inputs
+ *     (no seq_lens, no packed rows, not dla_forward_host); those instances hold
+ *     no capacity merge, so a stream whose segment count would pass C fails
+ *     the call's device check (DLA_ERR_DEVICE_CHECK, results undefined).
+ *     dla_decode_step and dla_backward take C <= 64.
  */
 #ifndef DLA_H
 #define DLA_H

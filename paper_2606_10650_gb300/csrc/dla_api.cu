@@ -203,7 +203,7 @@ dla_status check_params(const dla_params* p) {
   if (!isfinite(p->tau)) return fail(DLA_ERR_INVALID_ARG, "tau must be finite");
   if (!(p->eps >= 0.0) || !(p->rms_eps >= 0.0)) return fail(DLA_ERR_INVALID_ARG, "eps and rms_eps must be >= 0");
   if (p->capacity < 2) return fail(DLA_ERR_INVALID_ARG, "capacity must be >= 2 (Algorithm 2 merges a pair)");
-  if (p->capacity > dla::kMaxC) return fail(DLA_ERR_UNSUPPORTED, "capacity %d > %d", p->capacity, dla::kMaxC);
+  if (p->capacity > dla::kMaxCBig) return fail(DLA_ERR_UNSUPPORTED, "capacity %d > %d", p->capacity, dla::kMaxCBig);
   if (p->score_mode != 0 && p->score_mode != 1) return fail(DLA_ERR_INVALID_ARG, "score_mode must be 0 or 1");
   if (p->out_dtype != DLA_BF16 && p->out_dtype != DLA_F32) return fail(DLA_ERR_INVALID_ARG, "bad out_dtype");
   if (p->from_cache != 0 && p->from_cache != 1) return fail(DLA_ERR_INVALID_ARG, "from_cache must be 0 or 1");
@@ -665,6 +665,12 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   if ((s = check_shape(dk, dv)) != DLA_OK) return s;
   const int d = dk, C = p->capacity;
   if ((long long)B * T * H * d >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
+  if (C > dla::kMaxC) {  // the DLA(I) instances (no capacity merge)
+    if (in_dtype != DLA_BF16 || d != 128)
+      return fail(DLA_ERR_UNSUPPORTED, "capacity %d > %d needs bf16 inputs with d = 128", C, dla::kMaxC);
+    if (p->seq_lens || vl || io)
+      return fail(DLA_ERR_UNSUPPORTED, "capacity %d > %d takes whole rows of device-resident inputs", C, dla::kMaxC);
+  }
   if (vl) {
     if (!vl->cu || !aligned(vl->cu, 4)) return fail(DLA_ERR_INVALID_ARG, "cu_seqlens must be non-NULL and 4-byte aligned");
     if (p->seq_lens) return fail(DLA_ERR_INVALID_ARG, "a packed batch takes its lengths from cu_seqlens: seq_lens must be NULL");
@@ -799,7 +805,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   // (one CTA per stream) where the Gram pre-pass runs over whole rows of
   // resident inputs (it is correct but slower on the benchmark workloads:
   // its per-chunk chain is bound by the latency of small tensor-core groups).
-  const bool scan_tc = tc && P.gram_chunks > 0 && !seq_lens && !stream_in && scan_tc_requested();
+  const bool scan_tc = tc && C <= dla::kMaxC && P.gram_chunks > 0 && !seq_lens && !stream_in && scan_tc_requested();
   auto launch_main_scan = [&](cudaStream_t s_) -> cudaError_t {
     return scan_tc ? dla::launch_scan_tc(sa, s_) : dla::launch_scan_mma(sa, d, pool_bf16, s_);
   };
@@ -1161,6 +1167,8 @@ dla_status dla_decode_step(const dla_params* p, const dla_cache* cache, dla_dtyp
   if (!cache) return fail(DLA_ERR_INVALID_ARG, "cache is NULL");
   if ((s = check_shape(cache->dk, cache->dv)) != DLA_OK) return s;
   if ((s = check_cache(cache, cache->B, cache->H, p->capacity, cache->dk)) != DLA_OK) return s;
+  if (p->capacity > dla::kMaxC)
+    return fail(DLA_ERR_UNSUPPORTED, "dla_decode_step takes capacities up to %d", dla::kMaxC);
   if (!q || !k || !v || !o) return fail(DLA_ERR_INVALID_ARG, "q, k, v and o must be non-NULL");
   if (lam && !aligned(lam, 4)) return fail(DLA_ERR_INVALID_ARG, "lambda must be 4-byte aligned");
   dla::DecodeArgs da;
@@ -1198,6 +1206,7 @@ dla_status dla_backward(const dla_params* p, dla_dtype in_dtype, int B, int T, i
   if ((long long)B * H > 65535) return fail(DLA_ERR_UNSUPPORTED, "B * H must be at most 65535");
   if ((long long)B * T * H * dk >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
   if (p->from_cache) return fail(DLA_ERR_UNSUPPORTED, "dla_backward starts from an empty cache (from_cache = 0)");
+  if (p->capacity > dla::kMaxC) return fail(DLA_ERR_UNSUPPORTED, "dla_backward takes capacities up to %d", dla::kMaxC);
   if (p->seq_lens) return fail(DLA_ERR_UNSUPPORTED, "dla_backward takes whole rows (seq_lens = NULL)");
   if (!q || !k || !v || !boundary || !merge_log || !grad_o || !grad_q || !grad_k || !grad_v)
     return fail(DLA_ERR_INVALID_ARG, "q, k, v, boundary, merge_log, grad_o, grad_q, grad_k, grad_v must be non-NULL");

@@ -10,7 +10,12 @@
 
 namespace dla {
 
-constexpr int kMaxC = 64;   // largest supported capacity C
+constexpr int kMaxC = 64;   // largest capacity C with the capacity merge of Algorithm 2 on the GPU
+// Largest C of the DLA(I) instances (Table 5: dynamic merging only): bf16
+// inputs, d = 128, capacities above kMaxC hold up to kMaxCBig states without
+// merge machinery; a stream that would need a capacity merge fails the call's
+// device check.
+constexpr int kMaxCBig = 256;
 constexpr int kScanL = 64;  // tokens per scan chunk (K1)
 // Floats per chunk of the Gram pre-pass output: suffix table gs[j][t], its
 // prefix table Q[j][t], a_t, and the exclusive prefix sums

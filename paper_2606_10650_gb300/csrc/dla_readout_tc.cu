@@ -48,7 +48,6 @@ constexpr int NT = 576;   // 18 warps
 constexpr int NEPI = 16;  // epilogue warps
 constexpr int NHS = 4;   // shared-memory stages (32 KB: an fp16 state, a K / Pt tile or a V tile)
 constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
-constexpr int MAXU = 2 * kMaxC;  // union of two lists
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTile = L * 128;  // one K-major 128B-swizzled tile: 128 rows x 64 bf16
 constexpr int kRows = L + 1;         // events 0 .. L of an interval
@@ -65,12 +64,19 @@ struct Side {      // per interval of the pair
   uint8_t bnd[L];  // boundary flags
 };
 
+// CAPB: the largest capacity of the instance.  CAPB > kMaxC is the DLA(I)
+// instance: no merges, so an entry's logical slot is its list index and the
+// entry opened at the interval's e-th boundary sits at slot m0 - 1 + e; it
+// keeps no slot tables.
+template <int CAPB>
 struct TcSmem {
+  static constexpr bool kBig = CAPB > kMaxC;
+  static constexpr int MAXU = 2 * CAPB;  // union of two lists
   uint8_t Q[2][2][kTile];      // [interval][k-half]: Q, the A operand                 64 KB
   uint8_t hs[NHS][2][kTile];   // [stage][half]: K then Pt, V, then state parts         128 KB
-  unsigned char tab[2][kTabBytes];
+  unsigned char tab[2][kBig ? 16 : kTabBytes];
   Side side[2];
-  int ids[2][kMaxC];           // pool ids of the two lists
+  int ids[2][CAPB];            // pool ids of the two lists
   int uid[MAXU];               // union: pool id
   int uxa[MAXU], uxb[MAXU];    // union: index in list A / list B, or -1
   float uscale[MAXU];          // union: scale s_x of the fp16 entry (S_x / s_x is stored)
@@ -166,13 +172,15 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
 // through L2) and the output copied back piece by piece (per-piece CTA counts).
 // kRagged: per-row lengths (padding after them).  Separate instances, so the
 // common one keeps its code unchanged.
-template <bool kStream, bool kRagged>
+template <bool kStream, bool kRagged, int CAPB = kMaxC>
 __global__ void __launch_bounds__(NT, 1)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
                       int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
-  TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  using Smem = TcSmem<CAPB>;
+  constexpr bool kBig = Smem::kBig;
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int bh = blockIdx.x, pair = blockIdx.y;  // streams fastest: CTAs dispatched interval pair by pair
   const int b = bh / a.H, h = bh % a.H;
@@ -257,8 +265,8 @@ __global__ void __launch_bounds__(NT, 1)
       tma_load_4d(sm.Q[1][1], &tmQ, &sm.bar_q, 64, h, tma_t + c0B, tma_b);
     }
   }
-  for (int i = tid; i < 2 * kMaxC; i += NT) {
-    const int side = i / kMaxC, x = i % kMaxC;
+  for (int i = tid; i < 2 * CAPB; i += NT) {
+    const int side = i / CAPB, x = i % CAPB;
     int id = (x < (side ? m0B : m0A)) ? __ldcg(a.snap_ids + (side ? lrowB : lrowA) * C + x) : -1;
     if (x < (side ? m0B : m0A) && (id < 0 || id >= a.pool_cap)) {  // a pool id outside the pool
       atomicCAS(a.status, 0, 6);
@@ -270,7 +278,7 @@ __global__ void __launch_bounds__(NT, 1)
   __syncthreads();
   if (warp == 0) {
     // union of the two lists: list A in order, then the entries of list B not in A
-    for (int x = lane; x < kMaxC; x += 32) {
+    for (int x = lane; x < CAPB; x += 32) {
       if (x < m0A) {
         sm.uid[x] = sm.ids[0][x];
         sm.uxa[x] = x;
@@ -451,8 +459,10 @@ __global__ void __launch_bounds__(NT, 1)
       sm.side[sd].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");
-    if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-    if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    if constexpr (!kBig) {
+      if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+      if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    }
     if (etid < 2 * L) {
       const int sd = etid / L, tt = etid % L;
       sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
@@ -469,7 +479,13 @@ __global__ void __launch_bounds__(NT, 1)
     // an interval without boundary events (the common case) weights every
     // column s <= t of row t by lambda of the open entry: loaded ahead of P
     const bool no_ev = sm.side[side].evt[L - 1] == 0;  // warp-uniform
-    const float w_open = (no_ev && t < Lcs) ? (lam_t ? lam_at(sm.tab[side][0]) : 1.f) : 0.f;
+    const int m0s = side ? m0B : m0A;
+    // slot, after this row's events, of the entry opened at event e (0: the open entry)
+    auto intra_slot = [&](const unsigned char* trow_, int e) -> int {
+      if constexpr (kBig) return min(m0s - 1 + e, C - 1);  // a consistent trace stays below C
+      else return trow_[e];
+    };
+    const float w_open = (no_ev && t < Lcs) ? (lam_t ? lam_at(intra_slot(sm.tab[side], 0)) : 1.f) : 0.f;
     bool ok;
     {  // P (accumulator 0) -> Pt over this interval's K tile (its MMAs are complete)
       ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[0], 0, abort, status));
@@ -478,7 +494,7 @@ __global__ void __launch_bounds__(NT, 1)
         const uint32_t base = lane_addr + 128u * side + 64 * ch;
         // the weight of column s depends on s only through evt[s], which changes
         // at the interval's boundaries: it is looked up again only then
-        const unsigned char* trow = sm.tab[side] + evt_t * (evt_t + 1) / 2;
+        const unsigned char* trow = kBig ? sm.tab[side] : sm.tab[side] + evt_t * (evt_t + 1) / 2;
         const int* evs = sm.side[side].evt;
         int last_e = -1;
         float last_w = 0.f;
@@ -503,7 +519,7 @@ __global__ void __launch_bounds__(NT, 1)
                   const int e = evs[ss];
                   if (e != last_e) {
                     last_e = e;
-                    last_w = lam_t ? lam_at(trow[e]) : 1.f;
+                    last_w = lam_t ? lam_at(intra_slot(trow, e)) : 1.f;
                   }
                   wt = last_w;
                 }
@@ -572,8 +588,10 @@ __global__ void __launch_bounds__(NT, 1)
       }
     }
     asm volatile("bar.sync 1, 512;" ::: "memory");  // every warp is past the intra tables
-    if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-    if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    if constexpr (!kBig) {
+      if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
+      if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+    }
     asm volatile("bar.sync 1, 512;" ::: "memory");
     float o[64];
     {  // o starts from O (accumulator 1)
@@ -593,14 +611,14 @@ __global__ void __launch_bounds__(NT, 1)
     }
     const int* ux = side ? sm.uxb : sm.uxa;
     {  // snapshot part
-      const unsigned char* tab_t = sm.tab[side] + evt_t * kMaxC;
+      const unsigned char* tab_t = sm.tab[side] + (kBig ? 0 : evt_t * kMaxC);
       // weight of union state x for this token (0 when not in its interval's list):
       // lambda times the entry's scale s_x and the row's inverse Q scale
       auto weight = [&](int x) -> float {
         if (x >= nu || t >= Lcs) return 0.f;
         const int xi = ux[x];
         if (xi < 0) return 0.f;
-        return (lam_t ? lam_at(tab_t[xi]) : 1.f) * sm.uscale[x] * qinv;
+        return (lam_t ? lam_at(kBig ? xi : (int)tab_t[xi]) : 1.f) * sm.uscale[x] * qinv;
       };
       float wn = weight(0);
       for (int x = 0; ok && x < nu; ++x) {
@@ -665,10 +683,13 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
       !tmap_tokens(&mv, a.v, mb, (int)mt, a.H) || !tmap_pool(&ms, a.pool, rows, true))
     return cudaErrorInvalidValue;
   if (a.row_start && !a.seq_lens) return cudaErrorInvalidValue;  // the packed layout needs per-row lengths
-  const size_t smem = sizeof(TcSmem) + 1024;
+  const bool big = a.C > kMaxC;  // DLA(I): device-resident whole rows only
+  const size_t smem = big ? sizeof(TcSmem<kMaxCBig>) + 1024 : sizeof(TcSmem<kMaxC>) + 1024;
   const bool stream = a.lam_l2 || a.out_done, ragged = a.seq_lens != nullptr;
-  auto kern = stream ? (ragged ? readout_tc_kernel<true, true> : readout_tc_kernel<true, false>)
-                     : (ragged ? readout_tc_kernel<false, true> : readout_tc_kernel<false, false>);
+  if (big && (stream || ragged || a.C > kMaxCBig)) return cudaErrorInvalidValue;
+  auto kern = big ? readout_tc_kernel<false, false, kMaxCBig>
+                  : stream ? (ragged ? readout_tc_kernel<true, true> : readout_tc_kernel<true, false>)
+                           : (ragged ? readout_tc_kernel<false, true> : readout_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
@@ -677,7 +698,7 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
   return cudaGetLastError();
 }
 
-size_t readout_tc_smem_bytes() { return sizeof(TcSmem) + 1024; }
+size_t readout_tc_smem_bytes() { return sizeof(TcSmem<kMaxCBig>) + 1024; }
 
 cudaError_t preload_readout_kernels() {
   cudaFuncAttributes fa;
@@ -685,7 +706,8 @@ cudaError_t preload_readout_kernels() {
   if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false, false>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<true, false>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<false, true>)) != cudaSuccess) return e;
-  return cudaFuncGetAttributes(&fa, readout_tc_kernel<true, true>);
+  if ((e = cudaFuncGetAttributes(&fa, readout_tc_kernel<true, true>)) != cudaSuccess) return e;
+  return cudaFuncGetAttributes(&fa, readout_tc_kernel<false, false, kMaxCBig>);
 }
 
 }  // namespace dla

@@ -29,8 +29,11 @@ constexpr int GS = L;              // row of a Gram table in shared memory (the 
 
 enum : int { OP_CLOSE = 0, OP_MERGE = 1 };
 
-template <int D, int CL>
+template <int D, int CL, int CAPB = kMaxC>
 struct MmaSmem {
+  // CAPB > kMaxC: the DLA(I) instance, whose cache metadata lives here (b*)
+  static constexpr bool kBig = CAPB > kMaxC;
+  static constexpr int NB = kBig ? CAPB : 1;
   static constexpr int RP = D + 8;  // padded bf16 row: 8 rows of a ldmatrix hit 8 bank groups
   __nv_bfloat16 kv[2][2][L * RP];   // [stage][k / v][t][RP]
   __nv_bfloat16 S2[2][D / CL * RP]; // this CTA's rows of the open state as bf16 hi / lo, [j][RP]
@@ -44,13 +47,17 @@ struct MmaSmem {
   uint64_t xbar[2];                 // [chunk parity] the partner's parts have arrived (CTA pairs)
   int abort_flag;                   // a wait for the partner gave up
   float gred[NW];
-  int slot[kMaxC];                  // physical slots at the round start
+  int slot[CAPB];                   // physical slots at the round start (DLA(I): the live map)
   int open_slot;                    // physical slot of the open entry (m - 1) after the last replay
   int bnd[L];
   int mlog[L];
   int ops[3 * L + 4][4];
-  int snap_src[kMaxC][2];
-  float snap_scale[kMaxC];          // scale s of each snapshot job (fp16 pool: S / s is stored)
+  int snap_src[CAPB][2];
+  float snap_scale[CAPB];           // scale s of each snapshot job (fp16 pool: S / s is stored)
+  // DLA(I) instance: n, Ibar, pool id, changed flag and norm bound of every entry
+  double bib[NB];
+  int bn[NB], bpid[NB], bdirty[NB];
+  float bnb[NB];
   int nops, nsnapjobs;
   int pend;                         // snapshot copies waiting for the next chunk's idle warps (bf16 pool)
   int gcnt[kMaxGramBlk];            // Gram pre-pass counters last read (thread 0)
@@ -421,8 +428,9 @@ __device__ __forceinline__ void put_pair(float* entry, int D, int j, int k, floa
 // rank 1 in both), and rank 0 writes the trace, the lists and the metadata.
 // kRagged: per-row lengths (padding after them); a separate instance, so the
 // common one keeps its code.
-template <int D, typename Tpool, int CL, bool kRagged = false>
+template <int D, typename Tpool, int CL, bool kRagged = false, int CAPB = kMaxC>
 __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
+  constexpr bool kBig = CAPB > kMaxC;  // DLA(I): up to CAPB states, no capacity merge
   constexpr int RP = D + 8;
   constexpr int R = D / CL;           // state rows of this CTA
   constexpr int MT = R / 16;          // 16-row bands of those rows
@@ -431,7 +439,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   constexpr int NT8 = KC / 8;         // n8 tiles per warp in the state build
   static_assert(L == 64 && KC % 16 == 0, "x GEMM tiling");
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  MmaSmem<D, CL>& sm = *reinterpret_cast<MmaSmem<D, CL>*>(smem_raw);
+  MmaSmem<D, CL, CAPB>& sm = *reinterpret_cast<MmaSmem<D, CL, CAPB>*>(smem_raw);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g = lane >> 2, tg = lane & 3;
@@ -500,7 +508,17 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
   int e_n[2] = {0, 0}, e_slot[2] = {0, 0}, e_pid[2] = {-1, -1}, e_dirty[2] = {0, 0};
   double e_ib[2] = {0.0, 0.0};
   float e_nb[2] = {0.f, 0.f};
-  if (warp == 0) {
+  if constexpr (kBig) {  // in shared memory: n, Ibar, pool id, changed, norm bound
+    for (int i = tid; i < C; i += NT) {
+      sm.bn[i] = a.n[(long long)bh * C + i];
+      sm.bib[i] = a.ibar[(long long)bh * C + i];
+      sm.bpid[i] = -1;
+      sm.bdirty[i] = 0;
+      sm.bnb[i] = (kF16 && pool && i < m_start) ? a.nbound[(long long)bh * C + i] : 0.f;
+      // no merge ever freed a physical slot: the live entries use slots 0 .. m - 1
+      if (i < m_start && sm.slot[i] >= m_start) atomicCAS(a.status, 0, 6);
+    }
+  } else if (warp == 0) {
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int i = lane + 32 * r;
@@ -529,13 +547,24 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     const long long lst = (long long)bh * a.snap_stride + a.snap_base;  // list row of this round's first interval
     if (a.carry_in) {  // the pool continues: the previous round wrote this interval's list
       if (tid == 0) sm.pool_next = a.pstate[bh];
-      if (warp == 0)
+      if constexpr (kBig) {
+        for (int i = tid; i < m_start; i += NT) sm.bpid[i] = a.pstate[a.B * a.H + (long long)bh * C + i];
+      } else if (warp == 0) {
 #pragma unroll
         for (int r = 0; r < 2; ++r)
           if (lane + 32 * r < m_start) e_pid[r] = a.pstate[a.B * a.H + (long long)bh * C + lane + 32 * r];
+      }
     } else {  // snapshot 0: every live entry at the start of the round
       if constexpr (kF16) {
-        if (warp == 0)
+        if constexpr (kBig) {
+          __syncthreads();  // the norm bounds above
+          for (int i = tid; i < m_start && i < a.pool_cap; i += NT) {
+            const float sc = f16_scale(sm.bnb[i]);
+            sm.snap_scale[i] = sc;
+            sm.bpid[i] = i;
+            if (lead) a.pool_scale[(long long)bh * a.pool_cap + i] = sc;
+          }
+        } else if (warp == 0) {
 #pragma unroll
           for (int r = 0; r < 2; ++r) {
             const int i = lane + 32 * r;
@@ -545,6 +574,7 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
               if (lead) a.pool_scale[(long long)bh * a.pool_cap + i] = sc;
             }
           }
+        }
         __syncthreads();
         for (int i = 0; i < m_start && i < a.pool_cap; ++i)
           copy_state_f16<D, R>(pool + (long long)i * kEntry + (long long)rbase * D, srows(sm.slot[i]),
@@ -833,7 +863,11 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       const float* qst = gst + L * L;
       const float aa = gst[2 * L * L + ta], ab = gst[2 * L * L + tb];
       // fp16 pool: the open entry's norm bound restarts from its exact norm
-      if (kF16 && m_chunk > 0) entry_set(e_nb, m_chunk - 1, sqrtf(fmaxf(gam_open, 0.f)));
+      if constexpr (kBig) {
+        if (m_chunk > 0 && lane == 0) sm.bnb[m_chunk - 1] = sqrtf(fmaxf(gam_open, 0.f));
+      } else {
+        if (kF16 && m_chunk > 0) entry_set(e_nb, m_chunk - 1, sqrtf(fmaxf(gam_open, 0.f)));
+      }
       // exclusive prefix sums of x_t and a_t over the chunk: with the table Q,
       // sum_{js <= u < t} (2 beta_u + a_u) = 2 (X(t) - X(js)) [open state] + 2 Q[js][t] + A(t) - A(js)
       float xpa, xpb, apa, apb;
@@ -898,112 +932,173 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
       // fp16 pool: a run [u0, u1) grows its entry's norm bound by SA(u1) - SA(u0)
       // (the chunk's prefix sums of |v_t| |k_t| = sqrt(a_t), in its Gram block)
       const float* sa_blk = gst + kGramSA;
-      int m = m_chunk;
-      int seg_u0 = 0, nops = 0, run0 = 0;
-      unsigned long long pend = bmask;
-      while (true) {
-        const int t = pend ? (__ffsll((long long)pend) - 1) : Lc;
-        pend &= pend - 1;
-        if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
-          const double part = (double)run_sum(run0, t);
-          // |S + sum v k^T|_F <= |S|_F + sum |v| |k|, and |v_t| |k_t| = sqrt(a_t)
-          float grow = 0.f;
-          if constexpr (kF16) grow = sa_blk[t] - sa_blk[run0];
-          const int e = m - 1;
-          if ((e & 31) == lane) {
-            if (e < 32) {
-              e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1; e_nb[0] += grow;
-            } else {
-              e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1; e_nb[1] += grow;
+      if constexpr (kBig) {
+        // DLA(I): entries only open and grow; a boundary into a full cache would
+        // need the capacity merge this instance does not hold
+        int m = m_chunk;
+        int seg_u0 = 0, nops = 0, run0 = 0;
+        unsigned long long pend = bmask;
+        while (true) {
+          const int t = pend ? (__ffsll((long long)pend) - 1) : Lc;
+          pend &= pend - 1;
+          if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
+            const double part = (double)run_sum(run0, t);
+            if (lane == 0) {
+              const int e = m - 1;
+              sm.bn[e] += t - run0;
+              sm.bib[e] += part;
+              sm.bdirty[e] = 1;
+              sm.bnb[e] += sa_blk[t] - sa_blk[run0];
             }
           }
-        }
-        run0 = t + 1;
-        if (t >= Lc) break;
-        if (m > 0) {
-          const int sl = entry_get(e_slot, m - 1);
+          run0 = t + 1;
+          if (t >= Lc) break;
+          if (m >= C) {  // no room: the call fails its device check (results undefined)
+            if (lane == 0) {
+              atomicCAS(a.status, 0, 6);
+              sm.mlog[t] = -1;
+              sm.bnd[t] = 0;  // the trace stays a valid replay: no entry was opened
+            }
+            run0 = t;  // the token stays in the open state
+            continue;
+          }
+          if (m > 0) {
+            if (lane == 0) {
+              sm.ops[nops][0] = OP_CLOSE;
+              sm.ops[nops][1] = sm.slot[m - 1];
+              sm.ops[nops][2] = seg_u0;
+              sm.ops[nops][3] = t;
+            }
+            ++nops;
+          }
+          const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
           if (lane == 0) {
-            sm.ops[nops][0] = OP_CLOSE;
-            sm.ops[nops][1] = sl;
-            sm.ops[nops][2] = seg_u0;
-            sm.ops[nops][3] = t;
+            sm.slot[m] = m;  // slots 0 .. m - 1 are the live ones: slot m is free
+            sm.bn[m] = 1;
+            sm.bib[m] = (double)it;
+            sm.bpid[m] = -1;
+            sm.bdirty[m] = 1;
+            sm.bnb[m] = sa_blk[t + 1] - sa_blk[t];
+            sm.mlog[t] = -1;
           }
-          ++nops;
+          m += 1;
+          seg_u0 = t;
         }
-        int j = -1, phys_new = m;
-        if (m == C) {
-          // pair densities (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}): fp64 sums, compared in fp32
-          int nn[2], ns[2], np_[2], nd[2];
-          double nb[2];
-          float nnb[2];
-          entry_next(e_n, nn);
-          entry_next(e_ib, nb);
-          entry_next(e_nb, nnb);
-          entry_next(e_slot, ns);
-          entry_next(e_pid, np_);
-          entry_next(e_dirty, nd);
-          float best = __int_as_float(0x7f800000);
-          int bi = 0x7fffffff;
-          if (lane + 1 < m) {
-            best = (float)(e_ib[0] + nb[0]) / (float)(e_n[0] + nn[0]);
-            bi = lane;
-          }
-          if (lane + 33 < m) {
-            const float d1 = (float)(e_ib[1] + nb[1]) / (float)(e_n[1] + nn[1]);
-            if (d1 < best) {
-              best = d1;
-              bi = lane + 32;
-            }
-          }
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, best, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ov < best || (ov == best && oi < bi)) {
-              best = ov;
-              bi = oi;
-            }
-          }
-          j = bi;
-          const int dst = entry_get(e_slot, j), srcs = entry_get(e_slot, j + 1);
-          if (lane == 0) {
-            sm.ops[nops][0] = OP_MERGE;
-            sm.ops[nops][1] = dst;
-            sm.ops[nops][2] = srcs;
-            sm.ops[nops][3] = 0;
-          }
-          ++nops;
-          // entry j absorbs j + 1; entries j + 2 .. m - 1 move down by one
-#pragma unroll
-          for (int r = 0; r < 2; ++r) {
-            const int i = lane + 32 * r;
-            if (i == j) {
-              e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1; e_nb[r] += nnb[r];
-            } else if (i > j && i < m - 1) {
-              e_n[r] = nn[r]; e_ib[r] = nb[r]; e_slot[r] = ns[r]; e_pid[r] = np_[r]; e_dirty[r] = nd[r];
-              e_nb[r] = nnb[r];
-            }
-          }
-          phys_new = srcs;
-          m -= 1;
+        __syncwarp();
+        if (lane == 0) {
+          sm.m = m;
+          sm.nops = nops;
+          sm.js = seg_u0;
+          sm.open_slot = (m > 0) ? sm.slot[m - 1] : 0;
         }
-        const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
-        if constexpr (kF16) entry_set(e_nb, m, sa_blk[t + 1] - sa_blk[t]);
-        entry_set(e_slot, m, phys_new);
-        entry_set(e_n, m, 1);
-        entry_set(e_ib, m, (double)it);
-        entry_set(e_pid, m, -1);
-        entry_set(e_dirty, m, 1);
-        if (lane == 0) sm.mlog[t] = j;
-        m += 1;
-        seg_u0 = t;
-      }
-      const int oslot = (m > 0) ? entry_get(e_slot, m - 1) : 0;
-      if (lane == 0) {
-        sm.m = m;
-        sm.nops = nops;
-        sm.js = seg_u0;
-        sm.open_slot = oslot;
+      } else {
+        int m = m_chunk;
+        int seg_u0 = 0, nops = 0, run0 = 0;
+        unsigned long long pend = bmask;
+        while (true) {
+          const int t = pend ? (__ffsll((long long)pend) - 1) : Lc;
+          pend &= pend - 1;
+          if (t > run0) {  // tokens [run0, t) joined the open state (entry m - 1)
+            const double part = (double)run_sum(run0, t);
+            // |S + sum v k^T|_F <= |S|_F + sum |v| |k|, and |v_t| |k_t| = sqrt(a_t)
+            float grow = 0.f;
+            if constexpr (kF16) grow = sa_blk[t] - sa_blk[run0];
+            const int e = m - 1;
+            if ((e & 31) == lane) {
+              if (e < 32) {
+                e_n[0] += t - run0; e_ib[0] += part; e_dirty[0] = 1; e_nb[0] += grow;
+              } else {
+                e_n[1] += t - run0; e_ib[1] += part; e_dirty[1] = 1; e_nb[1] += grow;
+              }
+            }
+          }
+          run0 = t + 1;
+          if (t >= Lc) break;
+          if (m > 0) {
+            const int sl = entry_get(e_slot, m - 1);
+            if (lane == 0) {
+              sm.ops[nops][0] = OP_CLOSE;
+              sm.ops[nops][1] = sl;
+              sm.ops[nops][2] = seg_u0;
+              sm.ops[nops][3] = t;
+            }
+            ++nops;
+          }
+          int j = -1, phys_new = m;
+          if (m == C) {
+            // pair densities (Ibar_i + Ibar_{i+1}) / (n_i + n_{i+1}): fp64 sums, compared in fp32
+            int nn[2], ns[2], np_[2], nd[2];
+            double nb[2];
+            float nnb[2];
+            entry_next(e_n, nn);
+            entry_next(e_ib, nb);
+            entry_next(e_nb, nnb);
+            entry_next(e_slot, ns);
+            entry_next(e_pid, np_);
+            entry_next(e_dirty, nd);
+            float best = __int_as_float(0x7f800000);
+            int bi = 0x7fffffff;
+            if (lane + 1 < m) {
+              best = (float)(e_ib[0] + nb[0]) / (float)(e_n[0] + nn[0]);
+              bi = lane;
+            }
+            if (lane + 33 < m) {
+              const float d1 = (float)(e_ib[1] + nb[1]) / (float)(e_n[1] + nn[1]);
+              if (d1 < best) {
+                best = d1;
+                bi = lane + 32;
+              }
+            }
+  #pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+              const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+              const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+              if (ov < best || (ov == best && oi < bi)) {
+                best = ov;
+                bi = oi;
+              }
+            }
+            j = bi;
+            const int dst = entry_get(e_slot, j), srcs = entry_get(e_slot, j + 1);
+            if (lane == 0) {
+              sm.ops[nops][0] = OP_MERGE;
+              sm.ops[nops][1] = dst;
+              sm.ops[nops][2] = srcs;
+              sm.ops[nops][3] = 0;
+            }
+            ++nops;
+            // entry j absorbs j + 1; entries j + 2 .. m - 1 move down by one
+  #pragma unroll
+            for (int r = 0; r < 2; ++r) {
+              const int i = lane + 32 * r;
+              if (i == j) {
+                e_n[r] += nn[r]; e_ib[r] += nb[r]; e_dirty[r] = 1; e_pid[r] = -1; e_nb[r] += nnb[r];
+              } else if (i > j && i < m - 1) {
+                e_n[r] = nn[r]; e_ib[r] = nb[r]; e_slot[r] = ns[r]; e_pid[r] = np_[r]; e_dirty[r] = nd[r];
+                e_nb[r] = nnb[r];
+              }
+            }
+            phys_new = srcs;
+            m -= 1;
+          }
+          const float it = __shfl_sync(0xffffffffu, (t & 1) ? Ib : Ia, t >> 1);
+          if constexpr (kF16) entry_set(e_nb, m, sa_blk[t + 1] - sa_blk[t]);
+          entry_set(e_slot, m, phys_new);
+          entry_set(e_n, m, 1);
+          entry_set(e_ib, m, (double)it);
+          entry_set(e_pid, m, -1);
+          entry_set(e_dirty, m, 1);
+          if (lane == 0) sm.mlog[t] = j;
+          m += 1;
+          seg_u0 = t;
+        }
+        const int oslot = (m > 0) ? entry_get(e_slot, m - 1) : 0;
+        if (lane == 0) {
+          sm.m = m;
+          sm.nops = nops;
+          sm.js = seg_u0;
+          sm.open_slot = oslot;
+        }
       }
     }
     __syncthreads();
@@ -1041,7 +1136,38 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
     const int snap_idx = (c + 1) / a.snap_chunks;
     const long long lrow = (long long)bh * a.snap_stride + a.snap_base + snap_idx;
     if (pool && interval_end && (snap_idx < a.nsnap || a.snap_at_end)) {
-      if (warp == 0) {  // entries whose state changed get a fresh pool entry
+      if (kBig && warp == 0) {  // the same over the shared-memory metadata
+        const int m = sm.m;
+        int nj = 0;
+        for (int base = 0; base < m; base += 32) {
+          const int i = base + lane;
+          const bool need = (i < m) && (sm.bdirty[i] || sm.bpid[i] < 0);
+          const unsigned bal = __ballot_sync(0xffffffffu, need);
+          if (need) {
+            const int rank_ = nj + __popc(bal & ((1u << lane) - 1u));
+            int p = sm.pool_next + rank_;
+            if (p >= a.pool_cap) {  // cannot happen with a correctly sized workspace
+              atomicExch(a.status, 6);
+              p = a.pool_cap - 1;
+            }
+            sm.bpid[i] = p;
+            sm.bdirty[i] = 0;
+            sm.snap_src[rank_][0] = p;
+            sm.snap_src[rank_][1] = (i == m - 1) ? -1 : sm.slot[i];
+            const float sc = f16_scale(sm.bnb[i]);
+            sm.snap_scale[rank_] = sc;
+            if (lead) a.pool_scale[(long long)bh * a.pool_cap + p] = sc;
+          }
+          nj += __popc(bal);
+          if (lead && i < m) a.snap_ids[lrow * C + i] = sm.bpid[i];
+        }
+        __syncwarp();
+        if (lane == 0) {
+          sm.pool_next += nj;
+          sm.nsnapjobs = nj;
+          if (lead) a.snap_m0[lrow] = m;
+        }
+      } else if (warp == 0) {  // entries whose state changed get a fresh pool entry
         const int m = sm.m;
         int nj = 0;
 #pragma unroll
@@ -1129,7 +1255,19 @@ __global__ void __launch_bounds__(NT, 1) scan_mma_kernel(ScanArgs a) {
         *reinterpret_cast<float2*>(dst + (jg0 + g + 8) * D + k) = make_float2(acc[n][2], acc[n][3]);
       }
     }
-    if (lead && warp == 0) {
+    if (kBig && lead && warp == 0) {
+      for (int i = lane; i < C; i += 32) {
+        a.slot[(long long)bh * C + i] = (i < m) ? sm.slot[i] : i;
+        a.n[(long long)bh * C + i] = (i < m) ? sm.bn[i] : 0;
+        a.ibar[(long long)bh * C + i] = (i < m) ? sm.bib[i] : 0.0;
+        if (pool && a.pstate && i < m) a.pstate[a.B * a.H + (long long)bh * C + i] = sm.bpid[i];
+        if (pool && i < m) a.nbound[(long long)bh * C + i] = sm.bnb[i];
+      }
+      if (lane == 0) {
+        a.m[bh] = m;
+        if (pool && a.pstate) a.pstate[bh] = sm.pool_next;
+      }
+    } else if (lead && warp == 0) {
 #pragma unroll
       for (int r = 0; r < 2; ++r) {
         const int i = lane + 32 * r;
@@ -1407,10 +1545,10 @@ cudaError_t launch_gram(const GramArgs& a, int d, cudaStream_t s) {
   return d == 128 ? launch_gram_t<128>(a, s) : launch_gram_t<64>(a, s);
 }
 
-template <int D, typename Tpool, int CL, bool kRagged>
+template <int D, typename Tpool, int CL, bool kRagged, int CAPB = kMaxC>
 static cudaError_t launch_scan_mma_r(const ScanArgs& a, cudaStream_t s) {
-  const size_t smem = sizeof(MmaSmem<D, CL>);
-  auto kern = scan_mma_kernel<D, Tpool, CL, kRagged>;
+  const size_t smem = sizeof(MmaSmem<D, CL, CAPB>);
+  auto kern = scan_mma_kernel<D, Tpool, CL, kRagged, CAPB>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -1519,6 +1657,8 @@ cudaError_t preload_scan_kernels() {
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 1>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 2, true>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 1, true>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 2, false, kMaxCBig>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&fa, scan_mma_kernel<128, __half, 1, false, kMaxCBig>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_kernel<128>)) != cudaSuccess) return e;
   if ((e = cudaFuncGetAttributes(&fa, gram_tc_kernel<128>)) != cudaSuccess) return e;
   return cudaFuncGetAttributes(&fa, gate_kernel);
@@ -1529,6 +1669,11 @@ cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStre
 }
 
 cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s) {
+  if (a.C > kMaxC) {  // DLA(I): bf16 inputs, d = 128, whole rows
+    if (d != 128 || !pool_bf16 || a.C > kMaxCBig || a.seq_lens) return cudaErrorInvalidValue;
+    return use_pairs(a) ? launch_scan_mma_r<128, __half, 2, false, kMaxCBig>(a, s)
+                        : launch_scan_mma_r<128, __half, 1, false, kMaxCBig>(a, s);
+  }
   if (d == 128) {
     if (use_pairs(a))
       return pool_bf16 ? launch_scan_mma_t<128, __half, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);

@@ -50,7 +50,9 @@ def _fwd(L, p, dt=dla.DLA_BF16, B=1, T=64, H=2, d=128, k=True, ws_bytes=1 << 40,
 def test_argument_errors_return_status_codes(L):
     p = dla.make_params(0.6, 8)
     assert _fwd(L, dla.make_params(0.6, 1)) == 1          # C < 2: Algorithm 2 needs a pair
-    assert _fwd(L, dla.make_params(0.6, 65)) == 2         # beyond the built capacity
+    assert _fwd(L, dla.make_params(0.6, 257)) == 2        # beyond the built capacity
+    assert _fwd(L, dla.make_params(0.6, 65), dt=dla.DLA_F32) == 2  # DLA(I) capacities: bf16 only
+    assert _fwd(L, dla.make_params(0.6, 65), d=64) == 2           # ... and d = 128
     assert _fwd(L, dla.make_params(float("nan"), 8)) == 1
     assert _fwd(L, dla.make_params(0.6, 8, score_mode=3)) == 1
     assert _fwd(L, p, d=96) == 2

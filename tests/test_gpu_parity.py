@@ -263,6 +263,50 @@ def test_dla_i_without_capacity_bound():
     structural_checks(w, g, w.T)
 
 
+@pytest.mark.timeout(900)
+@pytest.mark.parametrize("sched", ["concurrent", "rounds"])
+def test_dla_i_beyond_64_segments(sched, monkeypatch):
+    """DLA(I) (Table 5: dynamic merging without the capacity bound) at the regime
+    workload's length, where streams open up to about 80 segments: with C = 128
+    (the instances beyond 64, which hold no capacity merge) nothing merges, and
+    decisions, caches and outputs equal the oracle's.  Outputs are compared on
+    every 16th token (the oracle's read-out of up to 80 states at every token
+    takes much longer than the rest)."""
+    monkeypatch.setenv("DLA_SCHEDULE", sched)
+    w = W.get("regime", B=1, H=5, C=128)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    want = np.zeros(w.T, bool)
+    want[::16] = True
+    want[-1] = True
+    r = oracle.forward(q, k, v, lam, tau=w.tau, C=w.C, eps=w.eps, rms_eps=w.rms_eps, want_o=want)
+    rep = {}
+    compare(w, g, r, report=rep)
+    structural_checks(w, g, w.T)
+    assert (g["merge_log"] == -1).all()
+    ex = g["cache"].export()
+    assert ex["m"].max() > 64, ex["m"]
+    print("segments", ex["m"].tolist(), rep)
+
+
+def test_dla_i_segments_past_the_capacity_are_reported():
+    """A capacity above 64 with a stream whose segments pass it (the DLA(I)
+    instances hold no capacity merge): the call reports status 6 and the next
+    call on the stream is correct."""
+    w = W.get("regime", B=1, H=5, T=16384, C=65)
+    q, k, v, lam = W.host_batch(w, T=w.T)
+    qt, kt, vt, lt = upload(w, q, k, v, lam)
+    dev = torch.device("cuda:0")
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    o = torch.zeros((w.B, w.T, w.H, w.d), dtype=torch.float32, device=dev)
+    dla.dla_forward(p, qt, kt, vt, lt, o, dla.Cache(w.B, w.H, w.C, w.d, device=dev))
+    assert dla.dla_sync_status() == 6
+    w2 = W.get("regime", B=1, H=2, T=2000, C=96)
+    q2, k2, v2, l2 = _safe(w2)
+    g = run_gpu(w2, q2, k2, v2, l2)
+    compare(w2, g, run_oracle(w2, q2, k2, v2, l2))
+
+
 RAGGED = {
     # name: (workload, overrides, per-row lengths)
     "regime_bf16": ("regime", dict(B=3, H=2, T=1300), [1300, 517, 1]),
