@@ -111,6 +111,14 @@ __device__ __forceinline__ int slot_of(const int* f, int s) {
   return i;
 }
 
+// Slot of token s0 and whether tokens s0 .. s0 + 63 all share it (no later
+// entry starts inside the block): then one lookup serves a whole tile row.
+__device__ __forceinline__ int block_slot(const int* f, int s0, bool& uniform) {
+  const int sl = slot_of(f, s0);
+  uniform = (sl + 1 >= kMaxC) || (f[sl + 1] > s0 + BT - 1);
+  return sl;
+}
+
 // ---------------------------------------------------------------- shared tiles
 template <int D>
 struct BwdTiles {
@@ -281,6 +289,8 @@ __global__ void __launch_bounds__(NTB) dq_kernel(BackwardArgs a) {
       const int rl = r0 + g + 8 * half, t = t0 + rl;
       const int* f = sm.firsts + rl * kMaxC;
       const float* lw = sm.lam + rl * kMaxC;
+      bool uni = false;
+      const int slu = (rl < nt) ? block_slot(f, s0, uni) : 0;  // the common case: one entry over the tile
       int run_slot = -1;
       float run = 0.f;
 #pragma unroll
@@ -291,7 +301,7 @@ __global__ void __launch_bounds__(NTB) dq_kernel(BackwardArgs a) {
           const int idx = 2 * half + c;
           float w = 0.f;
           if (s <= t && rl < nt && s < a.T) {
-            const int sl = slot_of(f, s);
+            const int sl = uni ? slu : slot_of(f, s);
             w = lw[sl];
             const float pd = p[nt8][idx] * dp[nt8][idx];
             if (sl != run_slot) {
@@ -350,6 +360,8 @@ struct DkvSmem {
   __nv_bfloat16 K[BT * RP], V[BT * RP], Q[BT * RP], Ghi[BT * RP], Glo[BT * RP];
   float lam[BT * kMaxC];
   int firsts[BT * kMaxC];
+  int slot0[BT];   // per token t of the block: slot of token s0 after t
+  int uni[BT];     // and whether every token of the s block shares it
 };
 
 // dK and dV of one 64-token block of s of one stream: warps 0-3 dV, warps 4-7 dK
@@ -386,6 +398,12 @@ __global__ void __launch_bounds__(NTK) dkv_kernel(BackwardArgs a) {
     load_bf16_rows<D>(sm.Q, q + (long long)t0 * row_stride, row_stride, nt, tid, NTK);
     load_split_rows<D>(sm.Ghi, sm.Glo, gsrc + (long long)t0 * row_stride, row_stride, nt, tid, NTK);
     load_weights(sm.lam, sm.firsts, a, b, h, bh, t0, nt, tid, NTK);
+    __syncthreads();
+    if (tid < BT) {
+      bool u = false;
+      sm.slot0[tid] = (tid < nt) ? block_slot(sm.firsts + tid * kMaxC, s0, u) : 0;
+      sm.uni[tid] = u;
+    }
     __syncthreads();
     // X^T[s, t] (16 rows of s x 64 t): P^T = K Q^T (dV warps) or dP^T = V G^T (dK warps)
     float x[8][4];
@@ -424,7 +442,7 @@ __global__ void __launch_bounds__(NTK) dkv_kernel(BackwardArgs a) {
         for (int half = 0; half < 2; ++half) {
           const int s = s0 + r0 + g + 8 * half;
           float w = 0.f;
-          if (s <= t && tl < nt && s < a.T) w = sm.lam[tl * kMaxC + slot_of(f, s)];
+          if (s <= t && tl < nt && s < a.T) w = sm.lam[tl * kMaxC + (sm.uni[tl] ? sm.slot0[tl] : slot_of(f, s))];
           x[nt8][2 * half + c] *= w;
         }
       }
