@@ -176,7 +176,7 @@ template <bool kStream, bool kRagged, int CAPB = kMaxC>
 __global__ void __launch_bounds__(NT, 1)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
-                      int32_t* status) {
+                      const __grid_constant__ CUtensorMap tmO, int32_t* status) {
   extern __shared__ uint8_t smem_raw[];
   using Smem = TcSmem<CAPB>;
   constexpr bool kBig = Smem::kBig;
@@ -644,7 +644,33 @@ __global__ void __launch_bounds__(NT, 1)
         if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
       }
     }
-    if (ok && !*abort && side_in && t < Lcs) {
+    // fp32 output of the common instance: staged in the ring stages (free once
+    // every state product is complete, which this warp has seen) in the
+    // 128-byte swizzle and stored by TMA, eight 128-row x 32-column tiles per
+    // CTA (rows past T are clipped); otherwise per-row stores
+    bool tma_out = false;
+    if constexpr (!kStream && !kRagged) tma_out = (a.out_bf16 == 0);
+    if (tma_out) {
+      if (ok && side_in) {
+#pragma unroll
+        for (int cbl = 0; cbl < 2; ++cbl) {
+          const int box = side * 4 + 2 * ch + cbl;
+          uint8_t* tile = sm.hs[box >> 1][box & 1];
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<float4*>(tile + t * 128 + ((c ^ (t & 7)) << 4)) =
+                make_float4(o[32 * cbl + 4 * c], o[32 * cbl + 4 * c + 1], o[32 * cbl + 4 * c + 2], o[32 * cbl + 4 * c + 3]);
+        }
+      }
+      fence_proxy_async();  // the staged output feeds the TMA engine
+      asm volatile("bar.sync 1, 512;" ::: "memory");
+      if (ew == 0 && lane == 0 && !*abort) {
+        for (int box = 0; box < (hasB ? 8 : 4); ++box)
+          tma_store_4d(&tmO, sm.hs[box >> 1][box & 1], 32 * (box & 3), h, tma_t + c0_of(box >> 2), tma_b);
+        bulk_commit();
+        bulk_wait0();  // the CTA's shared memory stays valid until the stores are done
+      }
+    } else if (ok && !*abort && side_in && t < Lcs) {
       const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
       if (a.out_bf16) {
         __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
@@ -673,7 +699,7 @@ __global__ void __launch_bounds__(NT, 1)
 
 // ---------------------------------------------------------------- host side
 cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_t st) {
-  CUtensorMap mq, mk, mv, ms;
+  CUtensorMap mq, mk, mv, ms, mo;
   const long long rows = (long long)a.B * a.H * a.pool_cap * D;  // fp16 entries of D rows
   // packed layout: one batch coordinate over all token rows
   const int mb = a.row_start ? 1 : a.B;
@@ -694,7 +720,13 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
   if (e != cudaSuccess) return e;
   if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
   dim3 grid(a.B * a.H, (a.nsnap + 1) / 2);  // streams x pairs of intervals
-  kern<<<grid, NT, smem, st>>>(a, mq, mk, mv, ms, status);
+  // the common instance stores an fp32 output by TMA (the map is unused otherwise)
+  if (!stream && !ragged && !a.out_bf16) {
+    if (!tmap_out_f32(&mo, a.o, a.B, a.T, a.H)) return cudaErrorInvalidValue;
+  } else {
+    mo = mq;
+  }
+  kern<<<grid, NT, smem, st>>>(a, mq, mk, mv, ms, mo, status);
   return cudaGetLastError();
 }
 

@@ -36,6 +36,21 @@ inline bool tmap_tokens(CUtensorMap* m, const void* base, int B, int T, int H, i
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// [B, T, H, D] fp32 output rows: dims (k, h, t, b), box (32, 1, 128, 1) with the
+// 128-byte swizzle (a 128-token x 32-column tile, 16 KB; the store of the
+// read-out's output staging).  Rows past T are not written.
+inline bool tmap_out_f32(CUtensorMap* m, void* base, int B, int T, int H, int D = 128) {
+  auto fn = tmap_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)T, (cuuint64_t)B};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 4, (cuuint64_t)H * D * 4, (cuuint64_t)T * H * D * 4};
+  cuuint32_t box[4] = {32, 1, 128, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Snapshot pool as rows of 128 fp16 (the tensor-core read-out's entries) or
 // bf16: box (64, 128) with the 128-byte swizzle.
 inline bool tmap_pool(CUtensorMap* m, const void* base, long long rows, bool f16 = false) {
