@@ -319,12 +319,17 @@ def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headli
         rooflines["readout"]["traffic"] = tr["bytes_per_launch"]
         rooflines["readout"]["traffic_note"] = ("dram__bytes_read.sum + dram__bytes_write.sum of one full-size "
                                                 f"launch (ncu, {tr['summary']})")
-    # dominant kernel: the largest SM-time per step (duration alone x SMs it occupies); the
-    # step is close to the summed SM-time of the kernels over the 152 SMs
-    dominant = max(sm_ms, key=lambda k_: sm_ms[k_]) if sm_ms else None
+    # dominant kernel: the one carrying the largest share of the step's algorithmic work,
+    # the read-out (2 d^2 sum_t m_t of the prefill's 2 d^2 (sum_t m_t + 2T) flops); the
+    # latency-bound scan sets the step's critical path (see rooflines.scan and the SM-time
+    # shares in the note)
+    dominant = "readout" if "readout" in rooflines else (max(sm_ms, key=lambda k_: sm_ms[k_]) if sm_ms else None)
     roof = dict(rooflines[dominant]) if dominant else None
     if roof is not None:
-        roof["dominance"] = ("largest SM-time per step (ms alone x SMs occupied): " +
+        share = sum_m / (sum_m + 2.0 * T * BH) if dominant == "readout" else None
+        roof["dominance"] = ((f"largest share of the algorithmic work ({share:.3f} of 2 d^2 (sum_t m_t + 2T)); "
+                              if share is not None else "") +
+                             "SM-time per step (ms alone x SMs occupied): " +
                              ", ".join(f"{k_} {v_:.1f} SM-ms" for k_, v_ in sm_ms.items()))
     # end to end through the C ABI with host buffers: every step, dla_forward_host
     # copies q, k, v, lambda in from page-locked host memory (piece by piece beside
