@@ -763,11 +763,11 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   sa.row_start = row_start;
   const bool in_bf16 = (in_dtype == DLA_BF16);
   const bool tc = use_tc(in_dtype, d);
-  const bool pool_bf16 = tc;
+  const bool pool_f16 = tc;  // fp16 pool entries for the tensor-core read-out, else fp32
   if (!with_output) {
     sa.t_begin = 0; sa.t_end = T;
     sa.pool = nullptr; sa.pool_cap = 0; sa.nsnap = 1; sa.snap_chunks = 1;
-    e = timed(DLA_K_SCAN, st, [&] { return (in_bf16 ? dla::launch_scan_mma(sa, d, pool_bf16, st) : dla::launch_scan(sa, d, false, pool_bf16, st)); });
+    e = timed(DLA_K_SCAN, st, [&] { return (in_bf16 ? dla::launch_scan_mma(sa, d, pool_f16, st) : dla::launch_scan(sa, d, st)); });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     return ok();
   }
@@ -807,7 +807,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
   // its per-chunk chain is bound by the latency of small tensor-core groups).
   const bool scan_tc = tc && C <= dla::kMaxC && P.gram_chunks > 0 && !seq_lens && !stream_in && scan_tc_requested();
   auto launch_main_scan = [&](cudaStream_t s_) -> cudaError_t {
-    return scan_tc ? dla::launch_scan_tc(sa, s_) : dla::launch_scan_mma(sa, d, pool_bf16, s_);
+    return scan_tc ? dla::launch_scan_tc(sa, s_) : dla::launch_scan_mma(sa, d, pool_f16, s_);
   };
   const int gram_per_sm = scan_tc ? dla::kGramTcCtasPerSm : dla::kGramCtasPerSm;
   // Round r: the scan (high-priority stream) appends to the pool, then the
@@ -1050,7 +1050,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     if (r == 1 && gram_rest && (e = cudaStreamWaitEvent(S->hi, S->gram_done, 0)) != cudaSuccess)
       return cuda_fail(e, "stream wait");
     e = timed(DLA_K_SCAN, S->hi, [&] {
-      return in_bf16 ? launch_main_scan(S->hi) : dla::launch_scan(sa, d, false, pool_bf16, S->hi);
+      return in_bf16 ? launch_main_scan(S->hi) : dla::launch_scan(sa, d, S->hi);
     });
     if (e != cudaSuccess) return cuda_fail(e, "scan launch");
     if ((e = cudaEventRecord(S->scan_done[r % 2], S->hi)) != cudaSuccess) return cuda_fail(e, "event record");
@@ -1058,7 +1058,7 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     ra.t_begin = t0; ra.t_end = t1; ra.nsnap = sa.nsnap;
     e = timed(DLA_K_READOUT, S->lo, [&] {
       return tc ? dla::launch_readout_tc(ra, status, S->lo)
-                : dla::launch_readout_simt(ra, d, in_bf16, pool_bf16, S->lo);
+                : dla::launch_readout_simt(ra, d, in_bf16, S->lo);
     });
     if (e != cudaSuccess) return cuda_fail(e, "readout launch");
     if ((e = cudaEventRecord(S->ro_done[bsel], S->lo)) != cudaSuccess) return cuda_fail(e, "event record");

@@ -235,9 +235,10 @@ cudaError_t launch_varlen_rows(const int32_t* cu, int B, int T, long long total,
 // returns s (for entry points defined outside dla_api.cu).
 dla_status set_error(dla_status s, const char* fmt, ...);
 
-cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
+// K1 on CUDA cores for fp32 inputs (dla_scan.cu), fp32 pool entries.
+cudaError_t launch_scan(const ScanArgs& a, int d, cudaStream_t s);
 // K1 for bf16 inputs with its contractions on mma.sync (dla_scan_mma.cu).
-cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s);
+cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_f16, cudaStream_t s);
 // CTAs per stream of launch_scan_mma: 2 (a CTA pair) when 2*B*H CTAs fit the
 // device's SMs in one wave with d = 128, else 1.
 int scan_mma_ctas_per_stream(int BH, int d);
@@ -268,7 +269,7 @@ cudaError_t launch_scan_tc(const ScanArgs& a, cudaStream_t s);
 int scan_tc_resident_streams();
 cudaError_t preload_scan_tc_kernel();
 size_t scan_smem_bytes(int d);
-cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s);
+cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, cudaStream_t s);
 constexpr int kReadoutSimtInterval = 64;
 // K2 for bf16 inputs, d = 128, 128-token intervals (tcgen05 / TMEM / TMA,
 // snapshots stored as bf16 hi + lo): one CTA per pair of intervals computes the

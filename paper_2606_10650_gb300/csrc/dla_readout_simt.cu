@@ -232,15 +232,14 @@ static cudaError_t launch_ro_o(const ReadoutArgs& a, cudaStream_t st) {
   return a.out_bf16 ? launch_ro_t<D, Tin, Tpool, __nv_bfloat16>(a, st) : launch_ro_t<D, Tin, Tpool, float>(a, st);
 }
 
+// fp32 pool entries (the scans of the configurations this read-out serves write them)
 template <int D>
-static cudaError_t launch_ro_d(const ReadoutArgs& a, bool in_bf16, bool pool_bf16, cudaStream_t st) {
-  if (in_bf16) return pool_bf16 ? launch_ro_o<D, __nv_bfloat16, __nv_bfloat16>(a, st)
-                                : launch_ro_o<D, __nv_bfloat16, float>(a, st);
-  return pool_bf16 ? launch_ro_o<D, float, __nv_bfloat16>(a, st) : launch_ro_o<D, float, float>(a, st);
+static cudaError_t launch_ro_d(const ReadoutArgs& a, bool in_bf16, cudaStream_t st) {
+  return in_bf16 ? launch_ro_o<D, __nv_bfloat16, float>(a, st) : launch_ro_o<D, float, float>(a, st);
 }
 
-cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t st) {
-  return d == 128 ? launch_ro_d<128>(a, in_bf16, pool_bf16, st) : launch_ro_d<64>(a, in_bf16, pool_bf16, st);
+cudaError_t launch_readout_simt(const ReadoutArgs& a, int d, bool in_bf16, cudaStream_t st) {
+  return d == 128 ? launch_ro_d<128>(a, in_bf16, st) : launch_ro_d<64>(a, in_bf16, st);
 }
 
 }  // namespace dla

@@ -93,25 +93,11 @@ __device__ __forceinline__ void prefetch_kv(__nv_bfloat16* dk, __nv_bfloat16* dv
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
-// Copies a D x D fp32 state into a pool entry.  An fp32 pool keeps the value;
-// a bf16 pool stores it as two bf16 matrices hi = bf16(S) and lo = bf16(S - hi)
-// (entry = [hi | lo]), so two bf16 tensor-core products reproduce S q to ~2^-17.
+// Copies a D x D fp32 state into an fp32 pool entry.
 template <int D>
 __device__ __forceinline__ void copy_state(float* dst, const float* src) {
   for (int e = threadIdx.x * 4; e < D * D; e += NT * 4) store4(dst + e, load4(src + e));
 }
-template <int D>
-__device__ __forceinline__ void copy_state(__nv_bfloat16* dst, const float* src) {
-  for (int e = threadIdx.x * 4; e < D * D; e += NT * 4) {
-    const float4 x = load4(src + e);
-    const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
-    const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
-    store4(dst + e, make_float4(f01.x, f01.y, f23.x, f23.y));
-    store4(dst + D * D + e, make_float4(x.x - f01.x, x.y - f01.y, x.z - f23.x, x.w - f23.y));
-  }
-}
-template <typename Tpool>
-constexpr int pool_parts() { return sizeof(Tpool) == 2 ? 2 : 1; }
 
 }  // namespace
 
@@ -133,7 +119,7 @@ __global__ void __launch_bounds__(NT, 1) scan_kernel(ScanArgs a) {
   const Tin* vbase = reinterpret_cast<const Tin*>(a.v) + (tok0 * a.H + h) * D;
   const int row_stride = a.H * D;
   float* states = a.states + (long long)bh * C * D * D;
-  constexpr long long kEntry = (long long)pool_parts<Tpool>() * D * D;  // elements per pool entry
+  constexpr long long kEntry = (long long)D * D;  // elements per pool entry
   Tpool* pool = a.pool ? reinterpret_cast<Tpool*>(a.pool) + (long long)bh * a.pool_cap * kEntry : nullptr;
   uint8_t* bnd_out = a.boundary + (long long)bh * a.T;
   int32_t* mlog_out = a.merge_log + (long long)bh * a.T;
@@ -608,15 +594,8 @@ static cudaError_t launch_scan_t(const ScanArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_scan(const ScanArgs& a, int d, bool in_bf16, bool pool_bf16, cudaStream_t s) {
-  if (d == 128) {
-    if (in_bf16) return pool_bf16 ? launch_scan_t<128, __nv_bfloat16, __nv_bfloat16>(a, s)
-                                  : launch_scan_t<128, __nv_bfloat16, float>(a, s);
-    return pool_bf16 ? launch_scan_t<128, float, __nv_bfloat16>(a, s) : launch_scan_t<128, float, float>(a, s);
-  }
-  if (in_bf16) return pool_bf16 ? launch_scan_t<64, __nv_bfloat16, __nv_bfloat16>(a, s)
-                                : launch_scan_t<64, __nv_bfloat16, float>(a, s);
-  return pool_bf16 ? launch_scan_t<64, float, __nv_bfloat16>(a, s) : launch_scan_t<64, float, float>(a, s);
+cudaError_t launch_scan(const ScanArgs& a, int d, cudaStream_t s) {
+  return d == 128 ? launch_scan_t<128, float, float>(a, s) : launch_scan_t<64, float, float>(a, s);
 }
 
 size_t scan_smem_bytes(int d) { return d == 128 ? sizeof(ScanSmem<128>) : sizeof(ScanSmem<64>); }

@@ -1670,18 +1670,18 @@ cudaError_t launch_gate(const int32_t* started, int n, int32_t* status, cudaStre
   return cudaGetLastError();
 }
 
-cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_bf16, cudaStream_t s) {
+cudaError_t launch_scan_mma(const ScanArgs& a, int d, bool pool_f16, cudaStream_t s) {
   if (a.C > kMaxC) {  // DLA(I): bf16 inputs, d = 128, whole rows
-    if (d != 128 || !pool_bf16 || a.C > kMaxCBig || a.seq_lens) return cudaErrorInvalidValue;
+    if (d != 128 || !pool_f16 || a.C > kMaxCBig || a.seq_lens) return cudaErrorInvalidValue;
     return use_pairs(a) ? launch_scan_mma_r<128, __half, 2, false, kMaxCBig>(a, s)
                         : launch_scan_mma_r<128, __half, 1, false, kMaxCBig>(a, s);
   }
   if (d == 128) {
     if (use_pairs(a))
-      return pool_bf16 ? launch_scan_mma_t<128, __half, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);
-    return pool_bf16 ? launch_scan_mma_t<128, __half, 1>(a, s) : launch_scan_mma_t<128, float, 1>(a, s);
+      return pool_f16 ? launch_scan_mma_t<128, __half, 2>(a, s) : launch_scan_mma_t<128, float, 2>(a, s);
+    return pool_f16 ? launch_scan_mma_t<128, __half, 1>(a, s) : launch_scan_mma_t<128, float, 1>(a, s);
   }
-  return pool_bf16 ? launch_scan_mma_t<64, __half, 1>(a, s) : launch_scan_mma_t<64, float, 1>(a, s);
+  return pool_f16 ? launch_scan_mma_t<64, __half, 1>(a, s) : launch_scan_mma_t<64, float, 1>(a, s);
 }
 
 }  // namespace dla
