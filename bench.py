@@ -144,6 +144,101 @@ def kernel_table(timing, steps):
 
 # ---------------------------------------------------------------- prefill
 
+_INPUTS = {}  # device inputs of the headline workload: (workload, q, k, v, lambda)
+
+
+def bench_backward(args, dist, pk, steps=3, warmup=2):
+    """dla_backward on the headline workload's inputs and decisions: dQ, dK, dV
+    and dlambda of the read-out for a seeded upstream gradient, timed with CUDA
+    events; the device status is checked."""
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+
+    w, qt, kt, vt, lt = _INPUTS[args.workload]
+    B, T, H, d = kt.shape
+    fwd = dla.forward(qt, kt, vt, lt, tau=w.tau, capacity=w.C, eps=w.eps, rms_eps=w.rms_eps)
+    g = torch.randn((B, T, H, d), dtype=torch.float32, device=kt.device,
+                    generator=torch.Generator(device=kt.device).manual_seed(11))
+    del fwd["o"]
+
+    def step():
+        return dla.backward(qt, kt, vt, lt, fwd["boundary"], fwd["merge_log"], g, capacity=w.C)
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    if dla.dla_sync_status() != 0:
+        raise RuntimeError("backward: device status reports a failure")
+    dla.dla_timing_read(reset=True)
+    dla.dla_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        out = step()
+    e1.record()
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(False)
+    if dla.dla_sync_status() != 0:
+        raise RuntimeError("backward: device status reports a failure in the timed steps")
+    launches = sum(v_[0] for v_ in dla.dla_timing_read(reset=True).values())
+    ms = e0.elapsed_time(e1) / steps
+    del out
+    # five d-long contractions per token pair s <= t: q_t.k_s, g_t.v_s and the
+    # three weighted gradient products (dq, dk, dv)
+    algorithmic = 10.0 * d * (T * (T + 1) / 2) * B * H
+    return {"workload": f"{w.name}: B={B} H={H} T={T} d={d} C={w.C}, decisions of a forward call, "
+                        "upstream gradient N(0, 1)",
+            "value": round(B * T / ms * 1e3, 1), "unit": "tokens/s", "ms_per_step": round(ms, 3), "steps": steps,
+            "outputs": "dQ, dK, dV [B, T, H, d] and dlambda [B, T, H, C], fp32",
+            "algorithmic_tflops": round(algorithmic / (ms * 1e-3) / 1e12, 2),
+            "algorithmic_flops": "10*d*T(T+1)/2*B*H (five d-long contractions per token pair s <= t)",
+            "note": "quadratic in T per stream (every token pair s <= t, 64 x 64 tiles on mma.sync)",
+            "gpu_launches": launches}
+
+
+def bench_dla_i(args, dist, pk, capacity=128, steps=5, warmup=3):
+    """DLA(I) (dynamic merging without the capacity bound) on the headline
+    workload's inputs: capacity 128 lies above every stream's segment count, so
+    no capacity merge occurs; the device status and the absence of merges are
+    checked."""
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+
+    w, qt, kt, vt, lt0 = _INPUTS[args.workload]
+    B, T, H, d = kt.shape
+    lt = torch.ones((B, T, H, capacity), dtype=torch.float32, device=kt.device)
+    lt[..., : w.C] = lt0
+
+    def step():
+        return dla.forward(qt, kt, vt, lt, tau=w.tau, capacity=capacity, eps=w.eps, rms_eps=w.rms_eps)
+
+    for _ in range(warmup):
+        r = step()
+    torch.cuda.synchronize()
+    if dla.dla_sync_status() != 0 or int((r["merge_log"] >= 0).sum().item()) != 0:
+        raise RuntimeError("DLA(I): a device failure or a capacity merge")
+    dla.dla_timing_read(reset=True)
+    dla.dla_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        r = step()
+    e1.record()
+    torch.cuda.synchronize()
+    dla.dla_timing_enable(False)
+    if dla.dla_sync_status() != 0:
+        raise RuntimeError("DLA(I): device status reports a failure in the timed steps")
+    launches = sum(v_[0] for v_ in dla.dla_timing_read(reset=True).values())
+    ms = e0.elapsed_time(e1) / steps
+    seg = r["boundary"].sum(dim=2)
+    return {"workload": f"{w.name}: B={B} H={H} T={T} d={d}, capacity {capacity} (DLA(I): no capacity merge)",
+            "value": round(B * T / ms * 1e3, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4), "steps": steps,
+            "segments_per_stream": {"min": int(seg.min()), "max": int(seg.max()), "mean": round(float(seg.float().mean()), 1)},
+            "merges": 0, "gpu_launches": launches}
+
+
 def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headline=True):
     """One workload's prefill: warm-up, `steps` timed dla_forward calls (the
     default concurrent schedule), the call's device status checked, the kernels
@@ -166,6 +261,8 @@ def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headli
     qt, kt, vt = (W.to_device(x, w.dtype, dev) for x in (q, k, v))
     lt = torch.from_numpy(lam).to(dev)
     del q, k, v, lam
+    if headline:
+        _INPUTS[workload] = (w, qt, kt, vt, lt)  # reused by the backward and DLA(I) lines
     B, T, H, d = kt.shape
     p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
     in_code = dla.DLA_BF16 if w.dtype == "bf16" else dla.DLA_F32
@@ -616,6 +713,19 @@ def main():
             others[name]["value"] = round(others[name]["value"], 1)
             others[name]["unit"] = "tokens/s"
             others[name]["algorithmic_frac_of_peak"] = round(r["algorithmic_tflops"] / pk["bf16"], 4)
+    extra = {}
+    if pre and pre["tc_path"] and not args.no_configs and args.workload in _INPUTS:
+        for key, fn in (("backward", bench_backward), ("dla_i", bench_dla_i)):
+            try:
+                extra[key] = fn(args, dist, pk)
+            except (RuntimeError, MemoryError) as exc:  # reported in the line; the headline stands
+                extra[key] = {"error": str(exc)}
+                import torch
+
+                from paper_2606_10650_gb300 import dla
+                torch.cuda.synchronize()
+                dla.dla_sync_status()
+    _INPUTS.clear()
     dec = None if args.no_decode else bench_decode(args, dist, pk)
     cpu = cpu_baseline(args) if (dist.rank == 0 and dist.world == 1 and not args.no_cpu) else None
     if dist.rank == 0:
@@ -634,6 +744,8 @@ def main():
                         trace={"sum_m": pre["sum_m"], "boundaries": pre["boundaries"], "merges": pre["merges"]})
         if others:
             line["other_prefill_workloads"] = others
+        if extra:
+            line.update(extra)
         if dec:
             line["decode"] = dec
         line["cpu_baseline"] = cpu
