@@ -952,8 +952,8 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     ra.pool_scale = sa.pool_scale;
     ra.progress = progress; ra.progress_ctas = ctas; ra.status = status;
     // the read-out follows the pre-pass on the read-out stream: one launch over
-    // the whole sequence, its CTAs dispatched interval pair by interval pair
-    // (streams fastest), each waiting for its stream's progress
+    // the whole sequence, its CTAs dispatched interval by interval (streams
+    // fastest), each waiting for its stream's progress
     ra.t_begin = 0; ra.t_end = T;
     ra.nsnap = P.nsnap_total; ra.snap_base = 0;
     // Streamed output: pieces of opp interval pairs, each copied back once its
@@ -974,7 +974,9 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
       const int tp = 2 * P.interval;  // tokens per interval pair
       for (int op = 0; op < nop; ++op) {
         const int p0 = op * opp, p1 = std::min(npairs, p0 + opp);
-        if (wait_value_fn()((CUstream)S->cpo, (CUdeviceptr)(out_done + op), (cuuint32_t)(B * H * (p1 - p0)), 0) !=
+        // one read-out CTA per (interval, stream): the piece's intervals
+        const int nint = std::min(P.nsnap_total, 2 * p1) - 2 * p0;
+        if (wait_value_fn()((CUstream)S->cpo, (CUdeviceptr)(out_done + op), (cuuint32_t)(B * H * nint), 0) !=
             CUDA_SUCCESS)
           return fail(DLA_ERR_CUDA, "stream memory wait failed");
         const int t0 = p0 * tp, t1 = std::min(T, p1 * tp);

@@ -159,8 +159,9 @@ struct ReadoutArgs {
   const int32_t* progress;  // [B*H][2] scan progress to wait for (the scan runs concurrently), or nullptr
   int progress_ctas;        // scan CTAs per stream (1 or 2): entries of progress[bh] that count
   // Output copied back piece by piece while the read-out runs (tensor-core
-  // read-out), or nullptr: every CTA adds 1 to out_done[pair / out_piece_pairs]
-  // once its rows of o are stored (after a device-scope fence)
+  // read-out), or nullptr: every CTA (one per interval and stream) adds 1 to
+  // out_done[(interval / 2) / out_piece_pairs] once its rows of o are stored
+  // (after a device-scope fence)
   int32_t* out_done;
   int out_piece_pairs;
   const int32_t* seq_lens;  // [B] tokens of each row (padding after them), or nullptr: T each

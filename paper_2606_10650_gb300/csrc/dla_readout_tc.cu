@@ -10,28 +10,36 @@
 // t.  The tokens of the interval itself belong to the entry opened by the last
 // boundary event at or before them (event 0: the snapshot's open entry).
 //
-// One CTA per (pair of consecutive intervals A, B, stream).  Consecutive
-// snapshot lists share most of their states (only entries that changed get new
-// pool entries), so the CTA loads the union of the two lists once and applies
-// each state to the tokens of both intervals: D_x^A = Q_A S_x^T and
-// D_x^B = Q_B S_x^T (M = 128 tokens each, N = 128, K = 128) in fp16: K1 stores
-// each snapshot as S_x / s_x in fp16 (s_x a power of two from a bound of
-// |S_x|_F, so that no element overflows and every element keeps 2^-12
-// relative rounding), and Q is converted in place to fp16 with a power-of-two
-// scale per row once the intra part has used it (exact: bf16 values fit fp16's
-// significand); the epilogue multiplies D_x by s_x and the row's inverse scale
-// together with lambda.  An interval's MMAs are skipped for a state that is
-// not in its list.  Before
-// the states, the intra part of each interval: P = Q K^T, Pt = P o W
-// (W_ts = lambda_{t, L_t(e(s))} for s <= t, else 0) written as bf16 over the K
-// tile, O = Pt V with V as loaded (an MN-major operand), which o starts from.
-// Roles: warp 0 issues TMA loads (the two Q, K and V tiles, then each union
-// state, 32 KB in fp16, through four 32 KB stages), warp 1
-// issues tcgen05.mma (one thread) into two TMEM buffers of two 128-column
-// accumulators (A, B), warps 2..17 read TMEM, weight by lambda and accumulate o
-// in registers (one token row, one interval and one 64-column half per thread;
-// warp w reads TMEM lane quadrant w % 4).  All waits are bounded (~2 s, then
-// an abort flag and status 5).
+// One CTA per (interval, stream), sized so that two CTAs share an SM (about
+// 110 KB of shared memory and 256 TMEM columns each): one CTA's fixed phases
+// (tables, the intra part, the output) run while the other's state products
+// keep the tensor core busy.  K1 stores each snapshot as S_x / s_x in fp16 (s_x
+// a power of two from a bound of |S_x|_F, so that no element overflows and
+// every element keeps 2^-12 relative rounding).  The weights are folded into
+// the A operand, so that the interval keeps one accumulator over all its
+// states: with q~_t = q_t 2^(14 - e_t) the row's fp16 image (exact: bf16 values
+// fit fp16's significand) and s_ref the largest s_x of the list,
+//   o_t = qinv_t s_ref sum_x A_x[t] . (S_x / s_x)[:, :],
+//   A_x[t] = fp16(lambda_{t, L_t(x)} (s_x / s_ref) q~_t),   qinv_t = 2^(e_t - 14),
+// one fp16 MMA chain (M = 128 tokens, N = 128, K = 128 per state) with A in
+// tensor memory.  A_x is formed in fp16 arithmetic (the weight rounded to fp16,
+// then the product): at most two roundings of 2^-11 relative each (plus fp16's
+// absolute spacing of 2^-24 for weights far below s_ref, i.e. states far
+// smaller than the largest), beside the entry's 2^-12.  The intra part comes
+// first and starts the same accumulator: P = Q K^T, Pt = P o W (W_ts =
+// lambda_{t, L_t(e(s))} for s <= t, else 0) scaled by 1 / (qinv_t s_ref) (a
+// power of two) and written as bf16 over the K tile, O = Pt V with V as loaded
+// (an MN-major operand).
+// Roles: warp 0 issues TMA loads (Q, K and V, then each state of the list, 32
+// KB in fp16, through three 32 KB stages); one thread of warp 1 issues
+// tcgen05.mma; warps 2..9 (one token row and one 64-wide half of q per thread;
+// warp w reads TMEM lane quadrant w % 4) form Pt and, per state, the A operand
+// in TMEM slot x % 2, and finally read the accumulator out.  An issuing thread
+// that waits on an mbarrier starves the tensor core, so the issuer takes one
+// wait (`ready`: the A operand written and the state's tile landed, signalled
+// by the epilogue warps) and one commit (the tile's stage, which also frees
+// the TMEM slot for the state two later) per state.  All waits are bounded
+// (~2 s, then an abort flag and status 5).
 #include "dla_common.cuh"
 #include "dla_sm100.cuh"
 #include "dla_tmap.h"
@@ -44,21 +52,24 @@ using namespace sm100;
 
 constexpr int L = 128;   // tokens per interval
 constexpr int D = 128;   // head dimension
-constexpr int NT = 576;   // 18 warps
-constexpr int NEPI = 16;  // epilogue warps
-constexpr int NHS = 4;   // shared-memory stages (32 KB: an fp16 state, a K / Pt tile or a V tile)
-constexpr int NBUF = 2;  // TMEM buffers (each: accumulator A, accumulator B)
-constexpr uint32_t kTmemCols = 512;
+constexpr int NT = 320;  // 10 warps
+constexpr int NEPI = 8;  // epilogue warps
+constexpr int NHS = 3;   // shared-memory stages (32 KB: Q, K then Pt, V, then states)
+// TMEM: P = Q K^T at columns 0..127 during the intra part, then the same
+// columns hold the weighted-Q A operands, two 64-column slots; the output
+// accumulator at 128..255 (Pt V, then every state product added).
+constexpr uint32_t kColO = 128;
+constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kTile = L * 128;  // one K-major 128B-swizzled tile: 128 rows x 64 bf16
 constexpr int kRows = L + 1;         // events 0 .. L of an interval
-// Slot tables of one interval, in one region: first the intra part's tab[e][i]
+// Slot tables of the interval, in one region: first the intra part's tab[e][i]
 // for the entry opened at event i <= e (row e at e (e + 1) / 2), later the
 // snapshot entries' slots tab[e][x] (row stride kMaxC).
 constexpr int kSnapTab = kRows * kMaxC;
 constexpr int kIntraTab = kRows * (kRows + 1) / 2;
 constexpr int kTabBytes = kSnapTab > kIntraTab ? kSnapTab : kIntraTab;
 
-struct Side {      // per interval of the pair
+struct Side {      // the interval's trace
   int evt[L];      // events (boundaries) at or before token t
   int mlog[L];     // merge indices
   uint8_t bnd[L];  // boundary flags
@@ -71,20 +82,17 @@ struct Side {      // per interval of the pair
 template <int CAPB>
 struct TcSmem {
   static constexpr bool kBig = CAPB > kMaxC;
-  static constexpr int MAXU = 2 * CAPB;  // union of two lists
-  uint8_t Q[2][2][kTile];      // [interval][k-half]: Q, the A operand                 64 KB
-  uint8_t hs[NHS][2][kTile];   // [stage][half]: K then Pt, V, then state parts         128 KB
-  unsigned char tab[2][kBig ? 16 : kTabBytes];
-  Side side[2];
-  int ids[2][CAPB];            // pool ids of the two lists
-  int uid[MAXU];               // union: pool id
-  int uxa[MAXU], uxb[MAXU];    // union: index in list A / list B, or -1
-  float uscale[MAXU];          // union: scale s_x of the fp16 entry (S_x / s_x is stored)
-  float qmax[2][2][L];         // [interval][k-half][row]: max |q| of the half row (Q's fp16 scales)
-  int logi[2][kRows];          // table-build scratch, per interval
-  int nu;                      // union size
-  uint64_t bar_q, bar_pt, bar_done;
-  uint64_t full[NHS], empty[NHS], acc_full[NBUF], acc_empty[NBUF];
+  uint8_t hs[NHS][2][kTile];   // [stage][k-half]: Q, K (then Pt), V; the states; finally the output   96 KB
+  unsigned char tab[kBig ? 16 : kTabBytes];
+  Side side;
+  int ids[CAPB];               // pool ids of the list
+  float uscale[CAPB];          // scale s_x of each entry (S_x / s_x is stored)
+  float qmax[2][L];            // [k-half][row]: max |q| of the half row (Q's fp16 scales)
+  int logi[kRows];             // table-build scratch
+  float sref;                  // the largest s_x of the list (1 if empty)
+  uint64_t full[NHS], empty[NHS];
+  uint64_t bar_p, bar_pt, bar_done;
+  uint64_t ready[2];           // state x: its A operand in slot x % 2 and its tile landed
   uint32_t tmem_base;
   int abort_flag;
   int skip;                    // the call has failed before this CTA's work: do none of it
@@ -165,15 +173,17 @@ __device__ __forceinline__ int events_before(const Side& sd, int tt, int lane) {
   return e;
 }
 
+
 }  // namespace
 
-// 18 warps: the sub-partitions holding five of them bound a thread to 96 registers.
+// Two CTAs per SM: 20 warps share the four sub-partitions, so a thread gets at
+// most 96 registers.
 // kStream: inputs streamed in by the host while the kernel runs (lambda read
 // through L2) and the output copied back piece by piece (per-piece CTA counts).
 // kRagged: per-row lengths (padding after them).  Separate instances, so the
 // common one keeps its code unchanged.
 template <bool kStream, bool kRagged, int CAPB = kMaxC>
-__global__ void __launch_bounds__(NT, 1)
+__global__ void __launch_bounds__(NT, 2)
     readout_tc_kernel(ReadoutArgs a, const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmS,
                       const __grid_constant__ CUtensorMap tmO, int32_t* status) {
@@ -182,10 +192,18 @@ __global__ void __launch_bounds__(NT, 1)
   constexpr bool kBig = Smem::kBig;
   Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int bh = blockIdx.x, pair = blockIdx.y;  // streams fastest: CTAs dispatched interval pair by pair
+  const int bh = blockIdx.x, si = blockIdx.y;  // streams fastest: CTAs dispatched interval by interval
   const int b = bh / a.H, h = bh % a.H;
   const int C = a.C;
-  const int sA = 2 * pair;
+  // Streamed output: each CTA counts in the piece of its interval pair
+  auto count_done = [&](bool fence) {
+    if constexpr (kStream) {
+      if (a.out_done && tid == 0) {
+        if (fence) __threadfence();
+        atomicAdd(a.out_done + (si / 2) / a.out_piece_pairs, 1);
+      }
+    }
+  };
   // token row of the row's token 0, and the TMA coordinates of it: (token, batch)
   // = (t, b) in the padded layout, (row_start[b] + t, 0) in the packed one (the
   // per-row-length instance only)
@@ -194,183 +212,123 @@ __global__ void __launch_bounds__(NT, 1)
   const int tma_t = packed ? (int)tok0 : 0, tma_b = packed ? 0 : b;
   // this row's end (padding after it)
   const int t_end = kRagged ? row_t_end(a.seq_lens, b, a.t_begin, a.t_end) : a.t_end;
+  const int c0 = a.t_begin + si * L;
   if constexpr (kRagged) {
-    if (a.t_begin + sA * L >= t_end) {  // the pair lies past the row's length: o not written
-      if constexpr (kStream) {
-        if (a.out_done && tid == 0) atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
-      }
+    if (c0 >= t_end) {  // the interval lies past the row's length: o not written
+      count_done(false);
       return;
     }
   }
-  const bool hasB = (sA + 1) < a.nsnap && (!kRagged || a.t_begin + (sA + 1) * L < t_end);
-  // with a scan running concurrently: both intervals of the pair must be complete
-  wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + sA + (hasB ? 2 : 1), a.status);
+  // with a scan running concurrently: the interval must be complete
+  wait_progress(a.progress, a.progress_ctas, bh, a.snap_base + si + 1, a.status);
   if (tid == 0) {
     // thread 0 issues the TMA loads: they read what the scan wrote (pool entries)
     // and the inputs streamed in before its progress
     if (a.progress) asm volatile("fence.proxy.async.global;" ::: "memory");
     // A failed call (a bounded wait that gave up, here or in another kernel, or a
-    // device check): the scan may not have written this pair's lists, so the
+    // device check): the scan may not have written this interval's list, so the
     // CTA does none of the work and leaves o unwritten.
     sm.skip = (*(volatile int32_t*)a.status != 0);
   }
   __syncthreads();
   if (sm.skip) {
-    if constexpr (kStream) {
-      if (a.out_done && tid == 0) atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
-    }
+    count_done(false);
     return;
   }
-  // interval A (side 0) and B (side 1) of the pair
-  const int c0A = a.t_begin + sA * L, c0B = c0A + L;
-  const int LcA = min(L, t_end - c0A), LcB = hasB ? min(L, t_end - c0B) : 0;
-  const long long lrowA = (long long)bh * a.snap_stride + a.snap_base + sA, lrowB = lrowA + 1;
-  // lists and trace come from the scan: read past L1 (__ldcg)
-  // live entries of the two lists, checked against the capacity (a violation is
-  // a device-check failure and is clamped, so that nothing indexes out of bounds)
-  int m0A = __ldcg(a.snap_m0 + lrowA), m0B = hasB ? __ldcg(a.snap_m0 + lrowB) : 0;
-  if (m0A < 0 || m0A > C || m0B < 0 || m0B > C) {
+  const int Lc = min(L, t_end - c0);
+  const long long lrow = (long long)bh * a.snap_stride + a.snap_base + si;
+  // list and trace come from the scan: read past L1 (__ldcg).  Live entries of
+  // the list, checked against the capacity (a violation is a device-check
+  // failure and is clamped, so that nothing indexes out of bounds)
+  int m0 = __ldcg(a.snap_m0 + lrow);
+  if (m0 < 0 || m0 > C) {
     if (tid == 0) atomicCAS(a.status, 0, 6);
-    m0A = min(max(m0A, 0), C);
-    m0B = min(max(m0B, 0), C);
+    m0 = min(max(m0, 0), C);
   }
-  auto c0_of = [&](int side) { return side ? c0B : c0A; };
-  auto Lc_of = [&](int side) { return side ? LcB : LcA; };
   volatile int* abort = &sm.abort_flag;
 
   if (tid == 0) {
-    mbar_init(&sm.bar_q, 1);
+    mbar_init(&sm.bar_p, 1);
     mbar_init(&sm.bar_pt, NEPI);
     mbar_init(&sm.bar_done, 1);
     for (int i = 0; i < NHS; ++i) {
       mbar_init(&sm.full[i], 1);
       mbar_init(&sm.empty[i], 1);
     }
-    for (int i = 0; i < NBUF; ++i) {
-      mbar_init(&sm.acc_full[i], 1);
-      mbar_init(&sm.acc_empty[i], NEPI);
-    }
+    for (int j = 0; j < 2; ++j) mbar_init(&sm.ready[j], NEPI);
     sm.abort_flag = 0;
     fence_mbar_init();
-    // the Q tiles go out first; they depend on nothing
     prefetch_tmap(&tmQ);
     prefetch_tmap(&tmK);
     prefetch_tmap(&tmV);
     prefetch_tmap(&tmS);
-    mbar_expect_tx(&sm.bar_q, (hasB ? 4 : 2) * kTile);
-    tma_load_4d(sm.Q[0][0], &tmQ, &sm.bar_q, 0, h, tma_t + c0A, tma_b);
-    tma_load_4d(sm.Q[0][1], &tmQ, &sm.bar_q, 64, h, tma_t + c0A, tma_b);
-    if (hasB) {
-      tma_load_4d(sm.Q[1][0], &tmQ, &sm.bar_q, 0, h, tma_t + c0B, tma_b);
-      tma_load_4d(sm.Q[1][1], &tmQ, &sm.bar_q, 64, h, tma_t + c0B, tma_b);
-    }
+    // units 0, 1, 2: the Q, K and V tiles, each in the stage of its number
+    auto load_unit = [&](int g, const CUtensorMap* map) {
+      mbar_expect_tx(&sm.full[g], 2 * kTile);
+      tma_load_4d(sm.hs[g][0], map, &sm.full[g], 0, h, tma_t + c0, tma_b);
+      tma_load_4d(sm.hs[g][1], map, &sm.full[g], 64, h, tma_t + c0, tma_b);
+    };
+    load_unit(0, &tmQ);
+    load_unit(1, &tmK);
+    load_unit(2, &tmV);
   }
-  for (int i = tid; i < 2 * CAPB; i += NT) {
-    const int side = i / CAPB, x = i % CAPB;
-    int id = (x < (side ? m0B : m0A)) ? __ldcg(a.snap_ids + (side ? lrowB : lrowA) * C + x) : -1;
-    if (x < (side ? m0B : m0A) && (id < 0 || id >= a.pool_cap)) {  // a pool id outside the pool
-      atomicCAS(a.status, 0, 6);
-      id = 0;
-    }
-    sm.ids[side][x] = id;
-  }
-  if (warp == 1) tmem_alloc(&sm.tmem_base, kTmemCols);
-  __syncthreads();
-  if (warp == 0) {
-    // union of the two lists: list A in order, then the entries of list B not in A
+  if (warp == 0) {  // pool ids and scales of the list, and s_ref
+    float smax = 0.f;
     for (int x = lane; x < CAPB; x += 32) {
-      if (x < m0A) {
-        sm.uid[x] = sm.ids[0][x];
-        sm.uxa[x] = x;
-        sm.uxb[x] = -1;
-      }
-    }
-    __syncwarp();
-    int nb_only = 0;
-    for (int base = 0; base < m0B; base += 32) {
-      const int x = base + lane;
-      int match = -1;
-      if (x < m0B) {
-        const int id = sm.ids[1][x];
-        for (int y = 0; y < m0A; ++y)
-          if (sm.ids[0][y] == id) match = y;
-      }
-      const unsigned only = __ballot_sync(0xffffffffu, x < m0B && match < 0);
-      if (x < m0B) {
-        if (match >= 0) {
-          sm.uxb[match] = x;
-        } else {
-          const int u = m0A + nb_only + __popc(only & ((1u << lane) - 1u));
-          sm.uid[u] = sm.ids[1][x];
-          sm.uxa[u] = -1;
-          sm.uxb[u] = x;
+      int id = -1;
+      float sc = 1.f;
+      if (x < m0) {
+        id = __ldcg(a.snap_ids + lrow * C + x);
+        if (id < 0 || id >= a.pool_cap) {  // a pool id outside the pool
+          atomicCAS(a.status, 0, 6);
+          id = 0;
         }
+        sc = __ldcg(a.pool_scale + (long long)bh * a.pool_cap + id);
+        smax = fmaxf(smax, sc);
       }
-      nb_only += __popc(only);
+      sm.ids[x] = id;
+      sm.uscale[x] = sc;
     }
-    if (lane == 0) sm.nu = m0A + nb_only;
-    __syncwarp();
-    const int nu_w = m0A + nb_only;
-    for (int u = lane; u < nu_w; u += 32) sm.uscale[u] = __ldcg(a.pool_scale + (long long)bh * a.pool_cap + sm.uid[u]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) smax = fmaxf(smax, __shfl_xor_sync(0xffffffffu, smax, off));
+    // the scales are powers of two, so s_x / s_ref is exact
+    if (lane == 0) sm.sref = smax > 0.f ? smax : 1.f;
+  } else if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+  } else if (tid - 64 < L) {  // the interval's boundary flags and merge indices
+    const int tt = tid - 64;
+    const bool in = tt < Lc;
+    const long long tr = (long long)bh * a.T + c0 + tt;
+    sm.side.bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
+    sm.side.mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const int nu = sm.nu;
-  // Ring units: g = 0, 1 the K tiles of intervals A and B (then Pt over them),
-  // g = 2, 3 their V tiles (the MN-major B operand of O), g = 4 + x union state
-  // x (fp16).  Unit g uses stage g % NHS for the (g / NHS)-th time.
-  // Accumulators (TMEM buffer n % NBUF): n = 0 P = Q K^T, n = 1 O = Pt V,
-  // n = 2 + x union state x.
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int issued[NHS];  // uses of each stage so far
-      mbar_expect_tx(&sm.full[0], 2 * kTile);
-      tma_load_4d(sm.hs[0][0], &tmK, &sm.full[0], 0, h, tma_t + c0A, tma_b);
-      tma_load_4d(sm.hs[0][1], &tmK, &sm.full[0], 64, h, tma_t + c0A, tma_b);
-      mbar_expect_tx(&sm.full[2], 2 * kTile);
-      tma_load_4d(sm.hs[2][0], &tmV, &sm.full[2], 0, h, tma_t + c0A, tma_b);
-      tma_load_4d(sm.hs[2][1], &tmV, &sm.full[2], 64, h, tma_t + c0A, tma_b);
-      if (hasB) {
-        mbar_expect_tx(&sm.full[1], 2 * kTile);
-        tma_load_4d(sm.hs[1][0], &tmK, &sm.full[1], 0, h, tma_t + c0B, tma_b);
-        tma_load_4d(sm.hs[1][1], &tmK, &sm.full[1], 64, h, tma_t + c0B, tma_b);
-        mbar_expect_tx(&sm.full[3], 2 * kTile);
-        tma_load_4d(sm.hs[3][0], &tmV, &sm.full[3], 0, h, tma_t + c0B, tma_b);
-        tma_load_4d(sm.hs[3][1], &tmV, &sm.full[3], 64, h, tma_t + c0B, tma_b);
-      } else {  // first phase complete without data: the stages' later uses keep their parity
-        mbar_arrive(&sm.full[1]);
-        mbar_arrive(&sm.full[3]);
-      }
       for (int i = 0; i < NHS; ++i) issued[i] = 1;
-      for (int u = 0; u < nu; ++u) {
-        const int g = 4 + u, hsi = g % NHS, k = g / NHS;
+      for (int x = 0; x < m0; ++x) {
+        const int g = 3 + x, hsi = g % NHS, k = g / NHS;
         if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
-        const int row = (int)(((long long)bh * a.pool_cap + sm.uid[u]) * D);
+        const int row = (int)(((long long)bh * a.pool_cap + sm.ids[x]) * D);
         tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
         tma_load_2d(sm.hs[hsi][1], &tmS, &sm.full[hsi], 64, row);
         issued[hsi] = k + 1;
       }
       if (*abort) {  // let copies in flight land before the CTA exits
-        for (int i = 0; i < NHS; ++i)
-          if (issued[i] > 0) mbar_wait_drain(&sm.full[i], (uint32_t)((issued[i] - 1) & 1));
-        mbar_wait_drain(&sm.bar_q, 0);
+        for (int i = 0; i < NHS; ++i) mbar_wait_drain(&sm.full[i], (uint32_t)((issued[i] - 1) & 1));
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(L, D);
-      auto acc_acquire = [&](int n) -> bool {
-        const int buf = n % NBUF, kb = n / NBUF;
-        if (!mbar_wait(&sm.acc_empty[buf], (uint32_t)((kb & 1) ^ 1), abort, status)) return false;
-        tc_fence_after();
-        return true;
-      };
       auto unit_wait = [&](int g) -> bool {
         if (!mbar_wait(&sm.full[g % NHS], (uint32_t)((g / NHS) & 1), abort, status)) return false;
         tc_fence_after();
@@ -379,133 +337,146 @@ __global__ void __launch_bounds__(NT, 1)
       // Descriptors: a tile's descriptor plus (byte offset >> 4) addresses a
       // later part of it (shared-memory addresses stay below 2^18).  K step kk
       // of a K-major 128-row tile pair: k-half kk / 4, 32 bytes per step.
-      const uint64_t qd0 = desc_kmajor_sw128(smem_u32(sm.Q[0][0]));
-      const uint64_t qd1 = desc_kmajor_sw128(smem_u32(sm.Q[1][0]));
       const uint64_t hd0 = desc_kmajor_sw128(smem_u32(sm.hs[0][0]));
       constexpr uint64_t kStage = (2 * kTile) >> 4;
       auto kstep = [](int kk) -> uint64_t { return (uint64_t)((kk >> 2) * (kTile >> 4) + (kk & 3) * 2); };
-      bool ok = mbar_wait(&sm.bar_q, 0, abort, status) && unit_wait(0) && (!hasB || unit_wait(1));
-      if (ok) {  // P = Q K^T (accumulator 0; buffer 0 is fresh)
+      // A commit stands only behind MMAs of this thread: after a failed wait
+      // with none issued, the thread arrives on the barrier instead.
+      bool issued = false;
+      auto release = [&](uint64_t* bar) {
+        if (issued) mma_commit(bar);
+        else mbar_arrive(bar);
+      };
+      bool ok = unit_wait(0) && unit_wait(1);
+      if (ok) {  // P = Q K^T (columns 0..127): Q in stage 0, K in stage 1
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          mma_bf16(tmem, qd0 + kstep(kk), hd0 + kstep(kk), idesc, kk > 0);
-          if (hasB) mma_bf16(tmem + 128u, qd1 + kstep(kk), hd0 + kStage + kstep(kk), idesc, kk > 0);
-        }
-        mma_commit(&sm.acc_full[0]);
+        for (int kk = 0; kk < 8; ++kk) mma_bf16(tmem, hd0 + kstep(kk), hd0 + kStage + kstep(kk), idesc, kk > 0);
+        issued = true;
+        mma_commit(&sm.bar_p);
       }
-      // O = Pt V (accumulator 1; buffer 1 is fresh): Pt over the K tiles
-      // (stages 0, 1, written by the epilogue), V in stages 2, 3 as loaded:
-      // [s][j], the MN-major B operand (K step: 16 rows of 128 bytes)
-      if (ok && (ok = mbar_wait(&sm.bar_pt, 0, abort, status)) && (ok = unit_wait(2)) && (!hasB || (ok = unit_wait(3)))) {
+      // O = Pt V (columns 128..255): Pt over the K tile (stage 1, written by the
+      // epilogue), V in stage 2 as loaded: [s][j], the MN-major B operand (K
+      // step: 16 rows of 128 bytes)
+      if (ok && (ok = mbar_wait(&sm.bar_pt, 0, abort, status)) && (ok = unit_wait(2))) {
         constexpr uint32_t idesc_v = idesc_bf16_f32_bmn(L, D);
-        const uint64_t vd0 = desc_mnmajor_sw128(smem_u32(sm.hs[2][0]), kTile);
-        const uint64_t vd1 = desc_mnmajor_sw128(smem_u32(sm.hs[3][0]), kTile);
+        const uint64_t vd = desc_mnmajor_sw128(smem_u32(sm.hs[2][0]), kTile);
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          mma_bf16(tmem + 256u, hd0 + kstep(kk), vd0 + (uint64_t)(kk * (2048 >> 4)), idesc_v, kk > 0);
-          if (hasB) mma_bf16(tmem + 384u, hd0 + kStage + kstep(kk), vd1 + (uint64_t)(kk * (2048 >> 4)), idesc_v, kk > 0);
-        }
-        mma_commit(&sm.acc_full[1]);
+        for (int kk = 0; kk < 8; ++kk)
+          mma_bf16(tmem + kColO, hd0 + kStage + kstep(kk), vd + (uint64_t)(kk * (2048 >> 4)), idesc_v, kk > 0);
       }
-      for (int i = 0; i < NHS; ++i) mma_commit(&sm.empty[i]);  // every stage is free once O is done
-      // the state products, fp16 Q (converted by the epilogue before bar_pt) and fp16 states
+      for (int i = 0; i < NHS; ++i) release(&sm.empty[i]);  // every stage is free once O is done
+      // The state products, added to O: A = the weighted fp16 Q (TMEM slot
+      // x % 2, written by the epilogue: one row per lane, two fp16 per column,
+      // K step 8 columns), B = the fp16 state (shared memory).
       constexpr uint32_t idesc_h = idesc_f16_f32(L, D);
-      for (int x = 0; ok && x < nu; ++x) {
-        const int buf = x % NBUF;
-        const bool inA = sm.uxa[x] >= 0, inB = hasB && sm.uxb[x] >= 0;
-        if (!(ok = acc_acquire(x + 2))) break;
-        const uint32_t dA = tmem + 256u * buf, dB = dA + 128u;
-        const int g = 4 + x, hsi = g % NHS;
-        if (!(ok = unit_wait(g))) break;
+      for (int x = 0; ok && x < m0; ++x) {
+        const int j = x & 1, hsi = (3 + x) % NHS;
+        if (!(ok = mbar_wait(&sm.ready[j], (uint32_t)((x >> 1) & 1), abort, status))) break;
+        tc_fence_after();
         const uint64_t bd = hd0 + (uint64_t)hsi * kStage;
-        if (inA && inB) {
+        const uint32_t ad = tmem + 64u * j;
 #pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            mma_bf16(dA, qd0 + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
-            mma_bf16(dB, qd1 + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
-          }
-        } else if (inA || inB) {
-          const uint32_t dd = inA ? dA : dB;
-          const uint64_t qd = inA ? qd0 : qd1;
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) mma_bf16(dd, qd + kstep(kk), bd + kstep(kk), idesc_h, kk > 0);
-        }
-        mma_commit(&sm.empty[hsi]);
-        mma_commit(&sm.acc_full[buf]);
+        for (int kk = 0; kk < 8; ++kk) mma_ts(tmem + kColO, ad + 8u * kk, bd + kstep(kk), idesc_h, 1u);
+        mma_commit(&sm.empty[hsi]);  // the tile's stage, and TMEM slot j for state x + 2
       }
-      mma_commit(&sm.bar_done);  // every MMA issued above has completed once this fires
+      release(&sm.bar_done);  // every MMA issued above has completed once this fires
       mbar_wait_drain(&sm.bar_done, 0);
     }
   } else {
     // ------------------------------------------------------------ epilogue warps
-    // 16 warps: warp w reads TMEM lane quadrant w % 4; epilogue warp ew = w - 2
-    // owns interval (ew / 4) % 2 and the 64-column half ew / 8 of its rows.
-    const int ew = warp - 2;              // 0..15
+    // 8 warps: warp w reads TMEM lane quadrant w % 4; epilogue warp ew = w - 2
+    // owns the 64-column half ew / 4 of its token rows.
+    const int ew = warp - 2;              // 0..7
     const int quad = warp & 3;            // TMEM lane quadrant of this warp
-    const int side = (ew >> 2) & 1;       // interval A (0) or B (1)
-    const int ch = ew >> 3;               // column half
+    const int ch = ew >> 2;               // column half
     const int t = quad * 32 + lane;       // token row of this thread
     const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
-    const int etid = ew * 32 + lane;      // 0..511
-    const int c0s = c0_of(side), Lcs = Lc_of(side);
-    const bool side_in = (side == 0 || hasB);  // warp-uniform
-    const long long rowbase = (tok0 + c0s) * a.H + h;
-
-    if (etid < 2 * L) {  // both intervals' boundary flags and merge indices
-      const int sd = etid / L, tt = etid % L;
-      const bool in = tt < Lc_of(sd);
-      const long long tr = (long long)bh * a.T + c0_of(sd) + tt;
-      sm.side[sd].bnd[tt] = in ? __ldcg(a.boundary + tr) : (uint8_t)0;
-      sm.side[sd].mlog[tt] = in ? __ldcg(a.merge_log + tr) : -1;
-    }
-    asm volatile("bar.sync 1, 512;" ::: "memory");
+    const int etid = ew * 32 + lane;      // 0..255
+    const long long rowbase = (tok0 + c0) * a.H + h;
     if constexpr (!kBig) {
-      if (ew == 0) build_intra_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-      if (ew == 4 && hasB) build_intra_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+      if (ew == 0) build_intra_table(sm.side, sm.tab, sm.logi, m0, lane);
     }
-    if (etid < 2 * L) {
-      const int sd = etid / L, tt = etid % L;
-      sm.side[sd].evt[tt] = events_before(sm.side[sd], tt, lane);
-    }
-    asm volatile("bar.sync 1, 512;" ::: "memory");
-    const float* lam_t = (a.lam && t < Lcs) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
+    if (etid < L) sm.side.evt[etid] = events_before(sm.side, etid, lane);
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    const float* lam_t = (a.lam && t < Lc) ? a.lam + (rowbase + (long long)t * a.H) * C : nullptr;
     // lambda is read-only while the kernel runs (the read-only path), except when
     // the host streams it in beside the work (then through L2)
     auto lam_at = [&](int i) -> float {
       if constexpr (kStream) return __ldcg(lam_t + i);
       else return __ldg(lam_t + i);
     };
-    const int evt_t = sm.side[side].evt[t];
+    const int evt_t = sm.side.evt[t];
     // an interval without boundary events (the common case) weights every
     // column s <= t of row t by lambda of the open entry: loaded ahead of P
-    const bool no_ev = sm.side[side].evt[L - 1] == 0;  // warp-uniform
-    const int m0s = side ? m0B : m0A;
+    const bool no_ev = sm.side.evt[L - 1] == 0;  // warp-uniform
     // slot, after this row's events, of the entry opened at event e (0: the open entry)
     auto intra_slot = [&](const unsigned char* trow_, int e) -> int {
-      if constexpr (kBig) return min(m0s - 1 + e, C - 1);  // a consistent trace stays below C
+      if constexpr (kBig) return min(m0 - 1 + e, C - 1);  // a consistent trace stays below C
       else return trow_[e];
     };
-    const float w_open = (no_ev && t < Lcs) ? (lam_t ? lam_at(intra_slot(sm.tab[side], 0)) : 1.f) : 0.f;
-    bool ok;
-    {  // P (accumulator 0) -> Pt over this interval's K tile (its MMAs are complete)
-      ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[0], 0, abort, status));
-      if (ok && side_in) {
+    const float w_open = (no_ev && t < Lc) ? (lam_t ? lam_at(intra_slot(sm.tab, 0)) : 1.f) : 0.f;
+    // P = Q K^T is complete, so the Q and K tiles have landed
+    bool ok = __all_sync(0xffffffffu, mbar_wait(&sm.bar_p, 0, abort, status));
+    // This row's half of Q in fp16 registers: a power-of-two scale per row,
+    // agreed on by the two k-halves through qmax, keeps every element below
+    // 2^14 and in fp16's normal range (bf16 values fit fp16's significand, so
+    // only values below 2^-14 of the row's scale round); the output is
+    // multiplied back by its inverse, qinv.  Column c of the half row holds the
+    // elements 2c, 2c + 1 (the layout of an A operand in tensor memory).
+    uint32_t qh[32];
+    float qinv = 1.f, fpt = 1.f;
+    const float sref = sm.sref, rsref = 1.f / sref;  // powers of two
+    {
+      const uint8_t* qtile = sm.hs[0][ch];
+      float mx = 0.f;
+#pragma unroll
+      for (int c8 = 0; c8 < 8; ++c8) {
+        uint4 w = make_uint4(0u, 0u, 0u, 0u);
+        if (ok) w = *reinterpret_cast<const uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4));
+        qh[4 * c8] = w.x;
+        qh[4 * c8 + 1] = w.y;
+        qh[4 * c8 + 2] = w.z;
+        qh[4 * c8 + 3] = w.w;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qh[4 * c8 + i]));
+          mx = fmaxf(mx, fmaxf(fabsf(f.x), fabsf(f.y)));
+        }
+      }
+      sm.qmax[ch][t] = mx;
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      const float rm = fmaxf(sm.qmax[0][t], sm.qmax[1][t]);
+      int ex = 0;
+      if (rm > 0.f) frexpf(rm, &ex);  // rm < 2^ex
+      const float sc = ldexpf(1.f, 14 - ex);
+      qinv = ldexpf(1.f, ex - 14);
+      fpt = sc * rsref;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qh[i]));
+        const __half2 hh = __floats2half2_rn(f.x * sc, f.y * sc);
+        qh[i] = *reinterpret_cast<const uint32_t*>(&hh);
+      }
+    }
+    {  // P -> Pt over the K tile, in the accumulator's units: row t scaled by
+       // 2^(14 - ex) / s_ref (a power of two, so no extra rounding)
+      if (ok) {
         tc_fence_after();
-        const uint32_t base = lane_addr + 128u * side + 64 * ch;
+        const uint32_t base = lane_addr + 64 * ch;
         // the weight of column s depends on s only through evt[s], which changes
         // at the interval's boundaries: it is looked up again only then
-        const unsigned char* trow = kBig ? sm.tab[side] : sm.tab[side] + evt_t * (evt_t + 1) / 2;
-        const int* evs = sm.side[side].evt;
+        const unsigned char* trow = kBig ? sm.tab : sm.tab + evt_t * (evt_t + 1) / 2;
+        const int* evs = sm.side.evt;
         int last_e = -1;
         float last_w = 0.f;
-        uint8_t* ptile = sm.hs[side][ch];
+        uint8_t* ptile = sm.hs[1][ch];
 #pragma unroll
         for (int c = 0; c < 64; c += 16) {
           float p[16];
           tmem_ld16(base + c, p);
 #pragma unroll
           for (int h8 = 0; h8 < 2; ++h8) {
-            uint32_t packed[4];
+            uint32_t pk[4];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               float w2[2];
@@ -515,7 +486,7 @@ __global__ void __launch_bounds__(NT, 1)
                 float wt = 0.f;
                 if (no_ev) {
                   wt = (ss <= t) ? w_open : 0.f;
-                } else if (ss <= t && t < Lcs) {
+                } else if (ss <= t && t < Lc) {
                   const int e = evs[ss];
                   if (e != last_e) {
                     last_e = e;
@@ -523,156 +494,108 @@ __global__ void __launch_bounds__(NT, 1)
                   }
                   wt = last_w;
                 }
-                w2[u] = p[8 * h8 + 2 * i + u] * wt;
+                w2[u] = (p[8 * h8 + 2 * i + u] * wt) * fpt;
               }
               const __nv_bfloat162 pr = __floats2bfloat162_rn(w2[0], w2[1]);
-              packed[i] = *reinterpret_cast<const uint32_t*>(&pr);
+              pk[i] = *reinterpret_cast<const uint32_t*>(&pr);
             }
             const int c8 = (c >> 3) + h8;  // 16-byte chunk of the row
-            *reinterpret_cast<uint4*>(ptile + t * 128 + ((c8 ^ (t & 7)) << 4)) =
-                make_uint4(packed[0], packed[1], packed[2], packed[3]);
+            *reinterpret_cast<uint4*>(ptile + t * 128 + ((c8 ^ (t & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           }
         }
       }
-    }
-    // This row's half of Q into fp16 in place (the P MMAs, the only bf16 use of Q,
-    // are complete): a power-of-two scale per row, agreed on by the two k-halves
-    // through qmax, keeps every element below 2^14 and in fp16's normal range
-    // (bf16 values fit fp16's significand, so only values below 2^-14 of the
-    // row's scale round); the epilogue multiplies D by its inverse, qinv.
-    float qinv = 1.f;
-    {
-      uint8_t* qtile = sm.Q[side][ch];
-      const bool conv = ok && side_in;  // warp-uniform
-      float mx = 0.f;
-      if (conv) {
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          const uint4 w = *reinterpret_cast<const uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4));
-          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ws[i]));
-            mx = fmaxf(mx, fmaxf(fabsf(f.x), fabsf(f.y)));
-          }
-        }
-      }
-      sm.qmax[side][ch][t] = mx;
-      asm volatile("bar.sync 1, 512;" ::: "memory");
-      if (conv) {
-        const float rm = fmaxf(sm.qmax[side][0][t], sm.qmax[side][1][t]);
-        int ex = 0;
-        if (rm > 0.f) frexpf(rm, &ex);  // rm < 2^ex
-        const float sc = ldexpf(1.f, 14 - ex);
-        qinv = ldexpf(1.f, ex - 14);
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          uint4* ptr = reinterpret_cast<uint4*>(qtile + t * 128 + ((c8 ^ (t & 7)) << 4));
-          const uint4 w = *ptr;
-          uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ws[i]));
-            const __half2 hh = __floats2half2_rn(f.x * sc, f.y * sc);
-            ws[i] = *reinterpret_cast<const uint32_t*>(&hh);
-          }
-          *ptr = make_uint4(ws[0], ws[1], ws[2], ws[3]);
-        }
-      }
-      fence_proxy_async();  // the generic-proxy writes (Pt, fp16 Q) feed the tensor core
+      fence_proxy_async();  // the generic-proxy writes (Pt) feed the tensor core
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&sm.acc_empty[0]);
-        mbar_arrive(&sm.bar_pt);
-      }
+      if (lane == 0) mbar_arrive(&sm.bar_pt);
     }
-    asm volatile("bar.sync 1, 512;" ::: "memory");  // every warp is past the intra tables
+    asm volatile("bar.sync 1, 256;" ::: "memory");  // every warp is past the intra table and its P reads
     if constexpr (!kBig) {
-      if (ew == 0) build_snap_table(sm.side[0], sm.tab[0], sm.logi[0], m0A, lane);
-      if (ew == 4) build_snap_table(sm.side[1], sm.tab[1], sm.logi[1], m0B, lane);
+      if (ew == 0) build_snap_table(sm.side, sm.tab, sm.logi, m0, lane);
     }
-    asm volatile("bar.sync 1, 512;" ::: "memory");
-    float o[64];
-    {  // o starts from O (accumulator 1)
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[1], 0, abort, status));
-      if (ok && side_in) {
-        tc_fence_after();
-        const uint32_t base = lane_addr + 256u + 128u * side + 64 * ch;
-#pragma unroll
-        for (int c = 0; c < 64; c += 16) tmem_ld16(base + c, o + c);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 64; ++i) o[i] = 0.f;
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.acc_empty[1]);
-    }
-    const int* ux = side ? sm.uxb : sm.uxa;
-    {  // snapshot part
-      const unsigned char* tab_t = sm.tab[side] + (kBig ? 0 : evt_t * kMaxC);
-      // weight of union state x for this token (0 when not in its interval's list):
-      // lambda times the entry's scale s_x and the row's inverse Q scale
-      auto weight = [&](int x) -> float {
-        if (x >= nu || t >= Lcs) return 0.f;
-        const int xi = ux[x];
-        if (xi < 0) return 0.f;
-        return (lam_t ? lam_at(kBig ? xi : (int)tab_t[xi]) : 1.f) * sm.uscale[x] * qinv;
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+    {  // snapshot part: per state x of the list, the A operand
+       // A_x[t] = fp16(lambda_{t, L_t(x)} (s_x / s_ref) q~_t) into TMEM slot
+       // x % 2; the MMAs add A_x (S_x / s_x)^T to O
+      const unsigned char* tab_t = sm.tab + (kBig ? 0 : evt_t * kMaxC);
+      // lambda of state x for this row (0 past the interval's end).  With most
+      // of the shared memory taken, L1 does not hold the rows of lambda, so
+      // the loads are issued two states ahead of their use.
+      auto lam_raw = [&](int x) -> float {
+        if (x >= m0 || t >= Lc) return 0.f;
+        return lam_t ? lam_at(kBig ? x : (int)tab_t[x]) : 1.f;
       };
-      float wn = weight(0);
-      for (int x = 0; ok && x < nu; ++x) {
-        const int n = x + 2, buf = n % NBUF, kb = n / NBUF;
-        const bool in = side_in && ux[x] >= 0;  // warp-uniform
-        const float wx = wn;
-        wn = weight(x + 1);
-        // tcgen05.ld below is warp-wide: the warp takes one decision
-        if (!(ok = __all_sync(0xffffffffu, mbar_wait(&sm.acc_full[buf], (uint32_t)(kb & 1), abort, status)))) break;
+      float l0 = lam_raw(0), l1 = lam_raw(1);
+      for (int x = 0; ok && x < m0; ++x) {
+        const int j = x & 1;
+        const float wx = l0 * (sm.uscale[x] * rsref);
+        l0 = l1;
+        l1 = lam_raw(x + 2);
+        // slot j is free once the MMAs of state x - 2 are complete (the commit
+        // on its tile's stage, unit x + 1), and state x's tile must have landed
+        bool w_ok = true;
+        if (x >= 2) w_ok = mbar_wait(&sm.empty[(x + 1) % NHS], (uint32_t)(((x + 1) / NHS) & 1), abort, status);
+        w_ok = w_ok && mbar_wait(&sm.full[(3 + x) % NHS], (uint32_t)(((3 + x) / NHS) & 1), abort, status);
+        if (!(ok = __all_sync(0xffffffffu, w_ok))) break;
         tc_fence_after();
-        if (in) {
-          float dv[16];
-          const uint32_t base = lane_addr + 256u * buf + 128u * side + 64 * ch;
+        const uint32_t abase = lane_addr + 64u * j + 32u * ch;
+        const __half2 w2 = __float2half2_rn(wx);
 #pragma unroll
-          for (int c = 0; c < 64; c += 16) {
-            tmem_ld16(base + c, dv);
+        for (int cc = 0; cc < 2; ++cc) {
+          float hv[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) o[c + i] += wx * dv[i];
+          for (int i = 0; i < 16; ++i) {
+            const __half2 hh = __hmul2(*reinterpret_cast<const __half2*>(&qh[16 * cc + i]), w2);
+            hv[i] = __uint_as_float(*reinterpret_cast<const uint32_t*>(&hh));
           }
+          tmem_st16(abase + 16u * cc, hv);
         }
+        tmem_st_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.acc_empty[buf]);
+        if (lane == 0) mbar_arrive(&sm.ready[j]);
       }
     }
-    // fp32 output of the common instance: staged in the ring stages (free once
-    // every state product is complete, which this warp has seen) in the
-    // 128-byte swizzle and stored by TMA, eight 128-row x 32-column tiles per
-    // CTA (rows past T are clipped); otherwise per-row stores
+    // o = the accumulator times qinv s_ref, once every MMA is complete
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&sm.bar_done, 0, abort, status));
+    if (ok) tc_fence_after();
+    const uint32_t obase = lane_addr + kColO + 64 * ch;
+    const float f = qinv * sref;
+    // fp32 output of the common instance: staged in stages 0 and 1 (free once
+    // every MMA is complete, which this warp has seen) in the 128-byte swizzle
+    // and stored by TMA, four 128-row x 32-column tiles (rows past T are
+    // clipped); otherwise per-row stores
     bool tma_out = false;
     if constexpr (!kStream && !kRagged) tma_out = (a.out_bf16 == 0);
     if (tma_out) {
-      if (ok && side_in) {
-#pragma unroll
+      if (ok) {
+#pragma unroll 1
         for (int cbl = 0; cbl < 2; ++cbl) {
-          const int box = side * 4 + 2 * ch + cbl;
+          float v[32];
+          tmem_ld32(obase + 32 * cbl, v);
+          const int box = 2 * ch + cbl;
           uint8_t* tile = sm.hs[box >> 1][box & 1];
 #pragma unroll
           for (int c = 0; c < 8; ++c)
             *reinterpret_cast<float4*>(tile + t * 128 + ((c ^ (t & 7)) << 4)) =
-                make_float4(o[32 * cbl + 4 * c], o[32 * cbl + 4 * c + 1], o[32 * cbl + 4 * c + 2], o[32 * cbl + 4 * c + 3]);
+                make_float4(v[4 * c] * f, v[4 * c + 1] * f, v[4 * c + 2] * f, v[4 * c + 3] * f);
         }
       }
       fence_proxy_async();  // the staged output feeds the TMA engine
-      asm volatile("bar.sync 1, 512;" ::: "memory");
+      asm volatile("bar.sync 1, 256;" ::: "memory");
       if (ew == 0 && lane == 0 && !*abort) {
-        for (int box = 0; box < (hasB ? 8 : 4); ++box)
-          tma_store_4d(&tmO, sm.hs[box >> 1][box & 1], 32 * (box & 3), h, tma_t + c0_of(box >> 2), tma_b);
+        for (int box = 0; box < 4; ++box) tma_store_4d(&tmO, sm.hs[box >> 1][box & 1], 32 * box, h, tma_t + c0, tma_b);
         bulk_commit();
-        bulk_wait0();  // the CTA's shared memory stays valid until the stores are done
+        bulk_wait_read0();  // the CTA's shared memory stays valid until the stores have read it
       }
-    } else if (ok && !*abort && side_in && t < Lcs) {
+    } else if (ok && !*abort) {  // warp-uniform: the TMEM loads are warp-wide
+      float o[64];
+      tmem_ld32x2(obase, obase + 32, o);
+#pragma unroll
+      for (int i = 0; i < 64; ++i) o[i] *= f;
       const long long orow = (rowbase + (long long)t * a.H) * D + 64 * ch;
-      if (a.out_bf16) {
+      if (t >= Lc) {
+      } else if (a.out_bf16) {
         __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.o) + orow;
 #pragma unroll
         for (int i = 0; i < 64; i += 4) store4(out + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]));
@@ -689,12 +612,7 @@ __global__ void __launch_bounds__(NT, 1)
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
   // every CTA reaches this point, also after a failed wait: the host's copy of
   // the output piece waits for the count of its CTAs
-  if constexpr (kStream) {
-    if (a.out_done && tid == 0) {
-      __threadfence();
-      atomicAdd(a.out_done + pair / a.out_piece_pairs, 1);
-    }
-  }
+  count_done(true);
 }
 
 // ---------------------------------------------------------------- host side
@@ -718,8 +636,11 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
                            : (ragged ? readout_tc_kernel<false, true> : readout_tc_kernel<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  if ((a.nsnap + 1) / 2 > 65535) return cudaErrorInvalidConfiguration;
-  dim3 grid(a.B * a.H, (a.nsnap + 1) / 2);  // streams x pairs of intervals
+  // two CTAs per SM: the whole shared-memory carve-out
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  if (e != cudaSuccess) return e;
+  if (a.nsnap > 65535) return cudaErrorInvalidConfiguration;
+  dim3 grid(a.B * a.H, a.nsnap);  // streams x intervals
   // the common instance stores an fp32 output by TMA (the map is unused otherwise)
   if (!stream && !ragged && !a.out_bf16) {
     if (!tmap_out_f32(&mo, a.o, a.B, a.T, a.H)) return cudaErrorInvalidValue;
@@ -730,7 +651,7 @@ cudaError_t launch_readout_tc(const ReadoutArgs& a, int32_t* status, cudaStream_
   return cudaGetLastError();
 }
 
-size_t readout_tc_smem_bytes() { return sizeof(TcSmem<kMaxCBig>) + 1024; }
+size_t readout_tc_smem_bytes() { return sizeof(TcSmem<kMaxC>) + 1024; }
 
 cudaError_t preload_readout_kernels() {
   cudaFuncAttributes fa;
