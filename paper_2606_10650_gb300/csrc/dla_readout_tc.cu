@@ -92,6 +92,7 @@ struct TcSmem {
   float sref;                  // the largest s_x of the list (1 if empty)
   uint64_t full[NHS], empty[NHS];
   uint64_t bar_p, bar_pt, bar_done;
+  uint64_t qfree;              // the epilogue holds Q in registers: stage 0 may take state 0
   uint64_t ready[2];           // state x: its A operand in slot x % 2 and its tile landed
   uint32_t tmem_base;
   int abort_flag;
@@ -256,6 +257,7 @@ __global__ void __launch_bounds__(NT, 2)
       mbar_init(&sm.empty[i], 1);
     }
     for (int j = 0; j < 2; ++j) mbar_init(&sm.ready[j], NEPI);
+    mbar_init(&sm.qfree, NEPI);
     sm.abort_flag = 0;
     fence_mbar_init();
     prefetch_tmap(&tmQ);
@@ -314,7 +316,10 @@ __global__ void __launch_bounds__(NT, 2)
       for (int i = 0; i < NHS; ++i) issued[i] = 1;
       for (int x = 0; x < m0; ++x) {
         const int g = 3 + x, hsi = g % NHS, k = g / NHS;
-        if (!mbar_wait(&sm.empty[hsi], (uint32_t)((k & 1) ^ 1), abort, status)) break;
+        // state 0 takes Q's stage as soon as P is complete and the epilogue holds
+        // Q in registers; later states wait for the MMAs of the stage's last use
+        if (!mbar_wait(x == 0 ? &sm.qfree : &sm.empty[hsi], x == 0 ? 0u : (uint32_t)((k & 1) ^ 1), abort, status))
+          break;
         mbar_expect_tx(&sm.full[hsi], 2 * kTile);
         const int row = (int)(((long long)bh * a.pool_cap + sm.ids[x]) * D);
         tma_load_2d(sm.hs[hsi][0], &tmS, &sm.full[hsi], 0, row);
@@ -444,6 +449,8 @@ __global__ void __launch_bounds__(NT, 2)
         }
       }
       sm.qmax[ch][t] = mx;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.qfree);  // this warp's reads of the Q tile are done
       asm volatile("bar.sync 1, 256;" ::: "memory");
       const float rm = fmaxf(sm.qmax[0][t], sm.qmax[1][t]);
       int ex = 0;
@@ -460,7 +467,14 @@ __global__ void __launch_bounds__(NT, 2)
     }
     {  // P -> Pt over the K tile, in the accumulator's units: row t scaled by
        // 2^(14 - ex) / s_ref (a power of two, so no extra rounding)
-      if (ok) {
+      // a warp whose rows all lie before its 64 columns (rows 0..63, columns
+      // 64..127) writes zeros without reading P
+      const bool upper = (ch == 1) && (quad < 2);  // warp-uniform
+      if (ok && upper) {
+        uint8_t* ptile = sm.hs[1][ch];
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) *reinterpret_cast<uint4*>(ptile + t * 128 + (c8 << 4)) = make_uint4(0u, 0u, 0u, 0u);
+      } else if (ok) {
         tc_fence_after();
         const uint32_t base = lane_addr + 64 * ch;
         // the weight of column s depends on s only through evt[s], which changes
