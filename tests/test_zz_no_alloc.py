@@ -76,6 +76,45 @@ def test_noalloc_with_a_plan_limited_by_its_scratch():
     assert torch.equal(c["m"], c_ref["m"]) and torch.equal(c["n"], c_ref["n"])
 
 
+def test_noalloc_replayed_from_a_captured_graph():
+    """dla_forward_noalloc captured in a CUDA graph (after a first call on the
+    thread, which creates the library's internal streams and events), then the
+    graph replayed on other inputs copied into the captured buffers: trace,
+    cache and outputs equal dla_forward's on those inputs, and the capture
+    stream's status word reads 0."""
+    dev = torch.device("cuda:0")
+    w, t1 = _inputs(21, dev)
+    _, t2 = _inputs(22, dev)
+    q, k, v, lam = (x.clone() for x in t1)
+    B, T, H, d = k.shape
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    cache = dla.Cache(B, H, w.C, d, device=dev)
+    o = torch.full((B, T, H, d), float("nan"), device=dev)
+    bnd = torch.zeros((B, H, T), dtype=torch.uint8, device=dev)
+    ml = torch.zeros((B, H, T), dtype=torch.int32, device=dev)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        dla.dla_forward_noalloc(p, q, k, v, lam, o, cache, bnd, ml, stream=s)
+    assert dla.dla_sync_status(s) == 0
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        dla.dla_forward_noalloc(p, q, k, v, lam, o, cache, bnd, ml, stream=s)
+    for dst, src in zip((q, k, v, lam), t2):
+        dst.copy_(src)
+    o.fill_(float("nan"))
+    torch.cuda.synchronize()
+    g.replay()
+    torch.cuda.synchronize()
+    assert dla.dla_sync_status(s) == 0
+    o_ref, b_ref, m_ref, c_ref = _run("workspace", w, t2, dev)
+    assert torch.equal(bnd.cpu(), b_ref) and torch.equal(ml.cpu(), m_ref)
+    assert torch.isfinite(o).all()
+    assert (o.cpu() - o_ref).abs().max().item() <= TOL[w.dtype]
+    c = cache.export()
+    assert torch.equal(c["m"], c_ref["m"]) and torch.equal(c["n"], c_ref["n"])
+
+
 def test_noalloc_rejects_calls_beyond_its_scratch():
     """Without a caller cache the cache itself must live in the scratch; for a
     large batch that exceeds the 64 MiB limit and the call is refused with a
