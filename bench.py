@@ -18,6 +18,7 @@ path).  ``--impl reference`` times the oracle instead (the reference arm).
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import math
 import os
@@ -81,9 +82,12 @@ class Dist:
 
 
 class Clocks:
-    """nvidia-smi sampling (200 ms) around a timed region."""
+    """nvidia-smi sampling (every 50 ms) around a timed region and the untimed
+    steps of the same work run just before it (a timed region of a few tens of
+    ms holds one sample at most); samples whose timestamp falls inside the
+    timed region are also counted apart."""
 
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -91,13 +95,17 @@ class Clocks:
         self.index = index
         self.proc = None
         self.path = None
+        self.region = None  # wall-clock (start, end) of the timed region
+
+    def mark(self, t0, t1):
+        self.region = (t0, t1)
 
     def start(self):
         try:
             fd, self.path = tempfile.mkstemp(prefix="dla_clocks_", suffix=".csv")
             os.close(fd)
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -111,13 +119,19 @@ class Clocks:
             self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-        rows = []
         with open(self.path) as f:
-            for line in f:
-                parts = [p.strip() for p in line.split(",")]
-                if len(parts) >= 10:
-                    rows.append(parts)
+            lines = f.readlines()
         os.unlink(self.path)
+        return self.summarize(lines, self.region)
+
+    @staticmethod
+    def summarize(lines, region=None):
+        """The clock record of nvidia-smi CSV lines (the fields of Q)."""
+        rows = []
+        for line in lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 11:
+                rows.append(parts)
         if not rows:
             return None
 
@@ -127,13 +141,25 @@ class Clocks:
             except ValueError:
                 return float("nan")
 
-        loaded = [r for r in rows if num(r[4]) > 0] or rows
-        sm = [num(r[1]) for r in loaded]
+        def stamp(x):  # nvidia-smi's local time, e.g. 2026/12/02 15:01:16.123
+            try:
+                return datetime.datetime.strptime(x, "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            except ValueError:
+                return None
+
+        loaded = [r for r in rows if num(r[5]) > 0] or rows
+        sm = [num(r[2]) for r in loaded]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in loaded for i in range(4) if r[6 + i].lower().startswith("active")})
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(num(r[2]) for r in rows),
-                "power_w_max": max(num(r[3]) for r in rows), "samples": len(rows), "samples_under_load": len(loaded),
-                "reasons": reasons}
+        reasons = sorted({names[i] for r in loaded for i in range(4) if r[7 + i].lower().startswith("active")})
+        rec = {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(num(r[3]) for r in rows),
+               "power_w_max": max(num(r[4]) for r in rows), "samples": len(rows), "samples_under_load": len(loaded),
+               "reasons": reasons, "interval_ms": 50}
+        if region is not None:
+            inside = [r for r in rows if (stamp(r[0]) or -1.0) >= region[0] - 0.05 and (stamp(r[0]) or -1.0) <= region[1] + 0.05]
+            rec["samples_in_timed_region"] = len(inside)
+            if inside:
+                rec["sm_mhz_in_timed_region"] = statistics.median(num(r[2]) for r in inside)
+        return rec
 
 
 def kernel_table(timing, steps):
@@ -293,19 +319,34 @@ def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headli
     dla.dla_timing_read(reset=True)
     clocks = Clocks(dist.local) if headline else None
     if clocks:
+        # the clock record: sampled through 0.5 s of the same steps, untimed,
+        # right before the timed region, and through the timed region itself
         clocks.start()
+        t_soak = time.time() + 0.5
+        n_soak = 0
+        while time.time() < t_soak:
+            step()
+            n_soak += 1
+            if n_soak % 16 == 0:
+                torch.cuda.synchronize()
     dist.barrier()
     torch.cuda.synchronize()
     dla.dla_timing_enable(True)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
     e0.record(stream)
     for _ in range(steps):
         step()
     e1.record(stream)
     torch.cuda.synchronize()
+    w1 = time.time()
     dla.dla_timing_enable(False)
     dist.barrier()
+    if clocks:
+        clocks.mark(w0, w1)
     clk = clocks.stop() if clocks else None
+    if clk is not None:
+        clk["untimed_steps_before"] = n_soak
     ms = e0.elapsed_time(e1) / steps
     timing = dla.dla_timing_read(reset=True)
     check_status("the timed steps")

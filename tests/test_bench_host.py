@@ -76,3 +76,28 @@ def test_committed_traffic_table_is_well_formed():
             continue
         assert set(rec) >= {"source", "sha256_prefix", "workload", "bytes_per_launch", "summary"}
         assert os.path.exists(os.path.join(ROOT, rec["source"])) and os.path.exists(os.path.join(ROOT, rec["summary"]))
+
+
+def test_clock_record_counts_the_timed_region_apart():
+    """The clock summary of nvidia-smi lines: the median SM clock under load,
+    throttle reasons that were active, and the samples whose timestamps fall
+    inside the timed region (with a 50 ms margin) counted apart."""
+    import datetime
+    import time
+
+    sys.path.insert(0, ROOT)
+    import bench
+    now = time.time()
+
+    def line(dt, sm, util, thermal="Not Active"):
+        ts = datetime.datetime.fromtimestamp(now + dt).strftime("%Y/%m/%d %H:%M:%S.%f")[:-3]
+        return f"{ts}, 0, {sm}, 2070, 190.5, {util}, 0x0, Not Active, {thermal}, Not Active, Not Active\n"
+
+    lines = [line(-0.40, 1980, 99), line(-0.20, 2070, 99), line(0.01, 2070, 99), line(0.30, 300, 0)]
+    rec = bench.Clocks.summarize(lines, (now, now + 0.03))
+    assert rec["samples"] == 4 and rec["samples_under_load"] == 3
+    assert rec["sm_mhz"] == 2070.0 and rec["reasons"] == []
+    assert rec["samples_in_timed_region"] == 1 and rec["sm_mhz_in_timed_region"] == 2070.0
+    rec = bench.Clocks.summarize(lines + [line(0.02, 1500, 99, thermal="Active")], (now, now + 0.03))
+    assert rec["reasons"] == ["hw_thermal_slowdown"] and rec["samples_in_timed_region"] == 2
+    assert bench.Clocks.summarize(["garbage\n"]) is None
