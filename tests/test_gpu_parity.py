@@ -109,6 +109,20 @@ def test_edge_lengths(T):
     assert g["boundary"][0, 0, 0] == 1
 
 
+@pytest.mark.parametrize("T", [1, 2, 127, 128, 129, 255, 383])
+def test_edge_lengths_tensor_core_path(T):
+    """bf16, d = 128 (the scan on CTA pairs, the tensor-core read-out): a
+    single token, one interval exactly, one token past it, odd interval counts
+    and a ragged last interval, whose output rows past T the read-out's TMA
+    store must clip."""
+    w = W.get("regime", B=1, H=2, T=T, C=8, tau=1.2)
+    q, k, v, lam = _safe(w)
+    g = run_gpu(w, q, k, v, lam)
+    r = run_oracle(w, q, k, v, lam)
+    compare(w, g, r)
+    assert g["boundary"][0, 0, 0] == 1
+
+
 def test_many_rounds_small_workspace():
     """The smallest workspace forces one read-out interval per round; the
     result must not change."""
