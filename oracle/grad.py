@@ -86,3 +86,51 @@ def readout_grads(q, k, v, lam, boundary, merge_log, g):
         for t in range(T):
             np.add.at(dlam[t], slot[t, : t + 1], P[t, : t + 1])
     return dict(dq=dq, dk=dk, dv=dv, dlam=dlam)
+
+
+def readout_grads_sampled(q, k, v, lam, boundary, merge_log, g, rows, cols):
+    """The gradients of readout_grads at sampled tokens only, for sequences
+    too long for the T x T weight matrix: dq and dlambda at the tokens `rows`,
+    dk and dv at the tokens `cols`.  The same replay of Algorithm 2's decisions
+    on token ranges, evaluated one row (all s <= t) or one column (all t >= s)
+    of the dense form at a time.  Returns dict(rows, cols, dq, dlam, dk, dv)."""
+    q, k, v, g = (np.asarray(x, dtype=np.float64) for x in (q, k, v, g))
+    boundary = np.asarray(boundary)
+    merge_log = np.asarray(merge_log)
+    lam = None if lam is None else np.asarray(lam, dtype=np.float64)
+    T, d = k.shape
+    rows = sorted(int(t) for t in rows)
+    cols = sorted(int(s) for s in cols)
+    row_set = set(rows)
+    dq = np.zeros((len(rows), d))
+    dlam = None if lam is None else np.zeros((len(rows), lam.shape[1]))
+    col_slot = np.full((len(cols), T), -1, dtype=np.int64)  # slot_t(s) of every sampled column s
+    cols_arr = np.asarray(cols, dtype=np.int64)
+    firsts = []
+    for t in range(T):
+        if boundary[t] or not firsts:
+            j = int(merge_log[t])
+            if j >= 0:
+                del firsts[j + 1]
+            firsts.append(t)
+        fa = np.asarray(firsts)
+        live = cols_arr <= t
+        if live.any():
+            col_slot[live, t] = np.searchsorted(fa, cols_arr[live], side="right") - 1
+        if t in row_set:
+            r = rows.index(t)
+            sl = np.searchsorted(fa, np.arange(t + 1), side="right") - 1
+            w = np.ones(t + 1) if lam is None else lam[t, sl]
+            bg = v[: t + 1] @ g[t]   # (g_t . v_s)
+            a = k[: t + 1] @ q[t]    # (q_t . k_s)
+            dq[r] = (bg * w) @ k[: t + 1]
+            if lam is not None:
+                np.add.at(dlam[r], sl, a * bg)
+    dk = np.zeros((len(cols), d))
+    dv = np.zeros((len(cols), d))
+    for c, s in enumerate(cols):
+        ts = np.arange(s, T)
+        w = np.ones(T - s) if lam is None else lam[ts, col_slot[c, s:]]
+        dk[c] = ((g[s:] @ v[s]) * w) @ q[s:]
+        dv[c] = ((q[s:] @ k[s]) * w) @ g[s:]
+    return dict(rows=rows, cols=cols, dq=dq, dlam=dlam, dk=dk, dv=dv)

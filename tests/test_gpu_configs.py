@@ -121,3 +121,42 @@ def test_decode_workload_full_capacity():
     full = (m0 == w.C).numpy()
     assert (m_all[full] >= 0).sum() > 0, "merges must happen on full C = 64 caches"
     print("decode C=64: boundaries", int(b_all.sum()), "merges", int((m_all >= 0).sum()), "worst o", worst)
+
+
+@pytest.mark.timeout(900)
+def test_regime_backward_full_shape_sampled():
+    """dla_backward at the regime workload's full shape (B2 H16 T16384 d128
+    C32, the shape bench.py times) on the oracle's decision trace of the same
+    inputs: dq and dlambda at sampled tokens and dk and dv at sampled tokens of
+    four streams, against the fp64 gradient oracle evaluated row by row and
+    column by column (oracle/grad.py readout_grads_sampled), within 1e-4 of
+    the largest gradient of each kind."""
+    from oracle import grad as G
+    w = W.get("regime")
+    key = ("regime", 1)
+    if key not in _ORACLE_CACHE:
+        _ORACLE_CACHE[key] = safe_oracle_streams(w, T=w.T, want_o=None)
+    (q, k, v, lam), r = _ORACLE_CACHE[key]
+    dev = torch.device("cuda:0")
+    qt, kt, vt, lt = upload(w, q, k, v, lam)
+    gen = torch.Generator().manual_seed(29)
+    g = torch.randn((w.B, w.T, w.H, w.d), generator=gen, dtype=torch.float32)
+    bt = torch.from_numpy(np.ascontiguousarray(r["boundary"], dtype=np.uint8)).to(dev)
+    mt = torch.from_numpy(np.ascontiguousarray(r["merge_log"], dtype=np.int32)).to(dev)
+    out = dla.backward(qt, kt, vt, lt, bt, mt, g.to(dev), capacity=w.C)
+    assert dla.dla_sync_status() == 0
+    rows = [0, 1, 127, 128, 4095, 8191, 12000, w.T - 1]
+    cols = [0, 5, 128, 4096, 10000, w.T - 2, w.T - 1]
+    rep = {}
+    for b, h in [(0, 0), (0, 7), (1, 3), (1, 15)]:
+        s = G.readout_grads_sampled(q[b, :, h], k[b, :, h], v[b, :, h], lam[b, :, h], r["boundary"][b, h],
+                                    r["merge_log"][b, h], g[b, :, h].double().numpy(), rows, cols)
+        got = {"dq": out["dq"][b, rows, h], "dlam": out["dlam"][b, rows, h],
+               "dk": out["dk"][b, cols, h], "dv": out["dv"][b, cols, h]}
+        for key_ in ("dq", "dlam", "dk", "dv"):
+            ref = s[key_]
+            err = float(np.abs(got[key_].double().cpu().numpy() - ref).max())
+            scale = max(1.0, float(np.abs(ref).max()))
+            rep[(b, h, key_)] = (err, err / scale)
+            assert err <= 1e-4 * scale, (b, h, key_, err, scale)
+    print("backward, full shape, sampled tokens:", {k_: f"{v_[1]:.2e}" for k_, v_ in rep.items()})

@@ -85,3 +85,26 @@ def test_gradients_match_central_differences(seed):
             assert fd == pytest.approx(gr[key][idx], rel=1e-6, abs=1e-8), (name, idx)
             checked += 1
     assert checked >= 0.9 * (q.size + k.size + v.size + lam.size)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+@pytest.mark.parametrize("with_lam", [True, False])
+def test_sampled_gradients_equal_the_dense_ones(seed, with_lam):
+    """The row / column evaluation for long sequences (readout_grads_sampled)
+    equals the dense gradients at every sampled token, with and without
+    lambda, on streams with merges."""
+    q, k, v, lam, tau, g = _stream(seed, T=40)
+    lam_use = lam if with_lam else None
+    _, bnd, ml, _ = _run(q, k, v, lam, tau, 3)
+    assert (ml >= 0).sum() > 3
+    full = grad.readout_grads(q, k, v, lam_use, bnd, ml, g)
+    rows = [0, 1, 7, 20, 39]
+    cols = [0, 5, 19, 38, 39]
+    s = grad.readout_grads_sampled(q, k, v, lam_use, bnd, ml, g, rows, cols)
+    np.testing.assert_allclose(s["dq"], full["dq"][rows], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(s["dk"], full["dk"][cols], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(s["dv"], full["dv"][cols], rtol=1e-12, atol=1e-12)
+    if with_lam:
+        np.testing.assert_allclose(s["dlam"], full["dlam"][rows], rtol=1e-12, atol=1e-12)
+    else:
+        assert s["dlam"] is None
