@@ -160,3 +160,26 @@ def test_regime_backward_full_shape_sampled():
             rep[(b, h, key_)] = (err, err / scale)
             assert err <= 1e-4 * scale, (b, h, key_, err, scale)
     print("backward, full shape, sampled tokens:", {k_: f"{v_[1]:.2e}" for k_, v_ in rep.items()})
+
+
+@pytest.mark.timeout(1200)
+def test_regime_dla_i_full_shape():
+    """DLA(I) (Table 5: dynamic merging without the capacity bound) at the
+    regime workload's full shape: all 32 streams of 16384 tokens with C = 128,
+    above every stream's segment count, on the kernel instances for capacities
+    above 64 (metadata in shared memory, no capacity merge).  Nothing merges;
+    decisions and caches equal the oracle's bit for bit, outputs on every 16th
+    token within the bf16 tolerance."""
+    w = W.get("regime", C=128)
+    want = np.zeros(w.T, bool)
+    want[::16] = True
+    want[-1] = True
+    (q, k, v, lam), r = safe_oracle_streams(w, T=w.T, want_o=want)
+    g = run_gpu(w, q, k, v, lam)
+    rep = {}
+    compare(w, g, r, report=rep)
+    structural_checks(w, g, w.T)
+    assert (g["merge_log"] == -1).all()
+    m = g["cache"].export()["m"]
+    assert int(m.max()) > 64
+    print("DLA(I) full shape: segments per stream", int(m.min()), "-", int(m.max()), rep)
