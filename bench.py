@@ -731,7 +731,10 @@ def main():
     ap.add_argument("--decode-batch", type=int, default=0)
     ap.add_argument("--ws-gb", type=float, default=0.0, help="cap the prefill workspace (GiB)")
     ap.add_argument("--cpu-tokens", type=int, default=8192)
-    ap.add_argument("--ref-tokens", type=int, default=512)
+    # the reference arm's sample per step: the same as cpu_baseline's (first 8192
+    # tokens of batch row 0, all heads, about 2 s on 16 host cores), so that the
+    # two oracle rates describe one sample
+    ap.add_argument("--ref-tokens", type=int, default=8192)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 0)
     dist = Dist()
