@@ -134,3 +134,78 @@ def readout_grads_sampled(q, k, v, lam, boundary, merge_log, g, rows, cols):
         dk[c] = ((g[s:] @ v[s]) * w) @ q[s:]
         dv[c] = ((q[s:] @ k[s]) * w) @ g[s:]
     return dict(rows=rows, cols=cols, dq=dq, dlam=dlam, dk=dk, dv=dv)
+
+
+def readout_grads_linear(q, k, v, lam, boundary, merge_log, g):
+    """The gradients of readout_grads in time linear in T: two sweeps over the
+    tokens with the cache's states, never the T x T weights.
+
+    Forward sweep (the states S_i of Sec. 2, built as the forward pass builds
+    them): dq_t = sum_i lambda_{t,i} S_i^T g_t and dlambda_{t,i} = g_t . (S_i q_t)
+    over the cache after token t.
+
+    Reverse sweep (adjoint states): token s receives, from every later token t
+    whose state list holds s in slot i, the term lambda_{t,i} g_t q_t^T, so
+    dv_s = M(s) k_s and dk_s = M(s)^T v_s with M(s) = sum_{t >= s}
+    lambda_{t, slot_t(s)} g_t q_t^T.  Walking t from T - 1 down to 0 with one
+    d x d matrix A_i per state of the cache after token t: every A_i takes
+    lambda_{t,i} g_t q_t^T; token t, which lies in the newest state, reads
+    M(t) = A_newest; then token t's events are undone in reverse order (the
+    state it opened is dropped, a merge it caused is split and both halves keep
+    the merged state's A, since later tokens saw them as one).
+    Returns dict(dq, dk, dv, dlam) like readout_grads."""
+    q, k, v, g = (np.asarray(x, dtype=np.float64) for x in (q, k, v, g))
+    boundary = np.asarray(boundary)
+    merge_log = np.asarray(merge_log)
+    lamf = None if lam is None else np.asarray(lam, dtype=np.float64)
+    T, d = k.shape
+    dv_ = v.shape[1]
+
+    def lam_at(t, i):
+        return 1.0 if lamf is None else lamf[t, i]
+
+    # forward sweep: states and the events of every token (for the reverse one)
+    states = []   # S_i, [dv, d]
+    firsts = []   # first token of each state
+    events = []   # per token: (opened a state, merge index, first token of the state the merge removed)
+    dq = np.zeros((T, d))
+    dlam = None if lamf is None else np.zeros_like(lamf)
+    for t in range(T):
+        opened = bool(boundary[t]) or not states
+        j, removed_first = -1, -1
+        if opened:
+            j = int(merge_log[t])
+            if j >= 0:  # states j and j + 1 become one
+                states[j] = states[j] + states[j + 1]
+                removed_first = firsts[j + 1]
+                del states[j + 1]
+                del firsts[j + 1]
+            states.append(np.outer(v[t], k[t]))
+            firsts.append(t)
+        else:
+            states[-1] = states[-1] + np.outer(v[t], k[t])
+        events.append((opened, j, removed_first))
+        for i, S in enumerate(states):
+            w = lam_at(t, i)
+            dq[t] += w * (S.T @ g[t])
+            if dlam is not None:
+                dlam[t, i] = g[t] @ (S @ q[t])
+    # reverse sweep: adjoint matrices of the states after token t
+    A = [np.zeros((dv_, d)) for _ in states]
+    dk = np.zeros((T, d))
+    dvv = np.zeros((T, dv_))
+    for t in range(T - 1, -1, -1):
+        gq = np.outer(g[t], q[t])
+        for i in range(len(A)):
+            A[i] += lam_at(t, i) * gq
+        M = A[-1]  # token t lies in the newest state
+        dvv[t] = M @ k[t]
+        dk[t] = M.T @ v[t]
+        opened, j, removed_first = events[t]
+        if opened:
+            A.pop()
+            firsts.pop()
+            if j >= 0:  # undo the merge: both halves keep what later tokens gave the merged state
+                A.insert(j + 1, A[j].copy())
+                firsts.insert(j + 1, removed_first)
+    return dict(dq=dq, dk=dk, dv=dvv, dlam=dlam)

@@ -108,3 +108,21 @@ def test_sampled_gradients_equal_the_dense_ones(seed, with_lam):
         np.testing.assert_allclose(s["dlam"], full["dlam"][rows], rtol=1e-12, atol=1e-12)
     else:
         assert s["dlam"] is None
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+@pytest.mark.parametrize("with_lam", [True, False])
+def test_linear_time_gradients_equal_the_dense_ones(seed, with_lam):
+    """The two-sweep form (forward states for dq and dlambda, reverse adjoint
+    states through the undone merges for dk and dv) equals the dense form on
+    streams with merges, with and without lambda."""
+    q, k, v, lam, tau, g = _stream(seed, T=40)
+    lam_use = lam if with_lam else None
+    _, bnd, ml, _ = _run(q, k, v, lam, tau, 3)
+    assert (ml >= 0).sum() > 3
+    full = grad.readout_grads(q, k, v, lam_use, bnd, ml, g)
+    lin = grad.readout_grads_linear(q, k, v, lam_use, bnd, ml, g)
+    for key in ("dq", "dk", "dv"):
+        np.testing.assert_allclose(lin[key], full[key], rtol=1e-11, atol=1e-11)
+    if with_lam:
+        np.testing.assert_allclose(lin["dlam"], full["dlam"], rtol=1e-11, atol=1e-11)
