@@ -265,6 +265,113 @@ def bench_dla_i(args, dist, pk, capacity=128, steps=5, warmup=3):
             "merges": 0, "gpu_launches": launches}
 
 
+def _time_steps(step, steps, warmup, before=None):
+    """Mean CUDA-event time (ms) of `step` over `steps` calls after `warmup`
+    untimed ones; `before` (untimed) runs ahead of every call; the library's
+    launches inside the timed calls are counted."""
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+
+    for _ in range(warmup):
+        if before:
+            before()
+        step()
+    torch.cuda.synchronize()
+    if dla.dla_sync_status() != 0:
+        raise RuntimeError("device status reports a failure in the warm-up calls")
+    dla.dla_timing_read(reset=True)
+    total = 0.0
+    for _ in range(steps):
+        if before:
+            before()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        dla.dla_timing_enable(True)
+        e0.record()
+        step()
+        e1.record()
+        torch.cuda.synchronize()
+        dla.dla_timing_enable(False)
+        total += e0.elapsed_time(e1)
+    if dla.dla_sync_status() != 0:
+        raise RuntimeError("device status reports a failure in the timed calls")
+    launches = sum(v_[0] for v_ in dla.dla_timing_read(reset=True).values())
+    return total / steps, launches
+
+
+def bench_packed(args, dist, pk, steps=10, warmup=3):
+    """dla_forward_varlen on the headline workload's tokens regrouped as a
+    packed batch of four rows of different lengths (the serving layout,
+    cu_seqlens offsets), each row from an empty cache."""
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+
+    w, qt, kt, vt, lt = _INPUTS[args.workload]
+    B, T, H, d = kt.shape
+    if B != 2 or T % 4:
+        return None
+    cuts = [(0, 0, 3 * T // 4), (0, 3 * T // 4, T), (1, 0, T // 2), (1, T // 2, T)]  # (batch row, t0, t1)
+    lens = [t1 - t0 for _, t0, t1 in cuts]
+    pq, pk_, pv, pl = (torch.cat([x[b, t0:t1] for b, t0, t1 in cuts]).contiguous() for x in (qt, kt, vt, lt))
+    cu = torch.tensor([0] + list(__import__("itertools").accumulate(lens)), dtype=torch.int32, device=kt.device)
+    mx = max(lens)
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps)
+    o = torch.empty_like(pq, dtype=torch.float32)
+    bnd = torch.empty((len(lens), H, mx), dtype=torch.uint8, device=kt.device)
+    ml = torch.empty((len(lens), H, mx), dtype=torch.int32, device=kt.device)
+    cache = dla.Cache(len(lens), H, w.C, d, device=kt.device)
+    ws = dla.dla_forward_varlen(p, cu, mx, pq, pk_, pv, pl, o, cache, bnd, ml)  # sizes the workspace once
+
+    def step():
+        dla.dla_forward_varlen(p, cu, mx, pq, pk_, pv, pl, o, cache, bnd, ml, workspace=ws)
+
+    ms, launches = _time_steps(step, steps, warmup)
+    tokens = sum(lens)
+    return {"workload": f"{w.name} tokens regrouped: {len(lens)} packed rows of {lens} tokens, H={H} d={d} C={w.C}, "
+                        "each row from an empty cache (dla_forward_varlen, cu_seqlens)",
+            "value": round(tokens / ms * 1e3, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4), "steps": steps,
+            "gpu_launches": launches}
+
+
+def bench_continuation(args, dist, pk, steps=10, warmup=3):
+    """Prefill continuation: dla_forward with from_cache = 1 over the second
+    half of the headline workload's rows, on top of the cache the first half
+    left; the cache is restored (untimed) before every call."""
+    import torch
+
+    from paper_2606_10650_gb300 import dla
+
+    w, qt, kt, vt, lt = _INPUTS[args.workload]
+    B, T, H, d = kt.shape
+    half = T // 2
+    q2, k2, v2, l2 = (x[:, half:].contiguous() for x in (qt, kt, vt, lt))
+    cache = dla.Cache(B, H, w.C, d, device=kt.device)
+    dla.forward(qt[:, :half].contiguous(), kt[:, :half].contiguous(), vt[:, :half].contiguous(),
+                lt[:, :half].contiguous(), tau=w.tau, capacity=w.C, eps=w.eps, rms_eps=w.rms_eps, want_o=False,
+                cache=cache)
+    saved = cache.buf.clone()
+    p = dla.make_params(w.tau, w.C, w.eps, w.rms_eps, from_cache=1)
+    o = torch.empty((B, T - half, H, d), dtype=torch.float32, device=kt.device)
+    bnd = torch.empty((B, H, T - half), dtype=torch.uint8, device=kt.device)
+    ml = torch.empty((B, H, T - half), dtype=torch.int32, device=kt.device)
+    nb = dla.dla_forward_workspace(p, B, T - half, H, d, d, dla.DLA_BF16, True)
+    buf = torch.empty(nb + 256, dtype=torch.uint8, device=kt.device)
+    ws = (buf, (buf.data_ptr() + 255) // 256 * 256, nb)
+
+    def restore():
+        cache.buf.copy_(saved)
+
+    def step():
+        dla.dla_forward(p, q2, k2, v2, l2, o, cache, bnd, ml, workspace=ws)
+
+    ms, launches = _time_steps(step, steps, warmup, before=restore)
+    return {"workload": f"{w.name}: B={B} H={H} d={d} C={w.C}, tokens {half}..{T - 1} of every row on top of the "
+                        f"cache of tokens 0..{half - 1} (from_cache = 1; the cache restored, untimed, before each call)",
+            "value": round(B * (T - half) / ms * 1e3, 1), "unit": "tokens/s", "ms_per_step": round(ms, 4),
+            "steps": steps, "gpu_launches": launches}
+
+
 def bench_prefill(args, dist, pk, workload=None, steps=None, warmup=None, headline=True):
     """One workload's prefill: warm-up, `steps` timed dla_forward calls (the
     default concurrent schedule), the call's device status checked, the kernels
@@ -759,7 +866,8 @@ def main():
             others[name]["algorithmic_frac_of_peak"] = round(r["algorithmic_tflops"] / pk["bf16"], 4)
     extra = {}
     if pre and pre["tc_path"] and not args.no_configs and args.workload in _INPUTS:
-        for key, fn in (("backward", bench_backward), ("dla_i", bench_dla_i)):
+        for key, fn in (("backward", bench_backward), ("dla_i", bench_dla_i), ("packed", bench_packed),
+                        ("continuation", bench_continuation)):
             try:
                 extra[key] = fn(args, dist, pk)
             except (RuntimeError, MemoryError) as exc:  # reported in the line; the headline stands
