@@ -265,7 +265,10 @@ size_t dla_forward_host_workspace(const dla_params* p, int B, int T, int H, int 
 
 /* dla_forward with q, k, v, lam and o in HOST memory (same layouts and
  * semantics; the paper has no counterpart: this is the end-to-end call of a
- * caller whose tensors live on the host).  Page-locked host memory
+ * caller whose tensors live on the host).  Whole rows only: p->seq_lens must
+ * be NULL (DLA_ERR_UNSUPPORTED otherwise; ragged rows take dla_forward with
+ * device-resident inputs, since the copies move whole rows and the o rows
+ * past a row's length could not stay unwritten).  Page-locked host memory
  * (cudaHostAlloc / cudaHostRegister) makes the copies asynchronous; with
  * pageable memory they still work but do not overlap anything.
  *   cache, boundary, merge_log: device memory, as in dla_forward.

@@ -678,6 +678,9 @@ static dla_status forward_launch(const dla_params* p, dla_dtype in_dtype, int B,
     if (vl->total * H * d >= (1LL << 40)) return fail(DLA_ERR_UNSUPPORTED, "tensor too large");
     if (io) return fail(DLA_ERR_UNSUPPORTED, "packed batches take device-resident inputs");
   }
+  // the host copies move whole rows, so the o rows past a row's length could not
+  // stay unwritten, as seq_lens promises
+  if (io && p->seq_lens) return fail(DLA_ERR_UNSUPPORTED, "per-row lengths (seq_lens) take device-resident inputs");
   if (!k || !v) return fail(DLA_ERR_INVALID_ARG, "k and v must be non-NULL");
   const bool with_output = (o != nullptr);
   if (with_output && !q) return fail(DLA_ERR_INVALID_ARG, "q must be non-NULL when o is requested");

@@ -97,6 +97,12 @@ def test_host_buffer_entry_point_errors_and_workspace(L):
     assert fh(ws=False) == 3
     assert fh(ws_bytes=1024) == 3
     assert b"workspace" in L.dla_last_error()
+    # per-row lengths take device-resident inputs (the host copies move whole rows)
+    q = dla.make_params(0.6, 32)
+    q.seq_lens = 1 << 20
+    st = L.dla_forward_host(ctypes.byref(q), 0, 1, 64, 2, 128, 128, _fake(), _fake(), _fake(), None, _fake(), None,
+                            None, None, _fake(1 << 24), 1 << 40, None)
+    assert st == 2 and b"seq_lens" in L.dla_last_error()
 
 
 def test_params_layout_and_seq_lens_checks(L):

@@ -354,6 +354,12 @@ def test_ragged_rows(case, sched, monkeypatch):
     torch.cuda.synchronize()
     assert dla.workspace_status(ws) == 0, "device status word reports a failure"
     g = dict(o=o.double().cpu().numpy(), boundary=bnd.cpu().numpy(), merge_log=ml.cpu().numpy(), cache=cache)
+    _check_ragged(w, q, k, v, lam, lens, g, cache)
+
+
+def _check_ragged(w, q, k, v, lam, lens, g, cache):
+    """Each row against the oracle on its own tokens; padding untouched."""
+    B, T, H, d = k.shape
     r = dict(o=np.full((B, T, H, d), np.nan), boundary=np.zeros((B, H, T), np.uint8),
              merge_log=np.full((B, H, T), -1, np.int32), caches={})
     live = []
